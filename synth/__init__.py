@@ -1,0 +1,246 @@
+"""Seeded synthetic inputs for the crop + replay path.
+
+This module only draws random numbers and lays out the five workload shapes;
+it holds none of the method's arithmetic (no attention, no paging policy).
+Tests, the benchmark and the smoke check import it to feed the CUDA library and
+the fp64 oracle the very same bf16 bit patterns.
+
+Values are drawn with numpy's PCG64 generator (``SeedSequence([base, stream,
+index])``) as float32 standard normals, multiplied by the workload's standard
+deviation in float32 and rounded once to bf16 (round-to-nearest-even).  Every
+independent quantity has its own stream so that, e.g., the counterfactual
+suffix of an agent never shares draws with its original ("contaminated")
+suffix.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+BASE_SEED = 2609_04875
+
+# Stream identifiers: one independent generator per quantity.
+STREAM_PERM = 1          # physical page pop order of the pool
+STREAM_KV_ORIG = 2       # K/V of the original session, positions [0, T)
+STREAM_KV_CF = 3         # K'/V' of the counterfactual (sanitized) suffix
+STREAM_Q_CF = 4          # Q' of the counterfactual suffix
+STREAM_Q_PREFIX = 5      # Q of the prefix positions (full-reset comparator)
+STREAM_LENGTHS = 6       # per-agent T and tau/T (agent batch)
+STREAM_SAMPLE = 7        # query rows sampled for large-size checks
+
+
+def rng(seed: int, stream: int, index: int = 0) -> np.random.Generator:
+    """Independent generator for (seed, stream, index)."""
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, stream, index])))
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to bf16 (nearest, ties to even); returns uint16 bits."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    if not np.all(np.isfinite(x)):
+        raise ValueError("non-finite value in synthetic draw")
+    u = x.view(np.uint32).astype(np.uint64)
+    r = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return r.astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    """Exact widening of bf16 bit patterns to float32 (for host-side inspection)."""
+    return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def normal_bf16(g: np.random.Generator, shape, std: float = 1.0, chunk: int = 1 << 24) -> np.ndarray:
+    """i.i.d. N(0, std^2) draws rounded to bf16, as uint16 bits of the given shape."""
+    shape = tuple(int(s) for s in shape)
+    n = int(np.prod(shape)) if shape else 1
+    out = np.empty(n, dtype=np.uint16)
+    s32 = np.float32(std)
+    for lo in range(0, n, chunk):
+        hi = min(n, lo + chunk)
+        x = g.standard_normal(hi - lo, dtype=np.float32)
+        if std != 1.0:
+            x = x * s32
+        out[lo:hi] = f32_to_bf16_bits(x)
+    return out.reshape(shape)
+
+
+def page_permutation(seed: int, num_pages: int) -> np.ndarray:
+    """A seeded permutation of [0, num_pages): the pool's initial pop order."""
+    return rng(seed, STREAM_PERM).permutation(num_pages).astype(np.int32)
+
+
+def bits_to_torch(bits: np.ndarray):
+    """View uint16 bf16 bits as a torch.bfloat16 CPU tensor (no copy)."""
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
+
+
+def torch_to_bits(t) -> np.ndarray:
+    """bf16 torch tensor (any device) -> uint16 numpy bits."""
+    import torch
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+# --------------------------------------------------------------------------
+# Workloads.  Notation: page size ps, prefix P = tau-1 kept tokens,
+# suffix S = T - tau + 1 recomputed tokens, Hq/Hkv heads, head dim d, L layers.
+# --------------------------------------------------------------------------
+
+@dataclass
+class Agent:
+    T: int            # session length (tokens) before the forget request
+    tau: int          # 1-based position of the first tainted token
+    index: int        # agent index inside the workload (stream index)
+
+    @property
+    def P(self) -> int:
+        return self.tau - 1
+
+    @property
+    def S(self) -> int:
+        return self.T - self.tau + 1
+
+
+@dataclass
+class Workload:
+    name: str
+    seed: int
+    num_layers: int
+    num_q_heads: int
+    num_kv_heads: int
+    head_dim: int
+    page_size: int
+    std: float
+    agents: list = field(default_factory=list)
+    num_pages: int = 0
+    softmax_scale: float = 0.0
+
+    def pages_for(self, n_tokens: int) -> int:
+        return -(-n_tokens // self.page_size)
+
+    @property
+    def total_suffix(self) -> int:
+        return sum(a.S for a in self.agents)
+
+    @property
+    def max_pages_per_seq(self) -> int:
+        return max(self.pages_for(a.T) for a in self.agents)
+
+    def describe(self) -> dict:
+        return {
+            "workload": self.name,
+            "agents": len(self.agents),
+            "layers": self.num_layers,
+            "q_heads": self.num_q_heads,
+            "kv_heads": self.num_kv_heads,
+            "head_dim": self.head_dim,
+            "page_size": self.page_size,
+            "num_pages": self.num_pages,
+            "suffix_tokens": self.total_suffix,
+            "prefix_tokens": sum(a.P for a in self.agents),
+            "seed": self.seed,
+        }
+
+    # -- draws ---------------------------------------------------------------
+    def kv_original(self, agent: Agent):
+        """K, V of the original session: bf16 bits [L][T][Hkv][d] each."""
+        g = rng(self.seed, STREAM_KV_ORIG, agent.index)
+        shp = (self.num_layers, agent.T, self.num_kv_heads, self.head_dim)
+        return normal_bf16(g, shp, self.std), normal_bf16(g, shp, self.std)
+
+    def kv_counterfactual(self, agent: Agent):
+        """K', V' of the sanitized suffix: bf16 bits [L][S][Hkv][d] each."""
+        g = rng(self.seed, STREAM_KV_CF, agent.index)
+        shp = (self.num_layers, agent.S, self.num_kv_heads, self.head_dim)
+        return normal_bf16(g, shp, self.std), normal_bf16(g, shp, self.std)
+
+    def q_counterfactual(self, agent: Agent):
+        """Q' of the sanitized suffix: bf16 bits [L][S][Hq][d]."""
+        g = rng(self.seed, STREAM_Q_CF, agent.index)
+        return normal_bf16(g, (self.num_layers, agent.S, self.num_q_heads, self.head_dim), self.std)
+
+    def q_prefix(self, agent: Agent):
+        """Q of the prefix positions (only the full-reset comparator needs it): [L][P][Hq][d]."""
+        g = rng(self.seed, STREAM_Q_PREFIX, agent.index)
+        return normal_bf16(g, (self.num_layers, agent.P, self.num_q_heads, self.head_dim), self.std)
+
+    def init_free_order(self) -> np.ndarray:
+        return page_permutation(self.seed, self.num_pages)
+
+
+def _finish(w: Workload, slack_pages: int = 64) -> Workload:
+    if w.num_pages == 0:
+        w.num_pages = sum(w.pages_for(a.T) for a in w.agents) + slack_pages
+    if w.softmax_scale == 0.0:
+        w.softmax_scale = 1.0 / math.sqrt(w.head_dim)
+    return w
+
+
+def tiny() -> Workload:
+    """1 agent, 1 layer, 8/8 heads, d=64, ps=16, 64-page pool; T=640, prefix 512, suffix 128; N(0,1)."""
+    w = Workload("tiny", BASE_SEED + 1, 1, 8, 8, 64, 16, 1.0, num_pages=64)
+    w.agents = [Agent(T=640, tau=513, index=0)]
+    return _finish(w)
+
+
+def agent_batch(n_agents: int = 16) -> Workload:
+    """16 agents, 1 layer, GQA 32/8, d=128, ps=16; T ~ U{2048..8192}, tau/T ~ U[0.2, 0.9]; N(0,1)/sqrt(128)."""
+    w = Workload("agent_batch", BASE_SEED + 2, 1, 32, 8, 128, 16, 1.0 / math.sqrt(128))
+    g = rng(w.seed, STREAM_LENGTHS)
+    for i in range(n_agents):
+        T = int(g.integers(2048, 8192, endpoint=True))
+        r = float(g.uniform(0.2, 0.9))
+        P = int(round(r * T))
+        w.agents.append(Agent(T=T, tau=P + 1, index=i))
+    return _finish(w)
+
+
+def short_suffix(n_agents: int = 8, prefix: int = 32768, suffix: int = 16) -> Workload:
+    """8 agents, GQA 32/8, d=128, ps=16; prefix 32k, suffix 16; N(0,1)/sqrt(128)."""
+    w = Workload("short_suffix", BASE_SEED + 3, 1, 32, 8, 128, 16, 1.0 / math.sqrt(128))
+    w.agents = [Agent(T=prefix + suffix, tau=prefix + 1, index=i) for i in range(n_agents)]
+    return _finish(w)
+
+
+def long_suffix(n_agents: int = 4, prefix: int = 4096, suffix: int = 16384) -> Workload:
+    """4 agents, GQA 64/8, d=128, ps=64; prefix 4k, suffix 16k; N(0,1)/sqrt(128)."""
+    w = Workload("long_suffix", BASE_SEED + 4, 1, 64, 8, 128, 64, 1.0 / math.sqrt(128))
+    w.agents = [Agent(T=prefix + suffix, tau=prefix + 1, index=i) for i in range(n_agents)]
+    return _finish(w)
+
+
+TAU_SWEEP_RATIOS = (0.1, 0.3, 0.5, 0.7, 0.9)
+
+
+def tau_sweep(ratio: float, T: int = 16384, num_layers: int = 32) -> Workload:
+    """1 agent, 32 layers of GQA 32/8, d=128, ps=16, T=16k; prefix = round(ratio*T).
+
+    ratio = 0 is the full-reset comparator (empty prefix, whole sequence replayed).
+    """
+    w = Workload(f"tau_sweep_r{ratio:g}", BASE_SEED + 5, num_layers, 32, 8, 128, 16, 1.0 / math.sqrt(128))
+    P = int(round(ratio * T))
+    w.agents = [Agent(T=T, tau=P + 1, index=0)]
+    return _finish(w)
+
+
+WORKLOADS = {
+    "tiny": tiny,
+    "agent_batch": agent_batch,
+    "short_suffix": short_suffix,
+    "long_suffix": long_suffix,
+}
+
+
+def sample_rows(seed: int, n_q: int, n_random: int, tile_rows: int = 128, index: int = 0) -> np.ndarray:
+    """Query rows to check at full size: first/last row, both rows around every
+    tile boundary, plus ``n_random`` uniform rows (sorted, unique)."""
+    rows = {0, n_q - 1}
+    for b in range(tile_rows, n_q, tile_rows):
+        rows.add(b - 1)
+        rows.add(b)
+    g = rng(seed, STREAM_SAMPLE, index)
+    if n_q > 0 and n_random > 0:
+        rows.update(int(x) for x in g.integers(0, n_q, size=n_random))
+    return np.array(sorted(r for r in rows if 0 <= r < n_q), dtype=np.int64)

@@ -1,0 +1,63 @@
+"""Plant one plausible mistake at a time in a copy of the oracle (on the CPU) and
+check that the pins catch it.  This is evidence that the pins constrain every
+part of the oracle: a dropped term, a wrong index or alignment, a swapped
+operand, a wrong crop offset or push order."""
+import importlib.util
+import os
+import shutil
+import sys
+
+import pytest
+
+import oracle_pins as pins
+
+ORACLE_DIR = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "oracle")
+
+MUTANTS = [
+    ("gqa_mapping", "attention.c", "const int32_t kvh = h / group;", "const int32_t kvh = h % jb->hkv;"),
+    ("causal_off_by_one", "attention.c", "j <= a; ++j", "j < a; ++j"),
+    ("dropped_scale", "attention.c", "s *= jb->scale;", ""),
+    ("top_left_alignment", "attention.c", "const int64_t a = jb->n_keys - jb->n_q + i;", "const int64_t a = i;"),
+    ("value_from_keys", "attention.c", "const uint16_t *vrow = jb->v +", "const uint16_t *vrow = jb->k +"),
+    ("unnormalised", "attention.c", "o[c] /= den;", "o[c] /= 1.0;"),
+    ("crop_keeps_tau", "kvcache.py", "new_len = tau - 1\n", "new_len = min(tau, n)\n"),
+    ("push_ascending", "kvcache.py", "for p in reversed(freed):          # descending", "for p in freed:  #"),
+    ("slot_shift", "kvcache.py", "page, slot = tbl[pos // self.ps], pos % self.ps",
+     "page, slot = tbl[pos // self.ps], (pos + 1) % self.ps"),
+    ("counter_not_reset", "kvcache.py", "self.appended[seq] = 0\n        return list(freed)",
+     "return list(freed)"),
+]
+
+
+def _load_mutant(tmp_path, name, fname, old, new):
+    dst = tmp_path / f"oracle_mut_{name}"
+    shutil.copytree(ORACLE_DIR, dst, ignore=shutil.ignore_patterns("*.so", "__pycache__"))
+    path = dst / fname
+    src = path.read_text()
+    assert old in src, f"mutation anchor for {name} not found"
+    path.write_text(src.replace(old, new))
+    spec = importlib.util.spec_from_file_location(f"oracle_mut_{name}", dst / "__init__.py",
+                                                  submodule_search_locations=[str(dst)])
+    mod = importlib.util.module_from_spec(spec)
+    sys.modules[spec.name] = mod
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def _pins_fail(mod):
+    checks = [lambda: pins.pin_bruteforce(mod, full=False), lambda: pins.pin_closed_forms(mod),
+              lambda: pins.pin_splice(mod), lambda: pins.pin_corollary(mod),
+              lambda: pins.pin_bookkeeping(mod, n_ops=150)]
+    caught = 0
+    for chk in checks:
+        try:
+            chk()
+        except Exception:  # an assertion or any failure counts as caught
+            caught += 1
+    return caught
+
+
+@pytest.mark.parametrize("name,fname,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_planted_mistake(tmp_path, name, fname, old, new):
+    mod = _load_mutant(tmp_path, name, fname, old, new)
+    assert _pins_fail(mod) >= 1, f"no pin caught mutant {name}"
