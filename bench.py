@@ -1,0 +1,392 @@
+"""Benchmark of the crop + suffix replay path on GB300.
+
+One step = one forget request for every agent of the workload: batched crop
+to tau, batched append of the sanitized suffix K'/V', and batched causal
+replay attention of the suffix queries per layer, all through the C-ABI
+library.  Default workload: the 16-agent batch (GQA 32/8, d = 128, ps = 16,
+T ~ U{2048..8192}, tau/T ~ U[0.2, 0.9]).
+
+Prints one JSON line.  `value` = suffix tokens replayed per second over the
+whole job, inputs resident in HBM; `e2e` = the same with the step's inputs
+copied from pinned host memory and the outputs read back inside the timed
+region; `roofline` = the replay-attention kernel's algorithmic FLOP rate over
+the measured bf16 tensor peak; `cpu_baseline` = the fp64 CPU oracle timed on a
+bounded sample of the same workload.
+
+`--impl reference` times the oracle alone (the reference arm).
+Multi-GPU (torchrun): every rank runs its own replica of the workload
+(agents are independent; no collective on the data path), weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "suffix replay tokens/sec & % of roofline (BF16 peak / HBM BW); crop latency µs"
+UNIT = "tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def make_workload(name):
+    if name.startswith("tau_sweep_r"):
+        return synth.tau_sweep(float(name[len("tau_sweep_r"):]))
+    return synth.WORKLOADS[name]()
+
+
+def workload_flops(w):
+    pairs = sum(a.S * a.P + a.S * (a.S + 1) / 2 for a in w.agents)
+    return 4.0 * w.head_dim * w.num_q_heads * w.num_layers * pairs
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during a region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ------------------------------------------------------------------ CPU oracle
+def oracle_tokens_per_s(w, budget_s, seed=7):
+    """fp64 oracle on a bounded, uniformly random sample of suffix tokens
+    (all heads, all layers of the workload): returns (tokens/s, cores, sample text)."""
+    import oracle
+    cores = oracle.num_cpus()
+    g = synth.rng(seed, synth.STREAM_SAMPLE, 999)
+    weights = np.array([a.S for a in w.agents], dtype=np.float64)
+    weights /= weights.sum()
+    cache = {}
+
+    def seq_arrays(i):
+        if i not in cache:
+            a = w.agents[i]
+            k0, v0 = w.kv_original(a)
+            kc, vc = w.kv_counterfactual(a)
+            qc = w.q_counterfactual(a)
+            cache.clear()
+            cache[i] = (np.concatenate([k0[:, : a.P], kc], 1), np.concatenate([v0[:, : a.P], vc], 1), qc)
+        return cache[i]
+
+    done, spent, calls = 0, 0.0, 0
+    batch = 4
+    while spent < budget_s:
+        i = int(g.choice(len(w.agents), p=weights))
+        a = w.agents[i]
+        keys, vals, qc = seq_arrays(i)
+        rows = np.sort(g.integers(0, a.S, size=batch))
+        t0 = time.perf_counter()
+        for layer in range(w.num_layers):
+            oracle.causal_attention(qc[layer], keys[layer], vals[layer], w.softmax_scale, rows=rows)
+        spent += time.perf_counter() - t0
+        done += batch
+        calls += 1
+        batch = max(1, min(256, int(batch * 1.5)))
+    sample = (f"{done} suffix tokens drawn uniformly over the {len(w.agents)} agents' suffixes, all "
+              f"{w.num_q_heads} heads x {w.num_layers} layers, fp64 oracle, {spent:.1f} s")
+    return done / spent, cores, sample
+
+
+# ------------------------------------------------------------------ GPU arm
+def run_pe(args, rank, world, local_rank):
+    import torch
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    from paper_2609_04875_gb300.driver import ReplayDriver
+
+    w = make_workload(args.workload)
+    drv = ReplayDriver(w, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    L = w.num_layers
+    tokens_per_step = w.total_suffix
+    dist = world > 1
+
+    def barrier():
+        if dist:
+            import torch.distributed as tdist
+            tdist.barrier()
+
+    # ---- warm-up
+    for _ in range(args.warmup):
+        drv.step()
+    torch.cuda.synchronize(dev)
+
+    # ---- timed region (device-resident inputs)
+    n_ev = args.steps * L
+    attn_ev = [[torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)] for _ in range(n_ev)]
+    clocks = ClockSampler(local_rank) if rank == 0 else None
+    if clocks:
+        clocks.start()
+    launches0 = drv.cache.kernel_launches()
+    barrier()
+    torch.cuda.synchronize(dev)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(args.steps):
+        drv.step(attn_events=attn_ev[k * L:(k + 1) * L])
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier()
+    launches = drv.cache.kernel_launches() - launches0
+    clk = clocks.stop() if clocks else None
+    elapsed_ms = t_start.elapsed_time(t_end)
+    attn_ms = [a.elapsed_time(b) for a, b in attn_ev]
+    if dist:
+        import torch.distributed as tdist
+        t = torch.tensor([elapsed_ms], dtype=torch.float64)
+        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    ms_per_step = elapsed_ms / args.steps
+    value = world * tokens_per_step * args.steps / (elapsed_ms / 1e3)
+
+    # ---- crop latency: host call time and device time of the crop kernel
+    crop_host_us, crop_dev_us = [], []
+    for _ in range(20):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        h0 = time.perf_counter()
+        drv.crop()
+        h1 = time.perf_counter()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        crop_host_us.append((h1 - h0) * 1e6)
+        crop_dev_us.append(e0.elapsed_time(e1) * 1e3)
+        drv.append()
+        for layer in range(L):
+            drv.attend(layer)
+    torch.cuda.synchronize(dev)
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(drv, dev, stream, min(args.steps, args.e2e_steps), world, dist)
+
+    peaks, peak_src = load_peaks()
+    flops = workload_flops(w) / L  # per attention launch (one per layer)
+    attn_avg_s = statistics.mean(attn_ms) / 1e3
+    achieved = flops / attn_avg_s / 1e12
+    peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    result = {
+        "metric": METRIC,
+        "value": value,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1)/sqrt(128) bf16 Q/K/V; no dataset)",
+        "config": {
+            **w.describe(),
+            "parallelism": f"replicas x{world} (independent agents, no collective)",
+            "l2": "inputs larger than L2 (KV cache %.0f MB per GPU)" % (
+                sum(a.T for a in w.agents) * w.num_kv_heads * w.head_dim * 4 * w.num_layers / 1e6),
+        },
+        "roofline": {
+            "bound": "tensor",
+            "kernel": "replay_attn_kernel<128,false>",
+            "achieved": achieved,
+            "peak": peak,
+            "peak_source": f"bf16_tflops (burst) of {peak_src}",
+            "unit": "TFLOP/s",
+            "frac": achieved / peak,
+            "traffic": None,
+            "attn_ms_per_launch": attn_avg_s * 1e3,
+            "algorithmic_flop_per_launch": flops,
+        },
+        "attn_tflops_step": workload_flops(w) / (ms_per_step / 1e3) / 1e12,
+        "crop_us": {"host_call_median": statistics.median(crop_host_us),
+                    "device_median": statistics.median(crop_dev_us), "agents": len(w.agents)},
+        "gpu_launches": launches,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        tps, cores, sample = oracle_tokens_per_s(w, args.cpu_budget)
+        result["cpu_baseline"] = {"value": tps, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
+    elif rank == 0:
+        result["cpu_baseline"] = None
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+def run_e2e(drv, dev, stream, steps, world, dist):
+    """Same step through the public API with the step's inputs (K', V', Q') in
+    pinned host memory: H2D copies, crop + append + replay, D2H of the output."""
+    import torch
+    hK = drv.Kc.cpu().pin_memory()
+    hV = drv.Vc.cpu().pin_memory()
+    hQ = drv.Qc.cpu().pin_memory()
+    hO = torch.empty(drv.out.shape, dtype=drv.out.dtype).pin_memory()
+    h2d = (hK.numel() + hV.numel() + hQ.numel()) * 2
+    d2h = hO.numel() * 2
+
+    def one():
+        drv.Kc.copy_(hK, non_blocking=True)
+        drv.Vc.copy_(hV, non_blocking=True)
+        drv.Qc.copy_(hQ, non_blocking=True)
+        drv.step()
+        hO.copy_(drv.out, non_blocking=True)
+
+    for _ in range(3):
+        one()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1)
+    if dist:
+        import torch.distributed as tdist
+        t = torch.tensor([ms], dtype=torch.float64)
+        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+        ms = float(t.item())
+    tokens = world * drv.w.total_suffix * steps
+    return {"value": tokens / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "steps": steps, "ms_per_step": ms / steps}
+
+
+# ------------------------------------------------------------------ reference arm
+def run_reference(args, rank, world):
+    """The fp64 CPU oracle, timed as it stands on the host cores, on the same
+    workload; each step is a bounded sample of it."""
+    if rank != 0:
+        return
+    w = make_workload(args.workload)
+    per_step = []
+    tokens = []
+    samples = []
+    cores = None
+    for _ in range(args.warmup):
+        oracle_tokens_per_s(w, 0.2, seed=11)
+    for k in range(args.steps):
+        tps, cores, sample = oracle_tokens_per_s(w, args.ref_step_budget, seed=100 + k)
+        per_step.append(tps)
+        samples.append(sample)
+    value = statistics.mean(per_step)
+    result = {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": value,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": 1e3 * w.total_suffix / value,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic (seeded N(0,1)/sqrt(128) bf16 Q/K/V; no dataset)",
+        "config": {**w.describe(), "parallelism": "host cores (oracle)"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"per step: {samples[-1]}"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(result), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["pe", "reference"], default="pe")
+    ap.add_argument("--workload", default="agent_batch",
+                    help="agent_batch | tiny | short_suffix | long_suffix | tau_sweep_r<ratio>")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--ref-step-budget", type=float, default=3.0, help="seconds of oracle work per reference step")
+    args = ap.parse_args()
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch.distributed as tdist
+        tdist.init_process_group("gloo")
+    try:
+        run_pe(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as tdist
+            tdist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

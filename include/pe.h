@@ -1,0 +1,171 @@
+/*
+ * pe.h -- paged KV cache with crop and suffix replay, for one GB300 (sm_103a).
+ *
+ * The operations follow the problem statement of "Forgetting Without
+ * Restarting" (Provenance-Guided Selective Replay):
+ *   - a metadata-only checkpoint is a token offset, and restoring it is a crop
+ *     of the KV cache (Sec. 3.4(b); Sec. 4.1, KVEngine.crop);
+ *   - Alg. 1 Restore crops the cache to the last clean boundary; with every
+ *     token position a crop point that boundary is tau-1, the last position
+ *     before the target's injection step tau (Lemma 1: those states are shared
+ *     with the counterfactual run);
+ *   - Alg. 1's replay loop advances the state over the T - tau + 1 suffix
+ *     positions (Theorem 1, Corollary 1); counterfactually fixed content is
+ *     re-materialised by prefill on the cropped cache (Sec. 3.2, Sec. 4.5).
+ *     Here that prefill is: append the suffix K/V to the cache, then causal
+ *     attention of the suffix queries over prefix + suffix keys.
+ *
+ * Conventions shared by every call
+ *   - tau is 1-based (Sec. 3.1: the target enters at step tau >= 1); a crop to
+ *     tau keeps tau-1 tokens.
+ *   - Bookkeeping (free list, page tables, lengths) lives on the host, is
+ *     updated synchronously and deterministically inside the call, and is
+ *     mirrored to the device by work enqueued on `stream`.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Device work of a call runs in stream order; caller buffers
+ *     (K, V, Q, out) must stay valid until that work completes.  The library
+ *     keeps no reference to them after the call returns.
+ *   - All tensors are bf16, row-major, contiguous, 16-byte aligned device
+ *     memory unless stated otherwise.
+ *   - On any error the cache state is unchanged and pe_last_error() describes
+ *     the failure.  A cache is not thread-safe: calls on one cache must not run
+ *     concurrently.
+ *   - Allocation policy: the free list is a LIFO stack whose initial pop order
+ *     is `init_free_order`; an append pops one page per new logical page; crop
+ *     and release push the removed pages in descending logical order, so a
+ *     crop followed by an append of the same length restores the same table.
+ */
+#ifndef PE_H
+#define PE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pe_cache pe_cache; /* opaque, owned by the library */
+typedef int32_t pe_status;
+
+enum {
+    PE_OK = 0,
+    PE_ERR_INVALID = -1,        /* bad argument: null/misaligned pointer, tau < 1, unknown seq ... */
+    PE_ERR_RANGE = -2,          /* index or size out of range: tau-1 > len, n_q > len, layer ... */
+    PE_ERR_OOM = -3,            /* free list (or sequence slots) exhausted */
+    PE_ERR_CUDA = -4,           /* a CUDA runtime call failed */
+    PE_ERR_UNSUPPORTED = -5,    /* shape the kernels do not handle, or device call on a host-only cache */
+    PE_ERR_DEVICE_TIMEOUT = -6  /* a kernel's bounded wait ran out (see pe_device_status) */
+};
+
+typedef struct {
+    int32_t num_layers;         /* L >= 1; one page id addresses the same slot in every layer */
+    int32_t num_kv_heads;       /* Hkv >= 1 */
+    int32_t head_dim;           /* d: 64 or 128 */
+    int32_t page_size;          /* ps tokens per page: 8, 16, 32, 64 or 128 */
+    int32_t num_pages;          /* pages in the pool */
+    int32_t max_seqs;           /* sequence slots */
+    int32_t max_pages_per_seq;  /* page-table row length */
+    int32_t host_only;          /* 1: bookkeeping only (no device memory, no kernels); for tests */
+    const int32_t *init_free_order; /* host, nullable: pool pop order [num_pages]; NULL = 0,1,2,... */
+    void *k_pool;               /* device, nullable: caller-owned K pool, bf16 [L][num_pages][Hkv][ps][d] */
+    void *v_pool;               /* device, nullable: caller-owned V pool, same layout.  NULL = the
+                                   library allocates (cudaMalloc) and zero-fills both pools */
+    int64_t workspace_bytes;    /* split-KV scratch allocated at create; 0 = 64 MiB */
+} pe_cache_config;
+
+/* Creates a cache.  Sizes are checked (d, ps, positive counts, int32-addressable
+ * pool rows).  Device buffers are allocated on the current CUDA device.
+ * Errors: INVALID, UNSUPPORTED, OOM (host), CUDA. */
+pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out);
+pe_status pe_cache_destroy(pe_cache *cache);
+
+/* New empty sequence (len 0); the lowest free slot id is returned.  OOM if none. */
+pe_status pe_seq_create(pe_cache *cache, int32_t *seq_out);
+/* Frees every page of `seq` (pushed like a crop to tau = 1) and the slot. */
+pe_status pe_seq_release(pe_cache *cache, int32_t seq, void *stream);
+
+/* Crop = restore (Sec. 3.4(b); Alg. 1 Restore).  Keeps the first tau-1 tokens:
+ * pages at logical index >= ceil((tau-1)/ps) are removed from the table and
+ * pushed on the free list; the device table entries are set to -1 by a kernel
+ * on `stream`.  Resets the recomputation counter to 0.  tau = len+1 keeps
+ * every token.  freed_out (host, nullable) receives the freed page ids in
+ * ascending logical order; n_freed (nullable) their number.
+ * Errors: INVALID (tau < 1, unknown seq), RANGE (tau-1 > len, freed_cap too small). */
+pe_status pe_crop(pe_cache *cache, int32_t seq, int64_t tau, int32_t *freed_out, int32_t freed_cap,
+                  int32_t *n_freed, void *stream);
+
+/* Crops n sequences (host arrays seqs[n], taus[n]) with one device launch.
+ * All-or-nothing: every (seq, tau) is validated before any state changes;
+ * a sequence may appear once. */
+pe_status pe_crop_batch(pe_cache *cache, int32_t n, const int32_t *seqs, const int64_t *taus, void *stream);
+
+/* Prefill write of the replayed suffix (Sec. 3.2): appends n_tokens positions.
+ * K, V: device bf16 [L][n_tokens][Hkv][d].  New pages are popped from the
+ * free list before any device work; the copy into the pool runs on `stream`.
+ * The recomputation counter grows by n_tokens (Corollary 1 counts it).
+ * Errors: RANGE (exceeds max_pages_per_seq), OOM (not enough free pages),
+ * INVALID (null/misaligned pointers). */
+pe_status pe_append_kv(pe_cache *cache, int32_t seq, const void *K, const void *V, int32_t n_tokens,
+                       void *stream);
+
+/* Batched append: sequence i receives tokens [cu_tokens[i], cu_tokens[i+1]) of
+ * K_packed / V_packed, device bf16 [L][cu_tokens[n]][Hkv][d]; cu_tokens is a
+ * host array [n+1] starting at 0.  One device launch; all-or-nothing. */
+pe_status pe_append_kv_batch(pe_cache *cache, int32_t n, const int32_t *seqs, const void *K_packed,
+                             const void *V_packed, const int32_t *cu_tokens, void *stream);
+
+/* Replay attention (Alg. 1 replay loop; Sec. 3.2 prefill on the cropped cache).
+ * The n_q queries are the LAST n_q positions of `seq`: query i sits at
+ * position len-n_q+i and attends keys 0..len-n_q+i of `layer` (causal,
+ * bottom-right aligned).  q-head h reads kv-head h / (Hq/Hkv).
+ *   O = softmax(softmax_scale * q K^T) V, fp32 accumulation, bf16 output.
+ * Q: device bf16 [n_q][Hq][d]; out: device bf16 [n_q][Hq][d].
+ * Hq must be a multiple of Hkv with Hq/Hkv a power of two <= 128.
+ * Errors: RANGE (n_q > len, layer), INVALID, UNSUPPORTED. */
+pe_status pe_replay_attn(pe_cache *cache, int32_t seq, int32_t layer, const void *Q, void *out, int32_t n_q,
+                         int32_t num_q_heads, float softmax_scale, void *stream);
+
+/* Batched varlen replay attention: sequence i's queries are rows
+ * [cu_q[i], cu_q[i+1]) of Q_packed / out (device bf16 [cu_q[n]][Hq][d]), and
+ * are its last cu_q[i+1]-cu_q[i] positions.  cu_q: host [n+1], from 0. */
+pe_status pe_replay_attn_batch(pe_cache *cache, int32_t n, const int32_t *seqs, int32_t layer,
+                               const void *Q_packed, const int32_t *cu_q, void *out, int32_t num_q_heads,
+                               float softmax_scale, void *stream);
+
+/* Host-side state queries (no device work). */
+pe_status pe_seq_info(const pe_cache *cache, int32_t seq, int64_t *len, int64_t *appended_since_crop);
+pe_status pe_seq_page_table(const pe_cache *cache, int32_t seq, int32_t *out, int32_t cap, int32_t *n);
+pe_status pe_free_list(const pe_cache *cache, int32_t *out, int32_t cap, int32_t *n); /* top of stack first */
+
+/* Synchronous copy of a sequence's DEVICE page-table row (first `cap` entries)
+ * into host `out`, after all work on `stream`; for checking the mirror. */
+pe_status pe_seq_device_page_table(pe_cache *cache, int32_t seq, int32_t *out, int32_t cap, void *stream);
+
+/* Device pool pointers (for reading pool contents back). */
+pe_status pe_cache_pools(const pe_cache *cache, void **k_pool, void **v_pool);
+
+/* Options: "splitkv" = -1 (auto, default) / 0 (never) / 1 (always);
+ * "num_splits" = 0 (auto) or the split count; "debug_poison" = 0/1: crop
+ * fills freed pages and the stale tail of the last kept page with a finite
+ * sentinel (bf16 2^100), so that a kernel reading them unmasked gives a
+ * visibly wrong result. */
+pe_status pe_set_option(pe_cache *cache, const char *key, int64_t value);
+
+/* Synchronises `stream` and reads the device status word.  *code = 0 when no
+ * kernel reported a problem, else the first recorded code (1 = a bounded
+ * wait ran out).  clear != 0 resets it.  Returns DEVICE_TIMEOUT if *code != 0. */
+pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *stream);
+
+/* Number of kernel launches this cache has made so far (crop, append,
+ * attention, combine); lets a caller count its device work. */
+pe_status pe_kernel_launches(const pe_cache *cache, int64_t *count);
+
+/* Thread-local description of the last error on this thread ("" if none). */
+const char *pe_last_error(void);
+/* Library version string. */
+const char *pe_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PE_H */

@@ -1,0 +1,304 @@
+"""ctypes binding of libpe (include/pe.h): argument marshalling only.
+
+Every step of the path -- crop, append, replay attention, split-KV combine --
+runs in the library's CUDA kernels; this module passes tensor pointers, sizes
+and the current CUDA stream, and turns status codes into exceptions.  There is
+no other implementation behind it: if libpe.so is missing, importing this
+module fails.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libpe.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is not built; run `python -c 'import __graft_entry__ as g; g.build()'`")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+PE_OK = 0
+ERROR_KINDS = {-1: "invalid", -2: "range", -3: "oom", -4: "cuda", -5: "unsupported", -6: "device_timeout"}
+
+EXPORTED = [
+    "pe_cache_create", "pe_cache_destroy", "pe_seq_create", "pe_seq_release", "pe_crop", "pe_crop_batch",
+    "pe_append_kv", "pe_append_kv_batch", "pe_replay_attn", "pe_replay_attn_batch", "pe_seq_info",
+    "pe_seq_page_table", "pe_free_list", "pe_seq_device_page_table", "pe_cache_pools", "pe_set_option",
+    "pe_device_status", "pe_kernel_launches", "pe_last_error", "pe_version",
+]
+
+
+class PEError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{ERROR_KINDS.get(code, code)}: {msg}")
+        self.code = code
+        self.kind = ERROR_KINDS.get(code, str(code))
+
+
+class _Config(ctypes.Structure):
+    _fields_ = [
+        ("num_layers", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+        ("page_size", ctypes.c_int32), ("num_pages", ctypes.c_int32), ("max_seqs", ctypes.c_int32),
+        ("max_pages_per_seq", ctypes.c_int32), ("host_only", ctypes.c_int32),
+        ("init_free_order", ctypes.POINTER(ctypes.c_int32)), ("k_pool", ctypes.c_void_p),
+        ("v_pool", ctypes.c_void_p), ("workspace_bytes", ctypes.c_int64),
+    ]
+
+
+_P = ctypes.c_void_p
+_I32 = ctypes.c_int32
+_I64 = ctypes.c_int64
+_I32P = ctypes.POINTER(ctypes.c_int32)
+_I64P = ctypes.POINTER(ctypes.c_int64)
+
+_sigs = {
+    "pe_cache_create": [ctypes.POINTER(_Config), ctypes.POINTER(_P)],
+    "pe_cache_destroy": [_P],
+    "pe_seq_create": [_P, _I32P],
+    "pe_seq_release": [_P, _I32, _P],
+    "pe_crop": [_P, _I32, _I64, _I32P, _I32, _I32P, _P],
+    "pe_crop_batch": [_P, _I32, _I32P, _I64P, _P],
+    "pe_append_kv": [_P, _I32, _P, _P, _I32, _P],
+    "pe_append_kv_batch": [_P, _I32, _I32P, _P, _P, _I32P, _P],
+    "pe_replay_attn": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
+    "pe_replay_attn_batch": [_P, _I32, _I32P, _I32, _P, _I32P, _P, _I32, ctypes.c_float, _P],
+    "pe_seq_info": [_P, _I32, _I64P, _I64P],
+    "pe_seq_page_table": [_P, _I32, _I32P, _I32, _I32P],
+    "pe_free_list": [_P, _I32P, _I32, _I32P],
+    "pe_seq_device_page_table": [_P, _I32, _I32P, _I32, _P],
+    "pe_cache_pools": [_P, ctypes.POINTER(_P), ctypes.POINTER(_P)],
+    "pe_set_option": [_P, ctypes.c_char_p, _I64],
+    "pe_device_status": [_P, _I32P, _I32, _P],
+    "pe_kernel_launches": [_P, _I64P],
+}
+for _name, _args in _sigs.items():
+    _fn = getattr(_lib, _name)
+    _fn.argtypes = _args
+    _fn.restype = ctypes.c_int32
+_lib.pe_last_error.restype = ctypes.c_char_p
+_lib.pe_last_error.argtypes = []
+_lib.pe_version.restype = ctypes.c_char_p
+_lib.pe_version.argtypes = []
+
+
+def lib():
+    return _lib
+
+
+def version() -> str:
+    return _lib.pe_version().decode()
+
+
+def _check(rc: int):
+    if rc != PE_OK:
+        raise PEError(rc, _lib.pe_last_error().decode())
+
+
+def _i32_array(vals):
+    vals = [int(v) for v in vals]
+    return (ctypes.c_int32 * max(1, len(vals)))(*vals)
+
+
+def _i64_array(vals):
+    vals = [int(v) for v in vals]
+    return (ctypes.c_int64 * max(1, len(vals)))(*vals)
+
+
+def _stream(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _dev_ptr(t, name):
+    import torch
+    if t.dtype != torch.bfloat16:
+        raise TypeError(f"{name} must be bfloat16")
+    if not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+class PagedKVCache:
+    """Paged KV cache with crop and replay attention (one GPU).
+
+    Pool layout per layer: [num_pages][Hkv][page_size][d] bf16 for K and V.
+    ``k_pool`` / ``v_pool``: optional caller-owned CUDA tensors of shape
+    [L][num_pages][Hkv][page_size][d] (bf16); otherwise the library allocates.
+    ``host_only=True`` keeps only the host bookkeeping (no device memory).
+    """
+
+    def __init__(self, num_layers, num_kv_heads, head_dim, page_size, num_pages, max_seqs, max_pages_per_seq,
+                 init_free_order=None, k_pool=None, v_pool=None, host_only=False, workspace_bytes=0):
+        cfg = _Config()
+        cfg.num_layers, cfg.num_kv_heads, cfg.head_dim = num_layers, num_kv_heads, head_dim
+        cfg.page_size, cfg.num_pages, cfg.max_seqs = page_size, num_pages, max_seqs
+        cfg.max_pages_per_seq, cfg.host_only = max_pages_per_seq, 1 if host_only else 0
+        self._order = None
+        if init_free_order is not None:
+            self._order = _i32_array(init_free_order)
+            if len(init_free_order) != num_pages:
+                raise ValueError("init_free_order must list every page")
+            cfg.init_free_order = ctypes.cast(self._order, _I32P)
+        self._pools = (k_pool, v_pool)  # keep caller tensors alive
+        if k_pool is not None:
+            cfg.k_pool = _dev_ptr(k_pool, "k_pool").value
+            cfg.v_pool = _dev_ptr(v_pool, "v_pool").value
+        cfg.workspace_bytes = int(workspace_bytes)
+        self.num_layers, self.num_kv_heads, self.head_dim = num_layers, num_kv_heads, head_dim
+        self.page_size, self.num_pages, self.max_seqs = page_size, num_pages, max_seqs
+        self.max_pages_per_seq = max_pages_per_seq
+        self.host_only = host_only
+        h = ctypes.c_void_p()
+        _check(_lib.pe_cache_create(ctypes.byref(cfg), ctypes.byref(h)))
+        self._h = h
+
+    # -- lifetime ------------------------------------------------------------
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            _check(_lib.pe_cache_destroy(self._h))
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    @property
+    def handle(self):
+        return self._h
+
+    def _s(self, stream):
+        return ctypes.c_void_p(None) if self.host_only else _stream(stream)
+
+    # -- sequences -----------------------------------------------------------
+    def seq_create(self) -> int:
+        s = ctypes.c_int32()
+        _check(_lib.pe_seq_create(self._h, ctypes.byref(s)))
+        return s.value
+
+    def seq_release(self, seq, stream=None):
+        _check(_lib.pe_seq_release(self._h, seq, self._s(stream)))
+
+    # -- crop (restore) --------------------------------------------------------
+    def crop(self, seq, tau, stream=None):
+        """Keep the first tau-1 tokens; returns the freed page ids (ascending logical)."""
+        cap = self.max_pages_per_seq
+        buf = (ctypes.c_int32 * cap)()
+        n = ctypes.c_int32()
+        _check(_lib.pe_crop(self._h, seq, int(tau), buf, cap, ctypes.byref(n), self._s(stream)))
+        return list(buf[: n.value])
+
+    def crop_batch(self, seqs, taus, stream=None):
+        _check(_lib.pe_crop_batch(self._h, len(seqs), _i32_array(seqs), _i64_array(taus), self._s(stream)))
+
+    # -- append (prefill write) ------------------------------------------------
+    def append_kv(self, seq, K=None, V=None, n_tokens=None, stream=None):
+        """K, V: CUDA bf16 [L][n][Hkv][d].  Host-only caches take n_tokens instead."""
+        if K is None:
+            if not self.host_only:
+                raise ValueError("K and V are required")
+            _check(_lib.pe_append_kv(self._h, seq, None, None, int(n_tokens), self._s(stream)))
+            return
+        self._check_kv(K, V)
+        _check(_lib.pe_append_kv(self._h, seq, _dev_ptr(K, "K"), _dev_ptr(V, "V"), K.shape[1], self._s(stream)))
+
+    def append_kv_batch(self, seqs, K=None, V=None, cu_tokens=None, stream=None):
+        """K, V: CUDA bf16 [L][cu_tokens[-1]][Hkv][d]; sequence i gets tokens cu_tokens[i]:cu_tokens[i+1]."""
+        cu = _i32_array(cu_tokens)
+        if K is None:
+            if not self.host_only:
+                raise ValueError("K and V are required")
+            _check(_lib.pe_append_kv_batch(self._h, len(seqs), _i32_array(seqs), None, None, cu, self._s(stream)))
+            return
+        self._check_kv(K, V)
+        if K.shape[1] != cu_tokens[-1]:
+            raise ValueError("K token count does not match cu_tokens")
+        _check(_lib.pe_append_kv_batch(self._h, len(seqs), _i32_array(seqs), _dev_ptr(K, "K"), _dev_ptr(V, "V"),
+                                       cu, self._s(stream)))
+
+    def _check_kv(self, K, V):
+        if K.shape != V.shape or K.dim() != 4:
+            raise ValueError("K and V must both be [L][n][Hkv][d]")
+        if K.shape[0] != self.num_layers or K.shape[2] != self.num_kv_heads or K.shape[3] != self.head_dim:
+            raise ValueError(f"K shape {tuple(K.shape)} does not match the cache")
+
+    # -- replay attention ------------------------------------------------------
+    def replay_attn(self, seq, layer, Q, out=None, softmax_scale=None, stream=None):
+        """Attention of the last Q.shape[0] positions of ``seq``; Q, out: CUDA bf16 [n_q][Hq][d]."""
+        import torch
+        if Q.dim() != 3 or Q.shape[2] != self.head_dim:
+            raise ValueError("Q must be [n_q][Hq][d]")
+        if out is None:
+            out = torch.empty_like(Q)
+        scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
+        _check(_lib.pe_replay_attn(self._h, seq, layer, _dev_ptr(Q, "Q"), _dev_ptr(out, "out"), Q.shape[0],
+                                   Q.shape[1], scale, self._s(stream)))
+        return out
+
+    def replay_attn_batch(self, seqs, layer, Q, cu_q, out=None, softmax_scale=None, stream=None):
+        """Q, out: CUDA bf16 [cu_q[-1]][Hq][d]; rows cu_q[i]:cu_q[i+1] are the last positions of seqs[i]."""
+        import torch
+        if Q.dim() != 3 or Q.shape[2] != self.head_dim or Q.shape[0] != cu_q[-1]:
+            raise ValueError("Q must be [cu_q[-1]][Hq][d]")
+        if out is None:
+            out = torch.empty_like(Q)
+        scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
+        _check(_lib.pe_replay_attn_batch(self._h, len(seqs), _i32_array(seqs), layer, _dev_ptr(Q, "Q"),
+                                         _i32_array(cu_q), _dev_ptr(out, "out"), Q.shape[1], scale,
+                                         self._s(stream)))
+        return out
+
+    # -- state -----------------------------------------------------------------
+    def seq_info(self, seq):
+        n, a = ctypes.c_int64(), ctypes.c_int64()
+        _check(_lib.pe_seq_info(self._h, seq, ctypes.byref(n), ctypes.byref(a)))
+        return n.value, a.value
+
+    def page_table(self, seq):
+        n = ctypes.c_int32()
+        _check(_lib.pe_seq_page_table(self._h, seq, None, 0, ctypes.byref(n)))
+        buf = (ctypes.c_int32 * max(1, n.value))()
+        _check(_lib.pe_seq_page_table(self._h, seq, buf, n.value, ctypes.byref(n)))
+        return list(buf[: n.value])
+
+    def free_list(self):
+        n = ctypes.c_int32()
+        _check(_lib.pe_free_list(self._h, None, 0, ctypes.byref(n)))
+        buf = (ctypes.c_int32 * max(1, n.value))()
+        _check(_lib.pe_free_list(self._h, buf, n.value, ctypes.byref(n)))
+        return list(buf[: n.value])
+
+    def device_page_table(self, seq, n=None, stream=None):
+        n = self.max_pages_per_seq if n is None else n
+        buf = (ctypes.c_int32 * max(1, n))()
+        _check(_lib.pe_seq_device_page_table(self._h, seq, buf, n, self._s(stream)))
+        return list(buf[:n])
+
+    def set_option(self, key: str, value: int):
+        _check(_lib.pe_set_option(self._h, key.encode(), int(value)))
+
+    def kernel_launches(self) -> int:
+        n = ctypes.c_int64()
+        _check(_lib.pe_kernel_launches(self._h, ctypes.byref(n)))
+        return n.value
+
+    def device_status(self, clear=True, stream=None):
+        code = ctypes.c_int32()
+        rc = _lib.pe_device_status(self._h, ctypes.byref(code), 1 if clear else 0, self._s(stream))
+        if rc not in (PE_OK, -6):
+            _check(rc)
+        return code.value

@@ -1,0 +1,821 @@
+// Host side of the pe library: the paged KV store's bookkeeping (free list,
+// page tables, lengths, recomputation counters), argument checks, tensor maps
+// and kernel launches behind the C ABI declared in include/pe.h.
+//
+// Crop = restore of a metadata-only checkpoint (Sec. 3.4(b), Sec. 4.1 crop);
+// Alg. 1 Restore crops to tau-1; the replay loop re-prefills the T-tau+1
+// suffix positions (Theorem 1, Corollary 1, Sec. 3.2).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "pe.h"
+#include "pe_internal.h"
+
+using namespace pe;
+
+namespace {
+
+thread_local std::string g_err;
+
+pe_status fail(pe_status code, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return code;
+}
+
+pe_status cuda_fail(cudaError_t e, const char *what)
+{
+    return fail(PE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+}  // namespace
+
+struct pe_cache {
+    pe_cache_config cfg{};
+    bool host_only = false;
+    // host bookkeeping (authoritative)
+    std::vector<int32_t> free_stack;               // top = back()
+    std::vector<std::vector<int32_t>> table;       // per sequence slot
+    std::vector<int64_t> len, appended;
+    std::vector<uint8_t> alive;
+    // device state
+    int device = 0;
+    int num_sms = 148;
+    void *k_pool = nullptr, *v_pool = nullptr;
+    bool own_pools = false;
+    int32_t *d_table = nullptr;
+    int64_t *d_len = nullptr;
+    int32_t *d_status = nullptr;
+    float *d_ws = nullptr;
+    int64_t ws_bytes = 0;
+    int64_t pool_rows = 0;  // L * num_pages * Hkv * ps
+    CUtensorMap tm_k{}, tm_v{};
+    // options
+    int splitkv = -1, num_splits = 0, debug_poison = 0;
+    int64_t launches = 0;
+};
+
+namespace {
+
+pe_status check_seq(const pe_cache *c, int32_t seq)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (seq < 0 || seq >= c->cfg.max_seqs || !c->alive[seq]) return fail(PE_ERR_INVALID, "unknown sequence %d", seq);
+    return PE_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+pe_status encode_2d(CUtensorMap *m, void *base, uint64_t cols, uint64_t rows, uint32_t box_cols, uint32_t box_rows)
+{
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(PE_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {box_cols, box_rows};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(PE_ERR_CUDA, "cuTensorMapEncodeTiled (2d) failed: %d", static_cast<int>(r));
+    return PE_OK;
+}
+
+// Q viewed as [rows][Hq][d]: box (64, g, 128/g) gathers 128/g queries x g heads.
+pe_status encode_q(CUtensorMap *m, const void *q, int64_t rows, int hq, int d, int g)
+{
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(PE_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(hq), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2, static_cast<cuuint64_t>(hq) * d * 2};
+    cuuint32_t box[3] = {64, static_cast<cuuint32_t>(g), static_cast<cuuint32_t>(kBM / g)};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(q), dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(PE_ERR_CUDA, "cuTensorMapEncodeTiled (q) failed: %d", static_cast<int>(r));
+    return PE_OK;
+}
+
+void free_device(pe_cache *c)
+{
+    if (c->own_pools) {
+        if (c->k_pool) cudaFree(c->k_pool);
+        if (c->v_pool) cudaFree(c->v_pool);
+    }
+    if (c->d_table) cudaFree(c->d_table);
+    if (c->d_len) cudaFree(c->d_len);
+    if (c->d_status) cudaFree(c->d_status);
+    if (c->d_ws) cudaFree(c->d_ws);
+    c->k_pool = c->v_pool = nullptr;
+    c->d_table = nullptr;
+    c->d_len = nullptr;
+    c->d_status = nullptr;
+    c->d_ws = nullptr;
+}
+
+// ---- crop bookkeeping shared by pe_crop, pe_crop_batch and pe_seq_release
+struct CropPlan {
+    int32_t seq;
+    int32_t keep, old_n;
+    int64_t new_len;
+};
+
+void apply_crop(pe_cache *c, const CropPlan &pl, int32_t *freed_out)
+{
+    std::vector<int32_t> &t = c->table[pl.seq];
+    for (int32_t e = pl.keep; e < pl.old_n; ++e)
+        if (freed_out) freed_out[e - pl.keep] = t[e];
+    for (int32_t e = pl.old_n - 1; e >= pl.keep; --e)  // descending logical order onto the stack
+        c->free_stack.push_back(t[e]);
+    t.resize(pl.keep);
+    c->len[pl.seq] = pl.new_len;
+    c->appended[pl.seq] = 0;
+}
+
+pe_status launch_crops(pe_cache *c, const std::vector<CropPlan> &plans, cudaStream_t st)
+{
+    if (c->host_only) return PE_OK;
+    CropParams p{};
+    p.page_table = c->d_table;
+    p.seq_len = c->d_len;
+    p.k_pool = static_cast<uint4 *>(c->k_pool);
+    p.v_pool = static_cast<uint4 *>(c->v_pool);
+    p.poison = c->debug_poison;
+    p.L = c->cfg.num_layers;
+    p.hkv = c->cfg.num_kv_heads;
+    p.ps = c->cfg.page_size;
+    p.dvec = c->cfg.head_dim / 8;
+    p.num_pages = c->cfg.num_pages;
+    size_t i = 0;
+    while (i < plans.size()) {
+        p.n = 0;
+        while (i < plans.size() && p.n < kMaxCropSegs) {
+            const CropPlan &pl = plans[i++];
+            CropSeg &sg = p.segs[p.n++];
+            sg.table_row = pl.seq * c->cfg.max_pages_per_seq;
+            sg.keep = pl.keep;
+            sg.old_n = pl.old_n;
+            sg.seq = pl.seq;
+            sg.new_len = pl.new_len;
+        }
+        cudaError_t e = launch_crop(p, st);
+        if (e != cudaSuccess) return cuda_fail(e, "crop kernel launch");
+        c->launches++;
+    }
+    return PE_OK;
+}
+
+pe_status plan_crop(const pe_cache *c, int32_t seq, int64_t tau, CropPlan *pl)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if (tau < 1) return fail(PE_ERR_INVALID, "tau = %lld < 1", static_cast<long long>(tau));
+    if (tau - 1 > c->len[seq])
+        return fail(PE_ERR_RANGE, "tau - 1 = %lld exceeds the sequence length %lld", static_cast<long long>(tau - 1),
+                    static_cast<long long>(c->len[seq]));
+    pl->seq = seq;
+    pl->new_len = tau - 1;
+    pl->keep = static_cast<int32_t>(ceil_div(tau - 1, c->cfg.page_size));
+    pl->old_n = static_cast<int32_t>(c->table[seq].size());
+    return PE_OK;
+}
+
+// ---- append bookkeeping
+struct AppendPlan {
+    int32_t seq;
+    int32_t tok0;  // offset in the packed K/V
+    int32_t n;
+    int32_t need;  // pages to pop
+};
+
+pe_status plan_append(const pe_cache *c, int32_t seq, int64_t n, AppendPlan *pl)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if (n < 0) return fail(PE_ERR_INVALID, "negative token count");
+    const int64_t new_len = c->len[seq] + n;
+    const int64_t pages = ceil_div(new_len, c->cfg.page_size);
+    if (pages > c->cfg.max_pages_per_seq)
+        return fail(PE_ERR_RANGE, "sequence %d would need %lld pages > max_pages_per_seq %d", seq,
+                    static_cast<long long>(pages), c->cfg.max_pages_per_seq);
+    if (new_len > INT32_MAX) return fail(PE_ERR_RANGE, "sequence length exceeds int32");
+    pl->seq = seq;
+    pl->n = static_cast<int32_t>(n);
+    pl->need = static_cast<int32_t>(pages - static_cast<int64_t>(c->table[seq].size()));
+    return PE_OK;
+}
+
+// Pops pages for every plan (the caller checked there are enough), then
+// launches the copies.  Launches are cut so that each carries at most
+// kMaxSegs segments and kAppendMaxPages new page ids.
+pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const void *K, const void *V,
+                        int64_t n_total, cudaStream_t st)
+{
+    const int ps = c->cfg.page_size;
+    AppendParams *p = nullptr;
+    std::vector<char> pbuf;
+    if (!c->host_only) {
+        pbuf.resize(sizeof(AppendParams));
+        p = reinterpret_cast<AppendParams *>(pbuf.data());
+        std::memset(p, 0, sizeof(AppendParams));
+        p->K = static_cast<const uint4 *>(K);
+        p->V = static_cast<const uint4 *>(V);
+        p->k_pool = static_cast<uint4 *>(c->k_pool);
+        p->v_pool = static_cast<uint4 *>(c->v_pool);
+        p->page_table = c->d_table;
+        p->seq_len = c->d_len;
+        p->L = c->cfg.num_layers;
+        p->hkv = c->cfg.num_kv_heads;
+        p->dvec = c->cfg.head_dim / 8;
+        p->ps = ps;
+        p->num_pages = c->cfg.num_pages;
+        p->n_total = static_cast<int32_t>(n_total);
+    }
+    auto flush = [&]() -> pe_status {
+        if (c->host_only || p->n_segs == 0) return PE_OK;
+        p->seg_tokens = p->segs[p->n_segs - 1].cum0 + p->segs[p->n_segs - 1].n_tokens;
+        const int64_t chunks = static_cast<int64_t>(p->L) * p->seg_tokens * p->hkv * p->dvec;
+        if (chunks > 0 || p->n_segs > 0) {
+            cudaError_t e = launch_append(*p, chunks, st);
+            if (e != cudaSuccess) return cuda_fail(e, "append kernel launch");
+            c->launches++;
+        }
+        p->n_segs = 0;
+        return PE_OK;
+    };
+    int32_t pages_in_launch = 0;
+    for (const AppendPlan &pl : plans) {
+        int32_t done = 0;
+        while (done < pl.n) {
+            const int64_t len0 = c->len[pl.seq];
+            std::vector<int32_t> &t = c->table[pl.seq];
+            // tokens that fit without exceeding the page budget of this launch
+            const int64_t room_pages = kAppendMaxPages - pages_in_launch;
+            const int64_t have_slots = static_cast<int64_t>(t.size()) * ps - len0;  // free slots in last page
+            int64_t take = pl.n - done;
+            const int64_t max_take = have_slots + room_pages * ps;
+            if (take > max_take) take = max_take;
+            if (!c->host_only && (take <= 0 || p->n_segs == kMaxSegs)) {
+                pe_status s = flush();
+                if (s != PE_OK) return s;
+                pages_in_launch = 0;
+                continue;
+            }
+            const int32_t first_new_lp = static_cast<int32_t>(t.size());
+            const int32_t need = static_cast<int32_t>(ceil_div(len0 + take, ps) - static_cast<int64_t>(t.size()));
+            if (!c->host_only) {
+                AppendSeg &sg = p->segs[p->n_segs];
+                sg.tok0 = pl.tok0 + done;
+                sg.cum0 = p->n_segs == 0 ? 0 : p->segs[p->n_segs - 1].cum0 + p->segs[p->n_segs - 1].n_tokens;
+                sg.n_tokens = static_cast<int32_t>(take);
+                sg.len0 = static_cast<int32_t>(len0);
+                sg.first_new_lp = first_new_lp;
+                sg.last_page = first_new_lp > 0 ? t[first_new_lp - 1] : -1;
+                sg.new0 = pages_in_launch;
+                sg.n_new = need;
+                sg.table_row = pl.seq * c->cfg.max_pages_per_seq;
+                sg.seq = pl.seq;
+            }
+            for (int32_t i = 0; i < need; ++i) {
+                const int32_t pg = c->free_stack.back();
+                c->free_stack.pop_back();
+                t.push_back(pg);
+                if (!c->host_only) p->new_pages[pages_in_launch + i] = pg;
+            }
+            if (!c->host_only) {
+                pages_in_launch += need;
+                p->n_segs++;
+            }
+            c->len[pl.seq] = len0 + take;
+            c->appended[pl.seq] += take;
+            done += static_cast<int32_t>(take);
+        }
+    }
+    return flush();
+}
+
+// ---- attention planning
+struct AttnItem {
+    int32_t seq;
+    int32_t q_row0;
+    int32_t n_q;
+};
+
+pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t layer, const void *Q,
+                        int64_t q_rows, void *out, int32_t hq, float scale, cudaStream_t st)
+{
+    const pe_cache_config &cf = c->cfg;
+    const int hkv = cf.num_kv_heads;
+    const int d = cf.head_dim;
+    const int g = hq / hkv;
+    const int bmq = kBM / g;
+    // heaviest sequences first (more key tiles per q-tile)
+    std::vector<AttnItem> order;
+    for (const AttnItem &it : items)
+        if (it.n_q > 0) order.push_back(it);
+    std::stable_sort(order.begin(), order.end(), [&](const AttnItem &a, const AttnItem &b) {
+        return c->len[a.seq] > c->len[b.seq];
+    });
+    if (order.empty()) return PE_OK;
+
+    CUtensorMap tm_q;
+    pe_status s = encode_q(&tm_q, Q, q_rows, hq, d, g);
+    if (s != PE_OK) return s;
+
+    // split-KV decision over the whole launch group
+    auto plan_group = [&](size_t lo, size_t hi, AttnParams &p, bool &split) -> pe_status {
+        int64_t base_ctas = 0, total_tiles = 0, max_tiles = 0;
+        for (size_t i = lo; i < hi; ++i) {
+            const AttnItem &it = order[i];
+            const int64_t nqt = ceil_div(static_cast<int64_t>(it.n_q) * g, kBM);
+            base_ctas += nqt * hkv;
+            const int64_t ktiles = ceil_div(c->len[it.seq], kBN);
+            total_tiles += ktiles * nqt * hkv;
+            max_tiles = std::max(max_tiles, ktiles);
+        }
+        int split_tiles = static_cast<int>(max_tiles);
+        if (c->splitkv == 1 || (c->splitkv == -1 && base_ctas < c->num_sms && max_tiles >= 16)) {
+            if (c->num_splits > 0) {
+                split_tiles = static_cast<int>(ceil_div(max_tiles, c->num_splits));
+            } else {
+                const int64_t target = 4LL * c->num_sms;
+                split_tiles = static_cast<int>(std::max<int64_t>(4, ceil_div(total_tiles, target)));
+            }
+            split_tiles = std::max(1, split_tiles);
+            split = true;
+        } else {
+            split = false;
+        }
+        std::memset(&p, 0, sizeof p);
+        p.page_table = c->d_table;
+        p.out = out;
+        p.status = c->d_status;
+        p.hq = hq;
+        p.hkv = hkv;
+        p.group = g;
+        p.layer = layer;
+        p.num_pages = cf.num_pages;
+        p.ps = cf.page_size;
+        p.oob_row = static_cast<int32_t>(c->pool_rows);
+        p.scale_log2 = scale * 1.4426950408889634f;
+        for (;;) {
+            int32_t item = 0, comb = 0;
+            int64_t prow = 0;
+            p.n_seqs = 0;
+            for (size_t i = lo; i < hi; ++i) {
+                const AttnItem &it = order[i];
+                AttnSeq &q = p.seqs[p.n_seqs++];
+                q.table_row = it.seq * cf.max_pages_per_seq;
+                q.n_pages = static_cast<int32_t>(c->table[it.seq].size());
+                q.q_row0 = it.q_row0;
+                q.n_q = it.n_q;
+                q.n_keys = static_cast<int32_t>(c->len[it.seq]);
+                q.n_qtiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(it.n_q) * g, kBM));
+                const int64_t ktiles = ceil_div(c->len[it.seq], kBN);
+                q.n_splits = split ? static_cast<int32_t>(ceil_div(ktiles, split_tiles)) : 1;
+                q.item0 = item;
+                q.part_row0 = prow;
+                q.comb0 = comb;
+                item += q.n_qtiles * hkv * q.n_splits;
+                if (split) {
+                    prow += static_cast<int64_t>(q.n_qtiles) * hkv * q.n_splits * kBM;
+                    comb += q.n_qtiles * hkv * kBM;
+                }
+            }
+            p.total_items = item;
+            p.total_comb = comb;
+            p.split_tiles = split_tiles;
+            if (!split) break;
+            const int64_t need = prow * (static_cast<int64_t>(d) * 4 + 4);
+            if (need <= c->ws_bytes) {
+                p.part_o = c->d_ws;
+                p.part_lse = c->d_ws + prow * d;
+                break;
+            }
+            if (split_tiles >= max_tiles) {
+                split = false;  // cannot fit any split into the workspace: run unsplit
+                continue;
+            }
+            split_tiles *= 2;
+        }
+        (void)bmq;
+        return PE_OK;
+    };
+
+    std::vector<char> pbuf(sizeof(AttnParams));
+    AttnParams &p = *reinterpret_cast<AttnParams *>(pbuf.data());
+    for (size_t lo = 0; lo < order.size(); lo += kMaxSegs) {
+        const size_t hi = std::min(order.size(), lo + kMaxSegs);
+        bool split = false;
+        s = plan_group(lo, hi, p, split);
+        if (s != PE_OK) return s;
+        cudaError_t e = launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, p, st);
+        if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
+        c->launches++;
+        if (split) {
+            e = launch_splitkv_combine(d, p, st);
+            if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
+            c->launches++;
+        }
+    }
+    return PE_OK;
+}
+
+pe_status check_attn_args(const pe_cache *c, int32_t layer, const void *Q, const void *out, int32_t hq, float scale)
+{
+    if (c->host_only) return fail(PE_ERR_UNSUPPORTED, "attention on a host-only cache");
+    if (layer < 0 || layer >= c->cfg.num_layers) return fail(PE_ERR_RANGE, "layer %d out of range", layer);
+    if (!Q || !out) return fail(PE_ERR_INVALID, "null Q or out");
+    if (!aligned16(Q) || !aligned16(out)) return fail(PE_ERR_INVALID, "Q and out must be 16-byte aligned");
+    if (hq <= 0 || hq % c->cfg.num_kv_heads != 0)
+        return fail(PE_ERR_INVALID, "num_q_heads %d is not a multiple of num_kv_heads %d", hq, c->cfg.num_kv_heads);
+    const int g = hq / c->cfg.num_kv_heads;
+    if (g > kBM || (g & (g - 1)) != 0)
+        return fail(PE_ERR_UNSUPPORTED, "group size %d must be a power of two <= %d", g, kBM);
+    if (!(scale > 0.f) || !std::isfinite(scale)) return fail(PE_ERR_INVALID, "softmax_scale must be positive");
+    return PE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *pe_last_error(void) { return g_err.c_str(); }
+const char *pe_version(void) { return "pe 0.1 (sm_103a)"; }
+
+pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
+{
+    g_err.clear();
+    if (!cfg || !out) return fail(PE_ERR_INVALID, "null argument");
+    *out = nullptr;
+    const pe_cache_config &c = *cfg;
+    if (c.num_layers < 1 || c.num_kv_heads < 1 || c.num_pages < 1 || c.max_seqs < 1 || c.max_pages_per_seq < 1)
+        return fail(PE_ERR_INVALID, "all counts must be positive");
+    if (c.head_dim != 64 && c.head_dim != 128) return fail(PE_ERR_UNSUPPORTED, "head_dim must be 64 or 128");
+    const int ps = c.page_size;
+    if (ps != 8 && ps != 16 && ps != 32 && ps != 64 && ps != 128)
+        return fail(PE_ERR_UNSUPPORTED, "page_size must be 8, 16, 32, 64 or 128");
+    const int64_t pool_rows = static_cast<int64_t>(c.num_layers) * c.num_pages * c.num_kv_heads * ps;
+    if (pool_rows + ps >= INT32_MAX) return fail(PE_ERR_UNSUPPORTED, "pool too large for int32 row coordinates");
+    if (static_cast<int64_t>(c.max_seqs) * c.max_pages_per_seq >= INT32_MAX)
+        return fail(PE_ERR_UNSUPPORTED, "page table too large");
+    if ((c.k_pool == nullptr) != (c.v_pool == nullptr)) return fail(PE_ERR_INVALID, "give both pools or neither");
+    if (c.k_pool && (!aligned16(c.k_pool) || !aligned16(c.v_pool)))
+        return fail(PE_ERR_INVALID, "pools must be 16-byte aligned");
+    std::vector<int32_t> order(c.num_pages);
+    if (c.init_free_order) {
+        std::vector<uint8_t> seen(c.num_pages, 0);
+        for (int i = 0; i < c.num_pages; ++i) {
+            const int32_t pg = c.init_free_order[i];
+            if (pg < 0 || pg >= c.num_pages || seen[pg]) return fail(PE_ERR_INVALID, "init_free_order is not a permutation");
+            seen[pg] = 1;
+            order[i] = pg;
+        }
+    } else {
+        for (int i = 0; i < c.num_pages; ++i) order[i] = i;
+    }
+
+    pe_cache *cc = new (std::nothrow) pe_cache();
+    if (!cc) return fail(PE_ERR_OOM, "host allocation failed");
+    cc->cfg = c;
+    cc->cfg.init_free_order = nullptr;
+    cc->host_only = c.host_only != 0;
+    cc->free_stack.assign(order.rbegin(), order.rend());  // first popped = order[0]
+    cc->table.resize(c.max_seqs);
+    cc->len.assign(c.max_seqs, 0);
+    cc->appended.assign(c.max_seqs, 0);
+    cc->alive.assign(c.max_seqs, 0);
+    cc->pool_rows = pool_rows;
+    if (cc->host_only) {
+        *out = cc;
+        return PE_OK;
+    }
+
+    cudaError_t e = cudaGetDevice(&cc->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&cc->num_sms, cudaDevAttrMultiProcessorCount, cc->device);
+    if (e != cudaSuccess) {
+        delete cc;
+        return cuda_fail(e, "no CUDA device");
+    }
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, cc->device);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, cc->device);
+    if (major != 10) {
+        delete cc;
+        return fail(PE_ERR_UNSUPPORTED, "kernels are built for sm_103a; device is sm_%d%d", major, minor);
+    }
+    const size_t pool_bytes = static_cast<size_t>(pool_rows) * c.head_dim * 2;
+    const size_t table_bytes = static_cast<size_t>(c.max_seqs) * c.max_pages_per_seq * sizeof(int32_t);
+    cc->ws_bytes = c.workspace_bytes > 0 ? c.workspace_bytes : (64ll << 20);
+    pe_status st = PE_OK;
+    do {
+        if (c.k_pool) {
+            cc->k_pool = c.k_pool;
+            cc->v_pool = c.v_pool;
+        } else {
+            cc->own_pools = true;
+            if ((e = cudaMalloc(&cc->k_pool, pool_bytes)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc K pool"); break; }
+            if ((e = cudaMalloc(&cc->v_pool, pool_bytes)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc V pool"); break; }
+            // finite zeros: stale slots read under the causal mask must not hold NaN/Inf
+            if ((e = cudaMemset(cc->k_pool, 0, pool_bytes)) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
+            if ((e = cudaMemset(cc->v_pool, 0, pool_bytes)) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
+        }
+        if ((e = cudaMalloc(&cc->d_table, table_bytes)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc page table"); break; }
+        if ((e = cudaMemset(cc->d_table, 0xFF, table_bytes)) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
+        if ((e = cudaMalloc(&cc->d_len, sizeof(int64_t) * c.max_seqs)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
+        if ((e = cudaMemset(cc->d_len, 0, sizeof(int64_t) * c.max_seqs)) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
+        if ((e = cudaMalloc(&cc->d_status, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
+        if ((e = cudaMemset(cc->d_status, 0, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
+        if ((e = cudaMalloc(&cc->d_ws, cc->ws_bytes)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc workspace"); break; }
+        if ((st = encode_2d(&cc->tm_k, cc->k_pool, c.head_dim, pool_rows, 64, ps)) != PE_OK) break;
+        if ((st = encode_2d(&cc->tm_v, cc->v_pool, c.head_dim, pool_rows, 64, ps)) != PE_OK) break;
+        if ((e = cudaDeviceSynchronize()) != cudaSuccess) { st = cuda_fail(e, "create sync"); break; }
+    } while (false);
+    if (st != PE_OK) {
+        free_device(cc);
+        delete cc;
+        return st;
+    }
+    *out = cc;
+    return PE_OK;
+}
+
+pe_status pe_cache_destroy(pe_cache *cache)
+{
+    if (!cache) return fail(PE_ERR_INVALID, "null cache");
+    if (!cache->host_only) {
+        cudaDeviceSynchronize();
+        free_device(cache);
+    }
+    delete cache;
+    return PE_OK;
+}
+
+pe_status pe_seq_create(pe_cache *c, int32_t *seq_out)
+{
+    if (!c || !seq_out) return fail(PE_ERR_INVALID, "null argument");
+    for (int32_t s = 0; s < c->cfg.max_seqs; ++s) {
+        if (!c->alive[s]) {
+            c->alive[s] = 1;
+            c->table[s].clear();
+            c->len[s] = 0;
+            c->appended[s] = 0;
+            *seq_out = s;
+            return PE_OK;
+        }
+    }
+    return fail(PE_ERR_OOM, "no free sequence slot (max_seqs = %d)", c->cfg.max_seqs);
+}
+
+pe_status pe_seq_release(pe_cache *c, int32_t seq, void *stream)
+{
+    CropPlan pl{};
+    pe_status s = plan_crop(c, seq, 1, &pl);
+    if (s != PE_OK) return s;
+    apply_crop(c, pl, nullptr);
+    c->alive[seq] = 0;
+    return launch_crops(c, {pl}, static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_crop(pe_cache *c, int32_t seq, int64_t tau, int32_t *freed_out, int32_t freed_cap, int32_t *n_freed,
+                  void *stream)
+{
+    CropPlan pl{};
+    pe_status s = plan_crop(c, seq, tau, &pl);
+    if (s != PE_OK) return s;
+    const int32_t nf = pl.old_n - pl.keep;
+    if (freed_out && freed_cap < nf) return fail(PE_ERR_RANGE, "freed_cap %d < %d freed pages", freed_cap, nf);
+    apply_crop(c, pl, freed_out);
+    if (n_freed) *n_freed = nf;
+    return launch_crops(c, {pl}, static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_crop_batch(pe_cache *c, int32_t n, const int32_t *seqs, const int64_t *taus, void *stream)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (n < 0 || (n > 0 && (!seqs || !taus))) return fail(PE_ERR_INVALID, "bad batch arguments");
+    std::vector<CropPlan> plans(n);
+    std::vector<uint8_t> seen(c->cfg.max_seqs, 0);
+    for (int32_t i = 0; i < n; ++i) {
+        pe_status s = plan_crop(c, seqs[i], taus[i], &plans[i]);
+        if (s != PE_OK) return s;
+        if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice in the batch", seqs[i]);
+        seen[seqs[i]] = 1;
+    }
+    for (const CropPlan &pl : plans) apply_crop(c, pl, nullptr);
+    return launch_crops(c, plans, static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_append_kv(pe_cache *c, int32_t seq, const void *K, const void *V, int32_t n_tokens, void *stream)
+{
+    AppendPlan pl{};
+    pe_status s = plan_append(c, seq, n_tokens, &pl);
+    if (s != PE_OK) return s;
+    if (!c->host_only && n_tokens > 0) {
+        if (!K || !V) return fail(PE_ERR_INVALID, "null K or V");
+        if (!aligned16(K) || !aligned16(V)) return fail(PE_ERR_INVALID, "K and V must be 16-byte aligned");
+    }
+    if (pl.need > static_cast<int32_t>(c->free_stack.size()))
+        return fail(PE_ERR_OOM, "append needs %d pages, %zu free", pl.need, c->free_stack.size());
+    pl.tok0 = 0;
+    return apply_appends(c, {pl}, K, V, n_tokens, static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_append_kv_batch(pe_cache *c, int32_t n, const int32_t *seqs, const void *K, const void *V,
+                             const int32_t *cu_tokens, void *stream)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (n < 0 || (n > 0 && (!seqs || !cu_tokens))) return fail(PE_ERR_INVALID, "bad batch arguments");
+    if (n > 0 && cu_tokens[0] != 0) return fail(PE_ERR_INVALID, "cu_tokens[0] must be 0");
+    std::vector<AppendPlan> plans(n);
+    std::vector<uint8_t> seen(c->cfg.max_seqs, 0);
+    int64_t need = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        if (cu_tokens[i + 1] < cu_tokens[i]) return fail(PE_ERR_INVALID, "cu_tokens must be non-decreasing");
+        pe_status s = plan_append(c, seqs[i], cu_tokens[i + 1] - cu_tokens[i], &plans[i]);
+        if (s != PE_OK) return s;
+        if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice in the batch", seqs[i]);
+        seen[seqs[i]] = 1;
+        plans[i].tok0 = cu_tokens[i];
+        need += plans[i].need;
+    }
+    const int64_t total = n > 0 ? cu_tokens[n] : 0;
+    if (!c->host_only && total > 0) {
+        if (!K || !V) return fail(PE_ERR_INVALID, "null K or V");
+        if (!aligned16(K) || !aligned16(V)) return fail(PE_ERR_INVALID, "K and V must be 16-byte aligned");
+    }
+    if (need > static_cast<int64_t>(c->free_stack.size()))
+        return fail(PE_ERR_OOM, "batch append needs %lld pages, %zu free", static_cast<long long>(need),
+                    c->free_stack.size());
+    return apply_appends(c, plans, K, V, total, static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_replay_attn(pe_cache *c, int32_t seq, int32_t layer, const void *Q, void *out, int32_t n_q,
+                         int32_t num_q_heads, float softmax_scale, void *stream)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if ((s = check_attn_args(c, layer, Q, out, num_q_heads, softmax_scale)) != PE_OK) return s;
+    if (n_q < 0) return fail(PE_ERR_INVALID, "negative n_q");
+    if (n_q > c->len[seq])
+        return fail(PE_ERR_RANGE, "n_q = %d exceeds the sequence length %lld", n_q, static_cast<long long>(c->len[seq]));
+    if (n_q == 0) return PE_OK;
+    return run_attention(c, {AttnItem{seq, 0, n_q}}, layer, Q, n_q, out, num_q_heads, softmax_scale,
+                         static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_replay_attn_batch(pe_cache *c, int32_t n, const int32_t *seqs, int32_t layer, const void *Q_packed,
+                               const int32_t *cu_q, void *out, int32_t num_q_heads, float softmax_scale, void *stream)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (n < 0 || (n > 0 && (!seqs || !cu_q))) return fail(PE_ERR_INVALID, "bad batch arguments");
+    if (n == 0) return PE_OK;
+    pe_status s = check_attn_args(c, layer, Q_packed, out, num_q_heads, softmax_scale);
+    if (s != PE_OK) return s;
+    if (cu_q[0] != 0) return fail(PE_ERR_INVALID, "cu_q[0] must be 0");
+    std::vector<AttnItem> items(n);
+    for (int32_t i = 0; i < n; ++i) {
+        if ((s = check_seq(c, seqs[i])) != PE_OK) return s;
+        const int32_t nq = cu_q[i + 1] - cu_q[i];
+        if (nq < 0) return fail(PE_ERR_INVALID, "cu_q must be non-decreasing");
+        if (nq > c->len[seqs[i]])
+            return fail(PE_ERR_RANGE, "sequence %d: n_q = %d exceeds its length %lld", seqs[i], nq,
+                        static_cast<long long>(c->len[seqs[i]]));
+        items[i] = AttnItem{seqs[i], cu_q[i], nq};
+    }
+    if (cu_q[n] == 0) return PE_OK;
+    return run_attention(c, items, layer, Q_packed, cu_q[n], out, num_q_heads, softmax_scale,
+                         static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_seq_info(const pe_cache *c, int32_t seq, int64_t *len, int64_t *appended_since_crop)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if (len) *len = c->len[seq];
+    if (appended_since_crop) *appended_since_crop = c->appended[seq];
+    return PE_OK;
+}
+
+pe_status pe_seq_page_table(const pe_cache *c, int32_t seq, int32_t *out, int32_t cap, int32_t *n)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    const std::vector<int32_t> &t = c->table[seq];
+    if (n) *n = static_cast<int32_t>(t.size());
+    if (out) {
+        if (cap < static_cast<int32_t>(t.size())) return fail(PE_ERR_RANGE, "cap %d < %zu entries", cap, t.size());
+        std::copy(t.begin(), t.end(), out);
+    }
+    return PE_OK;
+}
+
+pe_status pe_free_list(const pe_cache *c, int32_t *out, int32_t cap, int32_t *n)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    const size_t nf = c->free_stack.size();
+    if (n) *n = static_cast<int32_t>(nf);
+    if (out) {
+        if (cap < static_cast<int32_t>(nf)) return fail(PE_ERR_RANGE, "cap %d < %zu free pages", cap, nf);
+        for (size_t i = 0; i < nf; ++i) out[i] = c->free_stack[nf - 1 - i];
+    }
+    return PE_OK;
+}
+
+pe_status pe_seq_device_page_table(pe_cache *c, int32_t seq, int32_t *out, int32_t cap, void *stream)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if (c->host_only) return fail(PE_ERR_UNSUPPORTED, "host-only cache has no device table");
+    if (!out || cap < 0 || cap > c->cfg.max_pages_per_seq) return fail(PE_ERR_INVALID, "bad output buffer");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(out, c->d_table + static_cast<int64_t>(seq) * c->cfg.max_pages_per_seq,
+                       sizeof(int32_t) * cap, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "device page table read");
+    return PE_OK;
+}
+
+pe_status pe_cache_pools(const pe_cache *c, void **k_pool, void **v_pool)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (k_pool) *k_pool = c->k_pool;
+    if (v_pool) *v_pool = c->v_pool;
+    return PE_OK;
+}
+
+pe_status pe_set_option(pe_cache *c, const char *key, int64_t value)
+{
+    if (!c || !key) return fail(PE_ERR_INVALID, "null argument");
+    if (!std::strcmp(key, "splitkv")) {
+        if (value < -1 || value > 1) return fail(PE_ERR_INVALID, "splitkv must be -1, 0 or 1");
+        c->splitkv = static_cast<int>(value);
+    } else if (!std::strcmp(key, "num_splits")) {
+        if (value < 0 || value > 4096) return fail(PE_ERR_INVALID, "num_splits out of range");
+        c->num_splits = static_cast<int>(value);
+    } else if (!std::strcmp(key, "debug_poison")) {
+        c->debug_poison = value ? 1 : 0;
+    } else {
+        return fail(PE_ERR_INVALID, "unknown option '%s'", key);
+    }
+    return PE_OK;
+}
+
+pe_status pe_kernel_launches(const pe_cache *c, int64_t *count)
+{
+    if (!c || !count) return fail(PE_ERR_INVALID, "null argument");
+    *count = c->launches;
+    return PE_OK;
+}
+
+pe_status pe_device_status(pe_cache *c, int32_t *code, int32_t clear, void *stream)
+{
+    if (!c || !code) return fail(PE_ERR_INVALID, "null argument");
+    *code = 0;
+    if (c->host_only) return PE_OK;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemcpy(code, c->d_status, sizeof(int32_t), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && clear) e = cudaMemset(c->d_status, 0, sizeof(int32_t));
+    if (e != cudaSuccess) return cuda_fail(e, "device status read");
+    if (*code != 0) return fail(PE_ERR_DEVICE_TIMEOUT, "a kernel reported status %d", *code);
+    return PE_OK;
+}
+
+}  // extern "C"

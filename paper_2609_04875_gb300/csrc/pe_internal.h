@@ -1,0 +1,100 @@
+// Private to the pe library: kernel parameter blocks shared by the host code
+// (pe_host.cu) and the kernels (pe_kv.cu, pe_attn.cu).
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace pe {
+
+constexpr int kBM = 128;               // query rows (GQA-packed) per attention tile
+constexpr int kBN = 128;               // keys per attention tile
+constexpr int kMaxSegs = 64;           // sequences per append / attention launch
+constexpr int kMaxCropSegs = 256;      // sequences per crop launch
+constexpr int kAppendMaxPages = 3072;  // new page ids carried by one append launch
+
+// Device status word codes (pe_device_status).
+constexpr int kStatusWaitTimeout = 1;
+
+// ---------------------------------------------------------------- append
+struct AppendSeg {
+    int32_t tok0;          // first token of this segment inside the packed K/V
+    int32_t cum0;          // prefix of segment tokens inside this launch
+    int32_t n_tokens;
+    int32_t len0;          // sequence length before this segment
+    int32_t first_new_lp;  // logical index of the first page popped for this segment
+    int32_t last_page;     // physical page holding logical page first_new_lp-1 (-1 if none)
+    int32_t new0;          // offset of this segment's new page ids in new_pages
+    int32_t n_new;
+    int32_t table_row;     // seq * max_pages_per_seq
+    int32_t seq;
+};
+
+struct AppendParams {
+    const uint4 *K;        // packed [L][n_total][Hkv][d] bf16, viewed as 16-byte chunks
+    const uint4 *V;
+    uint4 *k_pool;         // [L][num_pages][Hkv][ps][d]
+    uint4 *v_pool;
+    int32_t *page_table;   // device mirror [max_seqs][max_pages_per_seq]
+    int64_t *seq_len;      // device mirror [max_seqs]
+    int32_t L, hkv, dvec, ps, num_pages, n_total, n_segs, seg_tokens;
+    AppendSeg segs[kMaxSegs];
+    int32_t new_pages[kAppendMaxPages];
+};
+
+// ---------------------------------------------------------------- crop
+struct CropSeg {
+    int32_t table_row;
+    int32_t keep;          // pages kept
+    int32_t old_n;         // pages before the crop
+    int32_t seq;
+    int64_t new_len;
+};
+
+struct CropParams {
+    int32_t *page_table;
+    int64_t *seq_len;
+    uint4 *k_pool;
+    uint4 *v_pool;
+    int32_t n, poison, L, hkv, ps, dvec, num_pages;
+    CropSeg segs[kMaxCropSegs];
+};
+
+// ---------------------------------------------------------------- attention
+struct AttnSeq {
+    int32_t table_row;     // seq * max_pages_per_seq
+    int32_t n_pages;       // ceil(len / ps)
+    int32_t q_row0;        // first row of this sequence in packed Q / out
+    int32_t n_q;
+    int32_t n_keys;        // len
+    int32_t item0;         // first CTA work item of this sequence
+    int32_t n_qtiles;      // ceil(n_q * group / kBM)
+    int32_t n_splits;      // key splits per q-tile (1 without split-KV)
+    int64_t part_row0;     // first partial row in the workspace (split-KV)
+    int32_t comb0;         // first combine row item (split-KV)
+    int32_t pad_;
+};
+
+struct AttnParams {
+    const int32_t *page_table;
+    void *out;             // bf16 [rows][Hq][d]
+    float *part_o;         // split-KV partial outputs [rows][d]
+    float *part_lse;       // split-KV partial log2-sum-exp [rows]
+    int32_t *status;
+    int32_t n_seqs, hq, hkv, group, layer, num_pages, ps, oob_row;
+    int32_t split_tiles;   // key tiles per split
+    int32_t total_items;
+    int32_t total_comb;
+    float scale_log2;      // softmax_scale * log2(e)
+    AttnSeq seqs[kMaxSegs];
+};
+
+// Launchers (defined in the .cu files).
+cudaError_t launch_append(const AppendParams &p, int64_t chunks, cudaStream_t st);
+cudaError_t launch_crop(const CropParams &p, cudaStream_t st);
+cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
+                               const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
+cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);
+
+}  // namespace pe

@@ -1,0 +1,109 @@
+"""Forget-request driver over the C-ABI: turns a workload of agents, each with
+its injection step tau, into the calls of the replay path.
+
+For every agent the original session (T positions, suffix contaminated) is
+first written into one shared paged cache.  One `step()` then performs, for
+all agents at once:
+  1. crop to tau (Alg. 1 Restore; keeps tau-1 tokens)       -> pe_crop_batch
+  2. append the sanitized suffix K'/V' (T-tau+1 positions)   -> pe_append_kv_batch
+  3. replay attention of the suffix queries Q', per layer    -> pe_replay_attn_batch
+After a step every agent again holds T tokens, so steps repeat without reset.
+All inputs are device-resident bf16 tensors; the driver only orders the calls.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from .binding import PagedKVCache
+
+
+def _dev(bits: np.ndarray, device) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
+    return t.to(device)
+
+
+class ReplayDriver:
+    """Device-resident crop + replay of a synthetic workload (``synth.Workload``)."""
+
+    def __init__(self, w, device="cuda", fill=True, cache_kwargs=None):
+        self.w = w
+        self.device = torch.device(device)
+        L, hq, hkv, d = w.num_layers, w.num_q_heads, w.num_kv_heads, w.head_dim
+        self.cache = PagedKVCache(L, hkv, d, w.page_size, w.num_pages, max_seqs=len(w.agents),
+                                  max_pages_per_seq=w.max_pages_per_seq, init_free_order=w.init_free_order(),
+                                  **(cache_kwargs or {}))
+        self.seqs = [self.cache.seq_create() for _ in w.agents]
+        self.taus = [a.tau for a in w.agents]
+        S = [a.S for a in w.agents]
+        self.cu = [0] + list(np.cumsum(S).astype(int))
+        n = self.cu[-1]
+        # sanitized suffix inputs, packed over agents: K'/V' [L][sum S][Hkv][d], Q' [L][sum S][Hq][d]
+        self.Kc = torch.empty((L, n, hkv, d), dtype=torch.bfloat16, device=self.device)
+        self.Vc = torch.empty_like(self.Kc)
+        self.Qc = torch.empty((L, n, hq, d), dtype=torch.bfloat16, device=self.device)
+        for i, a in enumerate(w.agents):
+            k, v = w.kv_counterfactual(a)
+            lo, hi = self.cu[i], self.cu[i + 1]
+            self.Kc[:, lo:hi] = _dev(k, self.device)
+            self.Vc[:, lo:hi] = _dev(v, self.device)
+            self.Qc[:, lo:hi] = _dev(w.q_counterfactual(a), self.device)
+        self.out = torch.empty_like(self.Qc)
+        if fill:
+            self.fill_original()
+
+    def fill_original(self):
+        """Writes every agent's original session (T positions) in agent order."""
+        for s, a in zip(self.seqs, self.w.agents):
+            k, v = self.w.kv_original(a)
+            self.cache.append_kv(s, _dev(k, self.device), _dev(v, self.device))
+        torch.cuda.synchronize(self.device)
+
+    # -- the hot path ------------------------------------------------------------
+    def crop(self, stream=None):
+        self.cache.crop_batch(self.seqs, self.taus, stream=stream)
+
+    def append(self, stream=None):
+        self.cache.append_kv_batch(self.seqs, self.Kc, self.Vc, self.cu, stream=stream)
+
+    def attend(self, layer, stream=None):
+        self.cache.replay_attn_batch(self.seqs, layer, self.Qc[layer], self.cu, out=self.out[layer],
+                                     softmax_scale=self.w.softmax_scale, stream=stream)
+
+    def step(self, stream=None, attn_events=None):
+        """One forget request for every agent.  attn_events: optional list of
+        (start, end) CUDA event pairs, one per layer, recorded around attention."""
+        self.crop(stream)
+        self.append(stream)
+        for layer in range(self.w.num_layers):
+            if attn_events is not None:
+                attn_events[layer][0].record(stream)
+            self.attend(layer, stream)
+            if attn_events is not None:
+                attn_events[layer][1].record(stream)
+        return self.out
+
+    # -- bookkeeping -------------------------------------------------------------
+    def algorithmic_flops(self) -> float:
+        """4 d Hq sum_agents L [S P + S (S + 1) / 2]: unmasked (query, key) pairs x 2d for
+        QK^T and 2d for PV."""
+        w = self.w
+        pairs = sum(a.S * a.P + a.S * (a.S + 1) / 2 for a in w.agents)
+        return 4.0 * w.head_dim * w.num_q_heads * w.num_layers * pairs
+
+    def algorithmic_attn_bytes(self) -> float:
+        """Bytes one attention launch per layer must move: every cached K/V row of
+        each kv-head read once (prefix + suffix), Q read, O written."""
+        w = self.w
+        keys = sum(a.T for a in w.agents)
+        q = sum(a.S for a in w.agents)
+        return 2.0 * (2 * keys * w.num_kv_heads * w.head_dim + 2 * q * w.num_q_heads * w.head_dim)
+
+    def algorithmic_step_bytes(self) -> float:
+        """Per step, all layers: prefix K/V read + new K/V read and written + Q read + O written."""
+        w = self.w
+        P = sum(a.P for a in w.agents)
+        S = sum(a.S for a in w.agents)
+        per_layer = 2.0 * (2 * P * w.num_kv_heads * w.head_dim + 4 * S * w.num_kv_heads * w.head_dim
+                           + 2 * S * w.num_q_heads * w.head_dim)
+        return per_layer * w.num_layers

@@ -9,3 +9,16 @@ for p in (ROOT, os.path.dirname(os.path.abspath(__file__))):
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (runs the CUDA library's kernels)")
+
+
+def pytest_sessionstart(session):
+    # Build (or refresh) the in-tree CUDA library and the C oracle before
+    # collection; both builds are no-ops when up to date.
+    import importlib.util
+    spec = importlib.util.spec_from_file_location(
+        "_pe_build", os.path.join(ROOT, "paper_2609_04875_gb300", "build.py"))
+    pe_build = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(pe_build)
+    pe_build.build()
+    import oracle
+    oracle.build()

@@ -1,0 +1,124 @@
+"""The five workloads at full size, in the launch configuration bench.py times
+(ReplayDriver.step: one batched crop, one batched append, one batched replay
+launch per layer).  Bookkeeping is compared with the oracle in full; attention
+on sampled query rows (first/last rows, tile boundaries, random rows), each
+computed by the oracle from the counterfactual sequence's definition (retained
+prefix of the original session followed by the sanitized suffix)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from gpu_common import assert_close, requires_cuda
+
+pytestmark = [pytest.mark.gpu, requires_cuda]
+
+
+def _rows(w, a, n_random, edge_tiles=4):
+    g = w.num_q_heads // w.num_kv_heads
+    bmq = 128 // g
+    n_tiles = -(-a.S // bmq)
+    rows = {0, a.S - 1}
+    for t in list(range(1, min(edge_tiles, n_tiles))) + list(range(max(1, n_tiles - edge_tiles), n_tiles)):
+        rows.update({t * bmq - 1, t * bmq})
+    r = synth.rng(w.seed, synth.STREAM_SAMPLE, a.index)
+    rows.update(int(x) for x in r.integers(0, a.S, size=n_random))
+    return np.array(sorted(x for x in rows if 0 <= x < a.S), dtype=np.int64)
+
+
+def _check_bookkeeping(drv):
+    w = drv.w
+    orc = oracle.OracleKVCache(w.num_layers, w.num_kv_heads, w.head_dim, w.page_size, w.num_pages,
+                               len(w.agents), w.max_pages_per_seq, init_free_order=w.init_free_order(),
+                               store_values=False)
+    for a in w.agents:
+        s = orc.seq_create()
+        orc.append(s, n_tokens=a.T)
+    for s, a in enumerate(w.agents):
+        orc.crop(s, a.tau)
+    for s, a in enumerate(w.agents):
+        orc.append(s, n_tokens=a.S)
+    assert drv.cache.free_list() == orc.free_list()
+    for s, a in enumerate(w.agents):
+        assert drv.cache.page_table(s) == orc.page_table(s)
+        assert drv.cache.seq_info(s) == (a.T, a.S)          # Corollary 1: T - tau + 1 recomputed
+        tbl = drv.cache.page_table(s)
+        assert drv.cache.device_page_table(s, len(tbl)) == tbl
+
+
+def _check_attention(drv, agents, layers, n_random):
+    w = drv.w
+    worst = (0.0, 0.0)
+    for i in agents:
+        a = w.agents[i]
+        k0, v0 = w.kv_original(a)
+        kc, vc = w.kv_counterfactual(a)
+        qc = w.q_counterfactual(a)
+        rows = _rows(w, a, n_random)
+        for layer in layers:
+            keys = np.concatenate([k0[layer, : a.P], kc[layer]], axis=0)
+            vals = np.concatenate([v0[layer, : a.P], vc[layer]], axis=0)
+            ref = oracle.causal_attention(qc[layer], keys, vals, w.softmax_scale, rows=rows)
+            got = drv.out[layer, drv.cu[i] + torch.from_numpy(rows).cuda()]
+            mx, mean = assert_close(got, ref, f"{w.name} agent {i} layer {layer}")
+            worst = (max(worst[0], mx), max(worst[1], mean))
+    return worst
+
+
+def _run(w):
+    from paper_2609_04875_gb300.driver import ReplayDriver
+    drv = ReplayDriver(w)
+    drv.step()
+    torch.cuda.synchronize()
+    assert drv.cache.device_status() == 0
+    return drv
+
+
+def test_tiny_full():
+    w = synth.tiny()
+    drv = _run(w)
+    _check_bookkeeping(drv)
+    a = w.agents[0]
+    k0, v0 = w.kv_original(a)
+    kc, vc = w.kv_counterfactual(a)
+    qc = w.q_counterfactual(a)
+    ref = oracle.causal_attention(qc[0], np.concatenate([k0[0, : a.P], kc[0]]),
+                                  np.concatenate([v0[0, : a.P], vc[0]]), w.softmax_scale)
+    assert_close(drv.out[0], ref, "tiny (all rows)")
+
+
+def test_agent_batch():
+    w = synth.agent_batch()
+    drv = _run(w)
+    _check_bookkeeping(drv)
+    _check_attention(drv, range(len(w.agents)), [0], n_random=24)
+    # a second step (steady state of the benchmark) gives the same output
+    first = drv.out.clone()
+    drv.step()
+    torch.cuda.synchronize()
+    assert torch.equal(first, drv.out)
+    _check_bookkeeping(drv)
+
+
+def test_short_suffix_splitkv():
+    w = synth.short_suffix()
+    drv = _run(w)
+    _check_bookkeeping(drv)
+    _check_attention(drv, [0, 7], [0], n_random=16)
+    _check_attention(drv, range(1, 7), [0], n_random=2)
+
+
+def test_long_suffix():
+    w = synth.long_suffix()
+    drv = _run(w)
+    _check_bookkeeping(drv)
+    _check_attention(drv, range(len(w.agents)), [0], n_random=32)
+
+
+@pytest.mark.parametrize("ratio", [0.1, 0.9, 0.0])
+def test_tau_sweep(ratio):
+    w = synth.tau_sweep(ratio)
+    drv = _run(w)
+    _check_bookkeeping(drv)
+    _check_attention(drv, [0], [0, w.num_layers - 1], n_random=24)

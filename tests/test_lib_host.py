@@ -1,0 +1,183 @@
+"""libpe on the CPU: it loads, exports every entry point of include/pe.h, and its
+host bookkeeping (free list, page tables, lengths, counters, error codes)
+matches the oracle bit for bit.  Host-only caches run no device work."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+import oracle_pins as pins
+import synth
+
+pe = pytest.importorskip("paper_2609_04875_gb300")
+from paper_2609_04875_gb300 import binding  # noqa: E402
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_symbols():
+    src = open(os.path.join(ROOT, "include", "pe.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(pe_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol():
+    names = declared_symbols()
+    assert "pe_crop" in names and "pe_replay_attn" in names and "pe_cache_create" in names
+    lib = ctypes.CDLL(binding.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in pe.h but not exported"
+    assert set(names) <= set(binding.EXPORTED)
+
+
+def test_version_and_error_string():
+    assert "sm_103a" in pe.version()
+    with pytest.raises(binding.PEError) as e:
+        pe.PagedKVCache(1, 1, 96, 16, 8, 1, 8, host_only=True)
+    assert e.value.kind == "unsupported" and "head_dim" in str(e.value)
+
+
+def _mk(cfg, **kw):
+    return pe.PagedKVCache(cfg["num_layers"], cfg["num_kv_heads"], 64, 8, cfg["num_pages"], cfg["max_seqs"],
+                           cfg["max_pages_per_seq"], init_free_order=cfg.get("init_free_order"), host_only=True, **kw)
+
+
+def test_golden_trace_page_granular():
+    """The hand-derived trace, replayed on libpe (ps = 4 in the trace; libpe needs
+    ps >= 8, so every token count and tau is scaled by 2: same pages, same order)."""
+    trace = pins.load_trace()
+    cfg = trace["config"]
+    c = _mk(cfg)
+    f = 8 // cfg["page_size"]
+    for idx, st in enumerate(trace["steps"]):
+        op = st["op"]
+        try:
+            if op == "create":
+                assert c.seq_create() == st["expect_seq"]
+                continue
+            if op == "append":
+                c.append_kv(st["seq"], n_tokens=st["n"] * f)
+            elif op == "crop":
+                freed = c.crop(st["seq"], (st["tau"] - 1) * f + 1)
+                assert freed == st["expect_freed"], f"step {idx}"
+            elif op == "release":
+                c.seq_release(st["seq"])
+                assert c.free_list() == st["expect_free"], f"step {idx}"
+                continue
+        except binding.PEError as e:
+            assert st.get("expect_error") == e.kind, f"step {idx}: {e}"
+            continue
+        assert "expect_error" not in st, f"step {idx}"
+        if "expect" in st:
+            ex = st["expect"]
+            assert c.page_table(st["seq"]) == ex["table"], f"step {idx}"
+            assert c.seq_info(st["seq"]) == (ex["len"] * f, ex["appended"] * f), f"step {idx}"
+            assert c.free_list() == ex["free"], f"step {idx}"
+
+
+@pytest.mark.parametrize("ps", [8, 16, 64])
+def test_random_ops_match_oracle(ps):
+    num_pages, max_pages = 96, 40
+    order = synth.page_permutation(99 + ps, num_pages)
+    lib = pe.PagedKVCache(2, 2, 64, ps, num_pages, 5, max_pages, init_free_order=order, host_only=True)
+    orc = oracle.OracleKVCache(2, 2, 64, ps, num_pages, 5, max_pages, init_free_order=order, store_values=False)
+    g = synth.rng(7, ps)
+    live = []
+    for step in range(1500):
+        r = g.random()
+        if r < 0.08 or not live:
+            try:
+                s1 = orc.seq_create()
+            except oracle.OracleError as e:
+                with pytest.raises(binding.PEError) as pe_err:
+                    lib.seq_create()
+                assert pe_err.value.kind == e.kind
+                continue
+            assert lib.seq_create() == s1
+            live.append(s1)
+            continue
+        s = live[int(g.integers(0, len(live)))]
+        n = orc.length[s]
+        try:
+            if r < 0.12:
+                orc.seq_release(s)
+                lib.seq_release(s)
+                live.remove(s)
+            elif r < 0.55:
+                tau = int(g.integers(-1, n + 3))
+                try:
+                    want = orc.crop(s, tau)
+                except oracle.OracleError as e:
+                    with pytest.raises(binding.PEError) as pe_err:
+                        lib.crop(s, tau)
+                    assert pe_err.value.kind == e.kind
+                    continue
+                assert lib.crop(s, tau) == want
+            else:
+                k = int(g.integers(0, 5 * ps))
+                try:
+                    orc.append(s, n_tokens=k)
+                except oracle.OracleError as e:
+                    with pytest.raises(binding.PEError) as pe_err:
+                        lib.append_kv(s, n_tokens=k)
+                    assert pe_err.value.kind == e.kind
+                    continue
+                lib.append_kv(s, n_tokens=k)
+        finally:
+            pass
+        assert lib.free_list() == orc.free_list(), f"step {step}"
+        for q in live:
+            assert lib.page_table(q) == orc.page_table(q), f"step {step}"
+            assert lib.seq_info(q) == orc.seq_info(q), f"step {step}"
+
+
+def test_batch_ops_all_or_nothing():
+    c = pe.PagedKVCache(1, 1, 64, 16, 20, 4, 10, host_only=True)
+    a, b = c.seq_create(), c.seq_create()
+    c.append_kv_batch([a, b], cu_tokens=[0, 40, 70])
+    assert c.seq_info(a) == (40, 40) and c.seq_info(b) == (30, 30)
+    state = (c.page_table(a), c.page_table(b), c.free_list())
+    with pytest.raises(binding.PEError) as e:
+        c.crop_batch([a, b], [10, 99])        # second tau out of range
+    assert e.value.kind == "range"
+    with pytest.raises(binding.PEError) as e:
+        c.crop_batch([a, a], [10, 5])         # duplicate sequence
+    assert e.value.kind == "invalid"
+    with pytest.raises(binding.PEError) as e:
+        c.append_kv_batch([a, b], cu_tokens=[0, 16, 16 + 16 * 20])   # OOM on the total
+    assert e.value.kind in ("oom", "range")
+    assert (c.page_table(a), c.page_table(b), c.free_list()) == state
+    c.crop_batch([a, b], [17, 1])
+    assert c.seq_info(a) == (16, 0) and c.seq_info(b) == (0, 0)
+    assert c.page_table(a) == state[0][:1] and c.page_table(b) == []
+
+
+def test_error_codes():
+    c = pe.PagedKVCache(1, 1, 64, 16, 4, 2, 4, host_only=True)
+    s = c.seq_create()
+    c.append_kv(s, n_tokens=20)
+    for tau, kind in ((0, "invalid"), (22, "range")):
+        with pytest.raises(binding.PEError) as e:
+            c.crop(s, tau)
+        assert e.value.kind == kind
+    with pytest.raises(binding.PEError) as e:
+        c.crop(3, 1)
+    assert e.value.kind == "invalid"
+    with pytest.raises(binding.PEError) as e:
+        c.append_kv(s, n_tokens=16 * 4)      # 84 tokens > 4 pages
+    assert e.value.kind == "range"
+    t = c.seq_create()
+    c.append_kv(t, n_tokens=30)
+    with pytest.raises(binding.PEError) as e:
+        c.append_kv(t, n_tokens=3)           # pool exhausted (2 + 2 pages used)
+    assert e.value.kind == "oom"
+    assert c.seq_info(t) == (30, 30)
+    with pytest.raises(binding.PEError) as e:
+        c.set_option("nonsense", 1)
+    assert e.value.kind == "invalid"
+    with pytest.raises(binding.PEError) as e:
+        pe.PagedKVCache(1, 1, 64, 16, 4, 2, 4, init_free_order=[0, 1, 1, 2], host_only=True)
+    assert e.value.kind == "invalid"
