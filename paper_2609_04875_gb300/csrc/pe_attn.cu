@@ -6,16 +6,23 @@
 // 0..len-n_q+i of kv-head h / (Hq/Hkv):
 //     O = softmax(scale * q K^T) V      (bf16 in, fp32 accumulate, bf16 out)
 //
-// One CTA computes one work item: (sequence, kv-head, q-tile[, key split]).
-// A q-tile packs 128 rows = (128/g queries) x (g q-heads of one kv-head), so K
-// and V tiles are read once for the whole GQA group.  Roles (192 threads):
-//   warps 0-3  softmax: thread r owns row r (TMEM lane r); masks, online
-//              softmax in fp32 (exp2), writes P (bf16) to shared memory,
-//              rescales O in TMEM when needed, epilogue.
-//   warp 4     producer: reads the page table and issues one TMA box per
-//              (page, 64-column half) into a K/V stage ring.
-//   warp 5     MMA: allocates TMEM; one thread issues tcgen05.mma for
-//              S = Q K^T (TMEM, double-buffered) and O += P V (TMEM).
+// One CTA computes one work item: (sequence, kv-head, pair of q-tiles[, key
+// split]).  A q-tile packs 128 rows = (128/g queries) x (g q-heads of one
+// kv-head), so each K/V tile brought into shared memory serves 2 x 128 rows.
+// Roles (320 threads):
+//   warps 0-3, 4-7  softmax of q-tile 0 / q-tile 1: thread r owns row r
+//                   (TMEM lane r); masks, online softmax in fp32 (exp2),
+//                   writes P (bf16) back into TMEM over its S columns,
+//                   rescales O in TMEM when needed, epilogue.
+//   warp 8          producer: reads the page table; its lanes issue one TMA
+//                   box per (page, 64-column half) into K and V stage rings.
+//   warp 9          MMA: allocates TMEM; one thread issues tcgen05.mma for
+//                   S_t = Q_t K^T (A, B from shared memory) and
+//                   O_t += P_t V (A = P from TMEM, B = V from shared memory).
+// Tensor-core order per key tile j:  PV_0(j), S_0(j+1), PV_1(j), S_1(j+1), so
+// one softmax group works while the tensor core runs the other group's GEMMs.
+// TMEM columns: S_0 [0,128), S_1 [128,256), O_0 and O_1 (HD each) from 256.
+//
 // Key tiles always start at logical key 0 (multiples of 128 keys), whatever
 // the physical pages, so a row's arithmetic depends only on its own keys.
 //
@@ -35,30 +42,25 @@ namespace pe {
 
 constexpr uint64_t kWaitNs = 1000000000ull;  // 1 s
 constexpr float kRescaleThreshold = 8.0f;    // log2 units
+constexpr int kThreads = 320;
 
 template <int HD>
 struct AttnCfg {
     static constexpr int kRegions = HD / 64;            // 128-byte swizzle atoms along d
     static constexpr int kTileBytes = kBM * HD * 2;     // one Q, K or V tile (128 rows)
     static constexpr int kRegionBytes = kBM * 128;      // 128 rows x 128 bytes
-    static constexpr int kStages = (HD == 128) ? 2 : 4;
-    static constexpr int kPBytes = kBM * kBN * 2;       // P tile: 128 rows x 128 keys bf16
-    static constexpr int kOffQ = 0;
-    static constexpr int kOffK = kOffQ + kTileBytes;
+    static constexpr int kStages = (HD == 128) ? 2 : 3; // K ring and V ring depth
+    static constexpr int kOffQ = 0;                     // Q_0, Q_1
+    static constexpr int kOffK = kOffQ + 2 * kTileBytes;
     static constexpr int kOffV = kOffK + kStages * kTileBytes;
-    static constexpr int kOffP = kOffV + kStages * kTileBytes;
-    static constexpr int kOffBar = kOffP + 2 * kPBytes;
-    // barriers: q_full, k_full[S], v_full[S], kv_empty[S], s_full[2], s_free[2], p_full[2], pv_done[2]
-    static constexpr int kNumBars = 1 + 3 * kStages + 8;
+    static constexpr int kOffBar = kOffV + kStages * kTileBytes;
+    // barriers: q_full, k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_full[2], o_done[2]
+    static constexpr int kNumBars = 1 + 4 * kStages + 6;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort flag
     static constexpr int kSmemBytes = kOffMisc + 16;
     static constexpr int kDynSmem = kSmemBytes + 1024;       // alignment slack
-    static constexpr uint32_t kTmemCols = 512;               // S0 | S1 | O
+    static constexpr uint32_t kTmemCols = 512;
     static_assert(kDynSmem <= 232448, "shared memory budget");
-};
-
-struct Bars {
-    uint32_t q_full, k_full0, v_full0, kv_empty0, s_full0, s_free0, p_full0, pv_done0;
 };
 
 struct WaitCtx {
@@ -99,20 +101,89 @@ __device__ __forceinline__ float ex2(float x)
     return y;
 }
 
+__device__ __forceinline__ float max3(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// (a*b + c) on two fp32 lanes at once
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c)
+{
+    uint64_t ra, rb, rc, rd;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(rc) : "f"(c.x), "f"(c.y));
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(rd) : "l"(ra), "l"(rb), "l"(rc));
+    float2 d;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+    return d;
+}
+
+__device__ __forceinline__ float2 add2(float2 a, float2 b)
+{
+    uint64_t ra, rb, rd;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(ra) : "f"(a.x), "f"(a.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(rb) : "f"(b.x), "f"(b.y));
+    asm("add.f32x2 %0, %1, %2;" : "=l"(rd) : "l"(ra), "l"(rb));
+    float2 d;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(d.x), "=f"(d.y) : "l"(rd));
+    return d;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t *>(&h);
 }
 
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
+// 32 lanes x 16 consecutive 32-bit TMEM columns from registers.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16])
 {
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
-                 : "memory");
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
 }
 
+// 32 lanes x 16 consecutive 32-bit TMEM columns into registers.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr)
+        : "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem] (A = P, bf16 packed two per column).
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Per q-tile geometry of a work item.
+struct TileGeo {
+    int qt;          // q-tile index within the sequence (-1: absent)
+    int q_first;     // first query of the tile
+    int q_last;      // last valid query of the tile
+    int pos_first;   // absolute position of the first query
+    int ntiles;      // key tiles this q-tile processes (from kt0)
+};
+
 template <int HD, bool SPLIT>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     replay_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                        const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ AttnParams p)
 {
@@ -125,73 +196,83 @@ __global__ void __launch_bounds__(192, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
 
-    // ---- work item -> (sequence, kv-head, split, q-tile); heaviest q-tiles first
+    // ---- work item -> (sequence, kv-head, split, q-tile pair); heaviest pairs first
     const int item = blockIdx.x;
     int si = 0;
     while (si + 1 < p.n_seqs && item >= p.seqs[si + 1].item0) ++si;
     const AttnSeq &sq = p.seqs[si];
+    const int n_pairs = (sq.n_qtiles + 1) >> 1;
     int local = item - sq.item0;
     const int kvh = local % p.hkv;
     local /= p.hkv;
     const int split = local % sq.n_splits;
     local /= sq.n_splits;
-    const int qt = sq.n_qtiles - 1 - local;
+    const int pair = n_pairs - 1 - local;
     const int g = p.group;
     const int bmq = kBM / g;
-    const int q_first = qt * bmq;
-    const int q_last = min(q_first + bmq, sq.n_q) - 1;
-    const int pos_first = sq.n_keys - sq.n_q + q_first;   // position of the tile's first query
-    const int k_end = sq.n_keys - sq.n_q + q_last + 1;    // keys needed by the tile's last query
-    const int nkt = (k_end + kBN - 1) / kBN;
-    int kt0 = 0, kt1 = nkt;
-    if (SPLIT) {
-        kt0 = split * p.split_tiles;
-        kt1 = min(nkt, kt0 + p.split_tiles);
+    const int kt0 = SPLIT ? split * p.split_tiles : 0;
+    TileGeo geo[2];
+#pragma unroll
+    for (int t = 0; t < 2; ++t) {
+        const int qt = 2 * pair + t;
+        TileGeo &G = geo[t];
+        if (qt < sq.n_qtiles) {
+            G.qt = qt;
+            G.q_first = qt * bmq;
+            G.q_last = min(G.q_first + bmq, sq.n_q) - 1;
+            G.pos_first = sq.n_keys - sq.n_q + G.q_first;
+            const int k_end = sq.n_keys - sq.n_q + G.q_last + 1;
+            const int nkt = (k_end + kBN - 1) / kBN;
+            const int kt1 = SPLIT ? min(nkt, kt0 + p.split_tiles) : nkt;
+            G.ntiles = max(0, kt1 - kt0);
+        } else {
+            G.qt = -1;
+            G.q_first = G.q_last = G.pos_first = 0;
+            G.ntiles = 0;
+        }
     }
-    const int ntiles = max(0, kt1 - kt0);
+    const int n_all = max(geo[0].ntiles, geo[1].ntiles);  // key tiles loaded for the pair
 
     // ---- shared memory carve-up
     const uint32_t q_smem = sbase + C::kOffQ;
     const uint32_t k_smem0 = sbase + C::kOffK;
     const uint32_t v_smem0 = sbase + C::kOffV;
-    const uint32_t p_smem0 = sbase + C::kOffP;
     const uint32_t bar0 = sbase + C::kOffBar;
-    Bars B;
-    B.q_full = bar0;
-    B.k_full0 = bar0 + 8;
-    B.v_full0 = B.k_full0 + 8 * C::kStages;
-    B.kv_empty0 = B.v_full0 + 8 * C::kStages;
-    B.s_full0 = B.kv_empty0 + 8 * C::kStages;
-    B.s_free0 = B.s_full0 + 16;
-    B.p_full0 = B.s_free0 + 16;
-    B.pv_done0 = B.p_full0 + 16;
+    const uint32_t b_q_full = bar0;
+    const uint32_t b_k_full = bar0 + 8;
+    const uint32_t b_k_empty = b_k_full + 8 * C::kStages;
+    const uint32_t b_v_full = b_k_empty + 8 * C::kStages;
+    const uint32_t b_v_empty = b_v_full + 8 * C::kStages;
+    const uint32_t b_s_full = b_v_empty + 8 * C::kStages;  // [2]
+    const uint32_t b_p_full = b_s_full + 16;               // [2]
+    const uint32_t b_o_done = b_p_full + 16;               // [2]
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 4);
     const WaitCtx wctx{abort_flag, p.status};
 
     if (threadIdx.x == 0) {
-        ptx::mbar_init(B.q_full, 1);
+        ptx::mbar_init(b_q_full, 1);
         for (int s = 0; s < C::kStages; ++s) {
-            ptx::mbar_init(B.k_full0 + 8 * s, 1);
-            ptx::mbar_init(B.v_full0 + 8 * s, 1);
-            ptx::mbar_init(B.kv_empty0 + 8 * s, 1);
+            ptx::mbar_init(b_k_full + 8 * s, 1);
+            ptx::mbar_init(b_k_empty + 8 * s, 1);
+            ptx::mbar_init(b_v_full + 8 * s, 1);
+            ptx::mbar_init(b_v_empty + 8 * s, 1);
         }
-        for (int b = 0; b < 2; ++b) {
-            ptx::mbar_init(B.s_full0 + 8 * b, 1);
-            ptx::mbar_init(B.s_free0 + 8 * b, 128);
-            ptx::mbar_init(B.p_full0 + 8 * b, 128);
-            ptx::mbar_init(B.pv_done0 + 8 * b, 1);
+        for (int t = 0; t < 2; ++t) {
+            ptx::mbar_init(b_s_full + 8 * t, 1);
+            ptx::mbar_init(b_p_full + 8 * t, 128);
+            ptx::mbar_init(b_o_done + 8 * t, 1);
         }
         *abort_flag = 0;
         ptx::fence_barrier_init();
         ptx::fence_proxy_async_smem();
     }
-    if (warp == 4 && lane == 0) {
+    if (warp == 8 && lane == 0) {
         ptx::prefetch_tensormap(&tm_q);
         ptx::prefetch_tensormap(&tm_k);
         ptx::prefetch_tensormap(&tm_v);
     }
-    if (warp == 5) {
+    if (warp == 9) {
         ptx::tmem_alloc(ptx::smem_addr(tmem_slot), C::kTmemCols);
         ptx::tmem_relinquish();
     }
@@ -199,159 +280,181 @@ __global__ void __launch_bounds__(192, 1)
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    const uint32_t tS0 = tmem;          // S buffer b at column 128*b
-    const uint32_t tO = tmem + 256;     // O accumulator: HD columns
 
-    if (ntiles > 0 && warp == 4) {
+    if (warp == 8 && n_all > 0) {
         // =================================================== producer (TMA)
         if (lane == 0) {
-            ptx::mbar_arrive_expect_tx(B.q_full, C::kTileBytes);
-            for (int r = 0; r < C::kRegions; ++r)
-                ptx::tma_load_3d(q_smem + r * C::kRegionBytes, &tm_q, r * 64, kvh * g, sq.q_row0 + q_first,
-                                 B.q_full);
+            const int nq = geo[1].qt >= 0 ? 2 : 1;
+            ptx::mbar_arrive_expect_tx(b_q_full, nq * C::kTileBytes);
+            for (int t = 0; t < nq; ++t)
+                for (int r = 0; r < C::kRegions; ++r)
+                    ptx::tma_load_3d(q_smem + t * C::kTileBytes + r * C::kRegionBytes, &tm_q, r * 64, kvh * g,
+                                     sq.q_row0 + geo[t].q_first, b_q_full);
         }
-        const int ppt = kBN / p.ps;  // pages per key tile
-        for (int i = 0; i < ntiles; ++i) {
+        const int ppt = kBN / p.ps;                 // pages per key tile
+        const int n_ops = ppt * C::kRegions;        // TMA boxes per K (or V) tile, <= 32
+        const int op_page = lane / C::kRegions;     // this lane's box: page index and half
+        const int op_reg = lane % C::kRegions;
+        const bool op_on = lane < n_ops;
+        const uint32_t op_off = op_reg * C::kRegionBytes + op_page * p.ps * 128;
+        int page_next = -1;
+        {
+            const int lp = kt0 * ppt + lane;
+            if (lane < ppt && lp < sq.n_pages) page_next = p.page_table[sq.table_row + lp];
+        }
+        for (int i = 0; i < n_all; ++i) {
             const int s = i % C::kStages;
-            if (i >= C::kStages && !wait_bar_warp(B.kv_empty0 + 8 * s, ((i / C::kStages) - 1) & 1, wctx)) break;
-            const int lp = (kt0 + i) * ppt + lane;
-            int page = -1;
-            if (lane < ppt && lp < sq.n_pages) page = p.page_table[sq.table_row + lp];
-            const uint32_t kdst = k_smem0 + s * C::kTileBytes;
-            const uint32_t vdst = v_smem0 + s * C::kTileBytes;
-            if (lane == 0) {
-                ptx::mbar_arrive_expect_tx(B.k_full0 + 8 * s, C::kTileBytes);
-                ptx::mbar_arrive_expect_tx(B.v_full0 + 8 * s, C::kTileBytes);
+            const int page = page_next;
+            if (i + 1 < n_all) {  // prefetch the next tile's page ids
+                const int lp = (kt0 + i + 1) * ppt + lane;
+                page_next = (lane < ppt && lp < sq.n_pages) ? p.page_table[sq.table_row + lp] : -1;
             }
-            for (int j = 0; j < ppt; ++j) {
-                const int pg = __shfl_sync(0xffffffffu, page, j);
-                if (lane == 0) {
-                    // rows of pages past the sequence read as zeros (out-of-bounds box)
-                    const int y = pg >= 0 ? ((p.layer * p.num_pages + pg) * p.hkv + kvh) * p.ps : p.oob_row;
-                    for (int r = 0; r < C::kRegions; ++r) {
-                        const uint32_t off = r * C::kRegionBytes + j * p.ps * 128;
-                        ptx::tma_load_2d(kdst + off, &tm_k, r * 64, y, B.k_full0 + 8 * s);
-                        ptx::tma_load_2d(vdst + off, &tm_v, r * 64, y, B.v_full0 + 8 * s);
-                    }
-                }
-            }
+            const int pg = __shfl_sync(0xffffffffu, page, op_page & 31);
+            // rows of pages past the sequence read as zeros (out-of-bounds box)
+            const int y = pg >= 0 ? ((p.layer * p.num_pages + pg) * p.hkv + kvh) * p.ps : p.oob_row;
+            if (i >= C::kStages && !wait_bar_warp(b_k_empty + 8 * s, ((i / C::kStages) - 1) & 1, wctx)) break;
+            if (lane == 0) ptx::mbar_arrive_expect_tx(b_k_full + 8 * s, C::kTileBytes);
+            __syncwarp();
+            if (op_on) ptx::tma_load_2d(k_smem0 + s * C::kTileBytes + op_off, &tm_k, op_reg * 64, y, b_k_full + 8 * s);
+            if (i >= C::kStages && !wait_bar_warp(b_v_empty + 8 * s, ((i / C::kStages) - 1) & 1, wctx)) break;
+            if (lane == 0) ptx::mbar_arrive_expect_tx(b_v_full + 8 * s, C::kTileBytes);
+            __syncwarp();
+            if (op_on) ptx::tma_load_2d(v_smem0 + s * C::kTileBytes + op_off, &tm_v, op_reg * 64, y, b_v_full + 8 * s);
         }
         __syncwarp();
         if (*abort_flag && lane == 0) {
             // give copies in flight a bounded chance to land before the CTA exits
-            const int first = max(0, ntiles - C::kStages);
-            for (int i = first; i < ntiles; ++i) {
+            const uint64_t t0 = ptx::globaltimer();
+            for (int i = max(0, n_all - C::kStages); i < n_all; ++i) {
                 const int s = i % C::kStages;
-                const uint64_t t0 = ptx::globaltimer();
-                while (!ptx::mbar_try_wait(B.k_full0 + 8 * s, (i / C::kStages) & 1) &&
-                       ptx::globaltimer() - t0 < 1000000ull) {}
-                while (!ptx::mbar_try_wait(B.v_full0 + 8 * s, (i / C::kStages) & 1) &&
+                while (!ptx::mbar_try_wait(b_k_full + 8 * s, (i / C::kStages) & 1) &&
                        ptx::globaltimer() - t0 < 2000000ull) {}
+                while (!ptx::mbar_try_wait(b_v_full + 8 * s, (i / C::kStages) & 1) &&
+                       ptx::globaltimer() - t0 < 4000000ull) {}
             }
         }
-    } else if (ntiles > 0 && warp == 5) {
+    } else if (warp == 9 && n_all > 0) {
         // =================================================== MMA issuer
         if (lane == 0) {
             constexpr uint32_t kIdescQK = ptx::idesc_bf16_f32(kBM, kBN, false);
             constexpr uint32_t kIdescPV = ptx::idesc_bf16_f32(kBM, HD, true);
-            bool ok = wait_bar(B.q_full, 0, wctx);
-            auto issue_pv = [&](int i) -> bool {
-                const int s = i % C::kStages;
-                const int b = i & 1;
-                if (!wait_bar(B.p_full0 + 8 * b, (i >> 1) & 1, wctx)) return false;
-                if (!wait_bar(B.v_full0 + 8 * s, (i / C::kStages) & 1, wctx)) return false;
-                ptx::tc_fence_after();
-                const uint32_t pa = p_smem0 + b * C::kPBytes;
-                const uint32_t vb = v_smem0 + s * C::kTileBytes;
-#pragma unroll
-                for (int kk = 0; kk < kBN / 16; ++kk) {
-                    const uint64_t da = ptx::smem_desc_sw128(pa + (kk >> 2) * C::kRegionBytes + (kk & 3) * 32, 16, 1024);
-                    const uint64_t db = ptx::smem_desc_sw128(vb + kk * 16 * 128, C::kRegionBytes, 1024);
-                    ptx::mma_bf16(tO, da, db, kIdescPV, (i > 0 || kk > 0) ? 1u : 0u);
-                }
-                ptx::mma_commit(B.kv_empty0 + 8 * s);
-                ptx::mma_commit(B.pv_done0 + 8 * b);
-                return true;
-            };
-            for (int i = 0; ok && i < ntiles; ++i) {
-                const int s = i % C::kStages;
-                const int b = i & 1;
-                if (!wait_bar(B.k_full0 + 8 * s, (i / C::kStages) & 1, wctx)) { ok = false; break; }
-                if (i >= 2 && !wait_bar(B.s_free0 + 8 * b, ((i >> 1) - 1) & 1, wctx)) { ok = false; break; }
-                ptx::tc_fence_after();
+            const int n0 = geo[0].ntiles, n1 = geo[1].ntiles;
+            auto issue_s = [&](int t, int s) {
+                const uint32_t qa = q_smem + t * C::kTileBytes;
                 const uint32_t kb = k_smem0 + s * C::kTileBytes;
 #pragma unroll
                 for (int kk = 0; kk < HD / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * C::kRegionBytes + (kk & 3) * 32;
-                    const uint64_t da = ptx::smem_desc_sw128(q_smem + off, 16, 1024);
-                    const uint64_t db = ptx::smem_desc_sw128(kb + off, 16, 1024);
-                    ptx::mma_bf16(tS0 + 128 * b, da, db, kIdescQK, kk > 0 ? 1u : 0u);
+                    ptx::mma_bf16(tmem + 128 * t, ptx::smem_desc_sw128(qa + off, 16, 1024),
+                                  ptx::smem_desc_sw128(kb + off, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
                 }
-                ptx::mma_commit(B.s_full0 + 8 * b);
-                if (i >= 1 && !issue_pv(i - 1)) { ok = false; break; }
+                ptx::mma_commit(b_s_full + 8 * t);
+            };
+            auto issue_pv = [&](int t, int s, bool acc) {
+                const uint32_t vb = v_smem0 + s * C::kTileBytes;
+#pragma unroll
+                for (int kk = 0; kk < kBN / 16; ++kk)
+                    mma_bf16_ts(tmem + 256 + HD * t, tmem + 128 * t + kk * 8,
+                                ptx::smem_desc_sw128(vb + kk * 16 * 128, C::kRegionBytes, 1024), kIdescPV,
+                                (acc || kk > 0) ? 1u : 0u);
+                ptx::mma_commit(b_o_done + 8 * t);
+            };
+            bool ok = wait_bar(b_q_full, 0, wctx) && wait_bar(b_k_full, 0, wctx);
+            if (ok) {
+                ptx::tc_fence_after();
+                if (n0 > 0) issue_s(0, 0);
+                if (n1 > 0) issue_s(1, 0);
+                if (n0 > 0 || n1 > 0) ptx::mma_commit(b_k_empty);
             }
-            if (ok) issue_pv(ntiles - 1);
+            for (int j = 0; ok && j < n_all; ++j) {
+                const int s = j % C::kStages;
+                const int s1 = (j + 1) % C::kStages;
+                const bool more = j + 1 < n_all;
+                if (!wait_bar(b_v_full + 8 * s, (j / C::kStages) & 1, wctx)) { ok = false; break; }
+                if (j < n0) {
+                    if (!wait_bar(b_p_full, j & 1, wctx)) { ok = false; break; }
+                    ptx::tc_fence_after();
+                    issue_pv(0, s, j > 0);
+                }
+                if (more && !wait_bar(b_k_full + 8 * s1, ((j + 1) / C::kStages) & 1, wctx)) { ok = false; break; }
+                ptx::tc_fence_after();
+                if (j + 1 < n0) issue_s(0, s1);
+                if (j < n1) {
+                    if (!wait_bar(b_p_full + 8, j & 1, wctx)) { ok = false; break; }
+                    ptx::tc_fence_after();
+                    issue_pv(1, s, j > 0);
+                }
+                if (j + 1 < n1) issue_s(1, s1);
+                if (more) ptx::mma_commit(b_k_empty + 8 * s1);  // K of tile j+1 consumed by its S GEMMs
+                ptx::mma_commit(b_v_empty + 8 * s);              // V of tile j consumed by its PV GEMMs
+            }
         }
         __syncwarp();
-    } else if (warp < 4) {
+    } else if (warp < 8) {
         // =================================================== softmax / epilogue
-        const int row = threadIdx.x;  // TMEM lane
-        const int qi = q_first + row / g;
-        const bool valid = qi <= q_last;
+        const int t = warp >> 2;                 // q-tile of this warpgroup
+        const TileGeo &G = geo[t];
+        const int row = threadIdx.x & 127;       // TMEM lane
+        const int qi = G.q_first + row / g;
+        const bool valid = G.qt >= 0 && qi <= G.q_last;
         const int pos = sq.n_keys - sq.n_q + qi;
-        const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+        const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+        const uint32_t tS = tmem + 128 * t + lane_off;
+        const uint32_t tO = tmem + 256 + HD * t + lane_off;
+        const uint32_t b_s = b_s_full + 8 * t, b_p = b_p_full + 8 * t, b_o = b_o_done + 8 * t;
         const float sl2 = p.scale_log2;
+        const float2 sl2x2 = make_float2(sl2, sl2);
         float m_ref = -INFINITY;
         float l = 0.f;
         bool ok = true;
-        for (int i = 0; i < ntiles; ++i) {
-            const int b = i & 1;
-            const int kbase = (kt0 + i) * kBN;
-            if (!wait_bar_warp(B.s_full0 + 8 * b, (i >> 1) & 1, wctx)) { ok = false; break; }
+        for (int j = 0; j < G.ntiles; ++j) {
+            const int kbase = (kt0 + j) * kBN;
+            if (!wait_bar_warp(b_s, j & 1, wctx)) { ok = false; break; }
             ptx::tc_fence_after();
-            __syncwarp();
             float s[kBN];
             {
                 float (&s0)[32] = *reinterpret_cast<float (*)[32]>(&s[0]);
                 float (&s1)[32] = *reinterpret_cast<float (*)[32]>(&s[32]);
                 float (&s2)[32] = *reinterpret_cast<float (*)[32]>(&s[64]);
                 float (&s3)[32] = *reinterpret_cast<float (*)[32]>(&s[96]);
-                const uint32_t ts = tS0 + 128 * b + lane_off;
-                ptx::tmem_ld32(ts + 0, s0);
-                ptx::tmem_ld32(ts + 32, s1);
-                ptx::tmem_ld32(ts + 64, s2);
-                ptx::tmem_ld32(ts + 96, s3);
+                ptx::tmem_ld32(tS + 0, s0);
+                ptx::tmem_ld32(tS + 32, s1);
+                ptx::tmem_ld32(tS + 64, s2);
+                ptx::tmem_ld32(tS + 96, s3);
                 ptx::tmem_wait_ld();
             }
-            ptx::tc_fence_before();
-            ptx::mbar_arrive(B.s_free0 + 8 * b);
-            if (kbase + kBN - 1 > pos_first) {  // tile crosses the causal diagonal of some row
+            if (kbase + kBN - 1 > G.pos_first) {  // tile crosses the causal diagonal of some row
 #pragma unroll
                 for (int c = 0; c < kBN; ++c)
                     if (kbase + c > pos) s[c] = -INFINITY;
             }
-            float mx = -INFINITY;
+            // row max: 8 independent chains of 3-input max, then a tree
+            float mx[8];
 #pragma unroll
-            for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, s[c]);
-            const float m_new = fmaxf(m_ref, mx * sl2);
-            if (i == 0) {
+            for (int k = 0; k < 8; ++k) mx[k] = fmaxf(s[k], s[8 + k]);
+#pragma unroll
+            for (int c = 16; c < kBN; c += 16)
+#pragma unroll
+                for (int k = 0; k < 8; ++k) mx[k] = max3(mx[k], s[c + k], s[c + 8 + k]);
+            const float mt = fmaxf(max3(mx[0], mx[1], mx[2]), max3(max3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
+            const float m_new = fmaxf(m_ref, mt * sl2);
+            if (j == 0) {
                 m_ref = (m_new == -INFINITY) ? 0.f : m_new;
             } else {
                 const bool need = m_new > m_ref + kRescaleThreshold;
                 if (__any_sync(0xffffffffu, need)) {
-                    // O holds PV of tiles < i once PV_{i-1} completed; PV_i waits for our P
-                    if (!wait_bar_warp(B.pv_done0 + 8 * ((i - 1) & 1), ((i - 1) >> 1) & 1, wctx)) { ok = false; break; }
+                    // O holds PV of tiles < j once PV(j-1) completed; PV(j) waits for our P
+                    if (!wait_bar_warp(b_o, (j - 1) & 1, wctx)) { ok = false; break; }
                     ptx::tc_fence_after();
-                    __syncwarp();
                     const float alpha = need ? ex2(m_ref - m_new) : 1.0f;
-#pragma unroll
-                    for (int ch = 0; ch < HD / 32; ++ch) {
-                        float o[32];
-                        ptx::tmem_ld32(tO + lane_off + ch * 32, o);
+#pragma unroll 1
+                    for (int ch = 0; ch < HD / 16; ++ch) {
+                        uint32_t o[16];
+                        tmem_ld16(tO + ch * 16, o);
                         ptx::tmem_wait_ld();
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) o[j] *= alpha;
-                        ptx::tmem_st32(tO + lane_off + ch * 32, o);
+                        for (int k = 0; k < 16; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * alpha);
+                        tmem_st16(tO + ch * 16, o);
                     }
                     ptx::tmem_wait_st();
                     if (need) {
@@ -360,91 +463,88 @@ __global__ void __launch_bounds__(192, 1)
                     }
                 }
             }
-            // P buffer b is free once PV_{i-2} completed
-            if (i >= 2 && !wait_bar_warp(B.pv_done0 + 8 * b, ((i >> 1) - 1) & 1, wctx)) { ok = false; break; }
-            const float neg_ref = -m_ref;
-            float rs = 0.f;
-            const uint32_t prow = p_smem0 + b * C::kPBytes + row * 128;
+            // P = exp2(s * scale_log2 - m_ref) as bf16 pairs, written over S's first 64 columns
+            const float2 nref = make_float2(-m_ref, -m_ref);
+            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                             make_float2(0.f, 0.f)};
 #pragma unroll
-            for (int cidx = 0; cidx < kBN / 8; ++cidx) {
-                float e[8];
+            for (int ch = 0; ch < kBN / 32; ++ch) {
+                uint32_t pk[16];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    e[j] = ex2(fmaf(s[cidx * 8 + j], sl2, neg_ref));
-                    rs += e[j];
+                for (int k = 0; k < 16; ++k) {
+                    const int c = ch * 32 + 2 * k;
+                    const float2 x = fma2(make_float2(s[c], s[c + 1]), sl2x2, nref);
+                    const float2 e = make_float2(ex2(x.x), ex2(x.y));
+                    acc[k & 3] = add2(acc[k & 3], e);
+                    pk[k] = pack_bf16(e.x, e.y);
                 }
-                const uint32_t addr = prow + (cidx >> 3) * C::kRegionBytes + ((((cidx & 7) ^ (row & 7))) << 4);
-                st_shared_v4(addr, pack_bf16(e[0], e[1]), pack_bf16(e[2], e[3]), pack_bf16(e[4], e[5]),
-                             pack_bf16(e[6], e[7]));
+                tmem_st16(tS + ch * 16, pk);
             }
-            l += rs;
-            ptx::fence_proxy_async_smem();
+            const float2 a01 = add2(acc[0], acc[1]);
+            const float2 a23 = add2(acc[2], acc[3]);
+            const float2 a = add2(a01, a23);
+            l += a.x + a.y;
+            ptx::tmem_wait_st();
             ptx::tc_fence_before();
-            ptx::mbar_arrive(B.p_full0 + 8 * b);
+            ptx::mbar_arrive(b_p);
         }
         // ---- epilogue: O / l
-        if (ok && ntiles > 0) {
-            const int last = ntiles - 1;
-            ok = wait_bar_warp(B.pv_done0 + 8 * (last & 1), (last >> 1) & 1, wctx);
-        }
-        if (ok && ntiles > 0) {
-            ptx::tc_fence_after();
-            __syncwarp();
-            const float inv = l > 0.f ? 1.0f / l : 0.f;
-            const int head = kvh * g + (row % g);
-            if (!SPLIT) {
-                __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) +
-                                     (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD;
+        if (ok && G.ntiles > 0) {
+            ok = wait_bar_warp(b_o, (G.ntiles - 1) & 1, wctx);
+            if (ok) {
+                ptx::tc_fence_after();
+                const float inv = l > 0.f ? 1.0f / l : 0.f;
+                const int head = kvh * g + (row % g);
+                if (!SPLIT) {
+                    __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) +
+                                         (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD;
 #pragma unroll
-                for (int ch = 0; ch < HD / 32; ++ch) {
-                    float o[32];
-                    ptx::tmem_ld32(tO + lane_off + ch * 32, o);
-                    ptx::tmem_wait_ld();
-                    if (valid) {
-                        uint4 *d4 = reinterpret_cast<uint4 *>(dst + ch * 32);
+                    for (int ch = 0; ch < HD / 32; ++ch) {
+                        float o[32];
+                        ptx::tmem_ld32(tO + ch * 32, o);
+                        ptx::tmem_wait_ld();
+                        if (valid) {
+                            uint4 *d4 = reinterpret_cast<uint4 *>(dst + ch * 32);
 #pragma unroll
-                        for (int j = 0; j < 4; ++j)
-                            d4[j] = make_uint4(pack_bf16(o[8 * j + 0] * inv, o[8 * j + 1] * inv),
-                                               pack_bf16(o[8 * j + 2] * inv, o[8 * j + 3] * inv),
-                                               pack_bf16(o[8 * j + 4] * inv, o[8 * j + 5] * inv),
-                                               pack_bf16(o[8 * j + 6] * inv, o[8 * j + 7] * inv));
+                            for (int k = 0; k < 4; ++k)
+                                d4[k] = make_uint4(pack_bf16(o[8 * k + 0] * inv, o[8 * k + 1] * inv),
+                                                   pack_bf16(o[8 * k + 2] * inv, o[8 * k + 3] * inv),
+                                                   pack_bf16(o[8 * k + 4] * inv, o[8 * k + 5] * inv),
+                                                   pack_bf16(o[8 * k + 6] * inv, o[8 * k + 7] * inv));
+                        }
                     }
-                }
-            } else {
-                const int64_t prow_idx =
-                    sq.part_row0 + (static_cast<int64_t>(qt * p.hkv + kvh) * sq.n_splits + split) * kBM + row;
-                float *dst = p.part_o + prow_idx * HD;
+                } else {
+                    const int64_t prow = sq.part_row0 +
+                                         (static_cast<int64_t>(G.qt * p.hkv + kvh) * sq.n_splits + split) * kBM + row;
+                    float *dst = p.part_o + prow * HD;
 #pragma unroll
-                for (int ch = 0; ch < HD / 32; ++ch) {
-                    float o[32];
-                    ptx::tmem_ld32(tO + lane_off + ch * 32, o);
-                    ptx::tmem_wait_ld();
-                    if (valid && l > 0.f) {
-                        float4 *d4 = reinterpret_cast<float4 *>(dst + ch * 32);
+                    for (int ch = 0; ch < HD / 32; ++ch) {
+                        float o[32];
+                        ptx::tmem_ld32(tO + ch * 32, o);
+                        ptx::tmem_wait_ld();
+                        if (valid && l > 0.f) {
+                            float4 *d4 = reinterpret_cast<float4 *>(dst + ch * 32);
 #pragma unroll
-                        for (int j = 0; j < 8; ++j)
-                            d4[j] = make_float4(o[4 * j] * inv, o[4 * j + 1] * inv, o[4 * j + 2] * inv,
-                                                o[4 * j + 3] * inv);
+                            for (int k = 0; k < 8; ++k)
+                                d4[k] = make_float4(o[4 * k] * inv, o[4 * k + 1] * inv, o[4 * k + 2] * inv,
+                                                    o[4 * k + 3] * inv);
+                        }
                     }
+                    if (valid) p.part_lse[prow] = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
                 }
-                if (valid) p.part_lse[prow_idx] = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
             }
         }
-    }
-    if (SPLIT && ntiles == 0 && warp < 4) {
-        // empty key range: this split contributes nothing to its rows
-        const int row = threadIdx.x;
-        const int qi = q_first + row / g;
-        if (qi <= q_last) {
-            const int64_t prow_idx =
-                sq.part_row0 + (static_cast<int64_t>(qt * p.hkv + kvh) * sq.n_splits + split) * kBM + row;
-            p.part_lse[prow_idx] = -INFINITY;
+        if (SPLIT && G.ntiles == 0 && valid) {
+            // empty key range: this split contributes nothing to these rows
+            const int64_t prow = sq.part_row0 +
+                                 (static_cast<int64_t>(G.qt * p.hkv + kvh) * sq.n_splits + split) * kBM + row;
+            p.part_lse[prow] = -INFINITY;
         }
     }
 
     ptx::tc_fence_before();
     __syncthreads();
-    if (warp == 5) {
+    if (warp == 9) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, C::kTmemCols);
     }
@@ -474,7 +574,7 @@ __global__ void __launch_bounds__(256) splitkv_combine_kernel(const __grid_const
     constexpr int kPer = HD / 32;
     float acc[kPer];
 #pragma unroll
-    for (int j = 0; j < kPer; ++j) acc[j] = 0.f;
+    for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
     float den = 0.f;
     if (mx != -INFINITY) {
         for (int s = 0; s < sq.n_splits; ++s) {
@@ -485,18 +585,18 @@ __global__ void __launch_bounds__(256) splitkv_combine_kernel(const __grid_const
             den += w;
             const float *src = p.part_o + r * HD + lane * kPer;
 #pragma unroll
-            for (int j = 0; j < kPer; ++j) acc[j] += w * src[j];
+            for (int k = 0; k < kPer; ++k) acc[k] += w * src[k];
         }
     }
     const float inv = den > 0.f ? 1.0f / den : 0.f;
     const int head = kvh * g + (row % g);
     __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) +
                          (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD + lane * kPer;
-    if (kPer == 4) {
-        uint2 v = make_uint2(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv));
-        *reinterpret_cast<uint2 *>(dst) = v;
+    if constexpr (kPer == 4) {
+        *reinterpret_cast<uint2 *>(dst) =
+            make_uint2(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv));
     } else {
-        *reinterpret_cast<uint32_t *>(dst) = pack_bf16(acc[0] * inv, acc[kPer - 1] * inv);
+        *reinterpret_cast<uint32_t *>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
     }
 }
 
@@ -512,7 +612,7 @@ static cudaError_t launch_attn_t(const CUtensorMap &q, const CUtensorMap &k, con
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    replay_attn_kernel<HD, SPLIT><<<p.total_items, 192, C::kDynSmem, st>>>(q, k, v, p);
+    replay_attn_kernel<HD, SPLIT><<<p.total_items, kThreads, C::kDynSmem, st>>>(q, k, v, p);
     return cudaGetLastError();
 }
 

@@ -363,7 +363,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         for (size_t i = lo; i < hi; ++i) {
             const AttnItem &it = order[i];
             const int64_t nqt = ceil_div(static_cast<int64_t>(it.n_q) * g, kBM);
-            base_ctas += nqt * hkv;
+            base_ctas += ceil_div(nqt, 2) * hkv;  // one CTA per pair of q-tiles
             const int64_t ktiles = ceil_div(c->len[it.seq], kBN);
             total_tiles += ktiles * nqt * hkv;
             max_tiles = std::max(max_tiles, ktiles);
@@ -411,7 +411,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
                 q.item0 = item;
                 q.part_row0 = prow;
                 q.comb0 = comb;
-                item += q.n_qtiles * hkv * q.n_splits;
+                item += ((q.n_qtiles + 1) / 2) * hkv * q.n_splits;
                 if (split) {
                     prow += static_cast<int64_t>(q.n_qtiles) * hkv * q.n_splits * kBM;
                     comb += q.n_qtiles * hkv * kBM;

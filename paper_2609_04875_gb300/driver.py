@@ -26,7 +26,9 @@ def _dev(bits: np.ndarray, device) -> torch.Tensor:
 class ReplayDriver:
     """Device-resident crop + replay of a synthetic workload (``synth.Workload``)."""
 
-    def __init__(self, w, device="cuda", fill=True, cache_kwargs=None):
+    def __init__(self, w, device="cuda", fill=True, cache_kwargs=None, inputs=None):
+        """inputs: optional {agent index: (k0, v0, kc, vc, qc)} host bf16 bits, as
+        drawn by the workload; drawn here when absent."""
         self.w = w
         self.device = torch.device(device)
         L, hq, hkv, d = w.num_layers, w.num_q_heads, w.num_kv_heads, w.head_dim
@@ -42,21 +44,27 @@ class ReplayDriver:
         self.Kc = torch.empty((L, n, hkv, d), dtype=torch.bfloat16, device=self.device)
         self.Vc = torch.empty_like(self.Kc)
         self.Qc = torch.empty((L, n, hq, d), dtype=torch.bfloat16, device=self.device)
+        self._inputs = inputs
         for i, a in enumerate(w.agents):
-            k, v = w.kv_counterfactual(a)
+            if inputs is not None:
+                _, _, k, v, q = inputs[i]
+            else:
+                (k, v), q = w.kv_counterfactual(a), w.q_counterfactual(a)
             lo, hi = self.cu[i], self.cu[i + 1]
             self.Kc[:, lo:hi] = _dev(k, self.device)
             self.Vc[:, lo:hi] = _dev(v, self.device)
-            self.Qc[:, lo:hi] = _dev(w.q_counterfactual(a), self.device)
+            self.Qc[:, lo:hi] = _dev(q, self.device)
+            del k, v, q
         self.out = torch.empty_like(self.Qc)
         if fill:
             self.fill_original()
 
     def fill_original(self):
         """Writes every agent's original session (T positions) in agent order."""
-        for s, a in zip(self.seqs, self.w.agents):
-            k, v = self.w.kv_original(a)
+        for i, (s, a) in enumerate(zip(self.seqs, self.w.agents)):
+            k, v = self._inputs[i][:2] if self._inputs is not None else self.w.kv_original(a)
             self.cache.append_kv(s, _dev(k, self.device), _dev(v, self.device))
+            del k, v
         torch.cuda.synchronize(self.device)
 
     # -- the hot path ------------------------------------------------------------

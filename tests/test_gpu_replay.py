@@ -9,7 +9,7 @@ import torch
 
 import oracle
 import synth
-from gpu_common import MAX_ABS, Pair, assert_close, dev, replay_case, requires_cuda
+from gpu_common import MAX_ABS, Pair, assert_close, assert_within_rounding_bound, dev, replay_case, requires_cuda
 
 pytestmark = [pytest.mark.gpu, requires_cuda]
 
@@ -41,10 +41,12 @@ def test_replay_matches_oracle(case):
 @pytest.mark.parametrize("scale_mult", [4.0, 8.0])
 def test_peaked_logits_exercise_rescaling(scale_mult):
     """Logit std 4-8: running maxima jump between key tiles, so the lazy rescale
-    of O in TMEM runs."""
+    of O in TMEM runs.  The output is then close to single value rows (|O| up
+    to max|V|), so the check uses the derived rounding bound."""
     d = 128
-    pair, s, outs, refs, _ = replay_case(1, 32, 8, d, 16, 700, 300, seed=5, scale=scale_mult / math.sqrt(d))
-    assert_close(outs[0], refs[0], f"peaked x{scale_mult}")
+    pair, s, outs, refs, inputs = replay_case(1, 32, 8, d, 16, 700, 300, seed=5, scale=scale_mult / math.sqrt(d))
+    vmax = float(np.abs(synth.bf16_bits_to_f32(np.concatenate([inputs[1], inputs[3]], 1))).max())
+    assert_within_rounding_bound(outs[0], refs[0], vmax, f"peaked x{scale_mult}")
 
 
 def test_multilayer_and_pool_contents():
@@ -53,7 +55,6 @@ def test_multilayer_and_pool_contents():
     for layer in range(L):
         assert_close(outs[layer], refs[layer], f"layer {layer}")
     # pool contents: every valid slot holds the oracle's bits
-    kp, vp = torch.empty(0), torch.empty(0)
     import ctypes
     from paper_2609_04875_gb300 import binding
     kptr, vptr = ctypes.c_void_p(), ctypes.c_void_p()
@@ -74,7 +75,7 @@ def test_multilayer_and_pool_contents():
 def _view_device(ptr, n):
     """A bf16 CUDA tensor over n elements at a raw device pointer (read-only use)."""
     class _Arr:
-        __cuda_array_interface__ = {"shape": (n,), "typestr": "<i2", "data": (ptr, True), "version": 3}
+        __cuda_array_interface__ = {"shape": (n,), "typestr": "<i2", "data": (ptr, False), "version": 3}
     return torch.as_tensor(_Arr(), device="cuda").view(torch.bfloat16)
 
 
@@ -244,7 +245,7 @@ def test_gpu_error_paths_leave_state_unchanged():
     k = torch.zeros((2, 40, 2, 128), dtype=torch.bfloat16, device="cuda")
     c.append_kv(s, k, k)
     s2 = c.seq_create()
-    c.append_kv(s2, k[:, :32], k[:, :32])   # 3 + 2 pages used, 1 free
+    c.append_kv(s2, k[:, :32].contiguous(), k[:, :32].contiguous())   # 3 + 2 pages used, 1 free
     before = (c.page_table(s), c.free_list(), c.seq_info(s))
     q = torch.zeros((41, 8, 128), dtype=torch.bfloat16, device="cuda")
     for fn, kind in [(lambda: c.replay_attn(s, 0, q), "range"),
