@@ -132,6 +132,28 @@ pe_status pe_replay_attn_batch(pe_cache *cache, int32_t n, const int32_t *seqs, 
                                const void *Q_packed, const int32_t *cu_q, void *out, int32_t num_q_heads,
                                float softmax_scale, void *stream);
 
+/* Variant of pe_replay_attn for callers that cannot allocate device memory at
+ * the time they run attention: code inside a stream host callback or a
+ * latency-critical serving loop where cudaMalloc (which may synchronise the
+ * device) is not allowed, or a process whose device memory is entirely
+ * reserved by its own allocator.  The paper has no counterpart; it is a
+ * property of this library, not of the method.
+ * It always takes the split-KV path and keeps the split partials in one fixed
+ * 16 MiB array compiled into the library (every GPU that loads the library
+ * holds it until the process exits) instead of the cache's workspace; it
+ * calls no cudaMalloc/cudaFree and no allocating routine.  Arguments, result
+ * and errors are those of pe_replay_attn; in addition RANGE when one key
+ * split of n_q x num_q_heads rows does not fit the array
+ * (ceil(n_q*(Hq/Hkv)/128) * Hkv * 128 * (4*d + 4) bytes must be <= 16 MiB).
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture.  Every call shares the array and overwrites what the previous call
+ * left there (no part of it needs to start at zero): calls that overlap on
+ * the GPU (different streams, concurrent threads) race and must be ordered by
+ * the caller. */
+pe_status pe_replay_attn_static_scratch(pe_cache *cache, int32_t seq, int32_t layer, const void *Q, void *out,
+                                        int32_t n_q, int32_t num_q_heads, float softmax_scale, void *stream);
+
 /* Host-side state queries (no device work). */
 pe_status pe_seq_info(const pe_cache *cache, int32_t seq, int64_t *len, int64_t *appended_since_crop);
 pe_status pe_seq_page_table(const pe_cache *cache, int32_t seq, int32_t *out, int32_t cap, int32_t *n);

@@ -27,7 +27,7 @@ EXPORTED = [
     "pe_cache_create", "pe_cache_destroy", "pe_seq_create", "pe_seq_release", "pe_crop", "pe_crop_batch",
     "pe_append_kv", "pe_append_kv_batch", "pe_replay_attn", "pe_replay_attn_batch", "pe_seq_info",
     "pe_seq_page_table", "pe_free_list", "pe_seq_device_page_table", "pe_cache_pools", "pe_set_option",
-    "pe_device_status", "pe_kernel_launches", "pe_last_error", "pe_version",
+    "pe_device_status", "pe_kernel_launches", "pe_replay_attn_static_scratch", "pe_last_error", "pe_version",
 ]
 
 
@@ -73,6 +73,7 @@ _sigs = {
     "pe_set_option": [_P, ctypes.c_char_p, _I64],
     "pe_device_status": [_P, _I32P, _I32, _P],
     "pe_kernel_launches": [_P, _I64P],
+    "pe_replay_attn_static_scratch": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
 }
 for _name, _args in _sigs.items():
     _fn = getattr(_lib, _name)
@@ -260,6 +261,19 @@ class PagedKVCache:
         _check(_lib.pe_replay_attn_batch(self._h, len(seqs), _i32_array(seqs), layer, _dev_ptr(Q, "Q"),
                                          _i32_array(cu_q), _dev_ptr(out, "out"), Q.shape[1], scale,
                                          self._s(stream)))
+        return out
+
+    def replay_attn_static_scratch(self, seq, layer, Q, out=None, softmax_scale=None, stream=None):
+        """pe_replay_attn_static_scratch: split-KV replay attention whose partials
+        live in the library's fixed device array (the call allocates nothing)."""
+        import torch
+        if Q.dim() != 3 or Q.shape[2] != self.head_dim:
+            raise ValueError("Q must be [n_q][Hq][d]")
+        if out is None:
+            out = torch.empty_like(Q)
+        scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
+        _check(_lib.pe_replay_attn_static_scratch(self._h, seq, layer, _dev_ptr(Q, "Q"), _dev_ptr(out, "out"),
+                                                  Q.shape[0], Q.shape[1], scale, self._s(stream)))
         return out
 
     # -- state -----------------------------------------------------------------

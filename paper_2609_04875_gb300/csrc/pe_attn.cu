@@ -35,6 +35,8 @@
 // all roles leave their loops, and TMEM is freed before exit.
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "pe_internal.h"
 #include "ptx.cuh"
 
@@ -598,6 +600,32 @@ __global__ void __launch_bounds__(256) splitkv_combine_kernel(const __grid_const
     } else {
         *reinterpret_cast<uint32_t *>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
     }
+}
+
+// Split-KV partials of pe_replay_attn_static_scratch: a fixed 16 MiB array that
+// every GPU loading the library holds until the process exits.  Host code must
+// not pass the symbol itself to a kernel (on the host it names a stand-in, not
+// device memory); static_scratch() looks up its device address instead.
+static __device__ __align__(256) float g_static_splitkv_scratch[kStaticScratchBytes / sizeof(float)];
+
+cudaError_t static_scratch(float **ptr)
+{
+    constexpr int kMaxDevices = 64;
+    static std::mutex mu;
+    static float *addr[kMaxDevices] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {  // once per device, with that device current
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_splitkv_scratch);
+        if (e != cudaSuccess) return e;
+        addr[dev] = static_cast<float *>(p);
+    }
+    *ptr = addr[dev];
+    return cudaSuccess;
 }
 
 template <int HD, bool SPLIT>

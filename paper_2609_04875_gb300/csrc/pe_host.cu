@@ -723,6 +723,82 @@ pe_status pe_replay_attn_batch(pe_cache *c, int32_t n, const int32_t *seqs, int3
                          static_cast<cudaStream_t>(stream));
 }
 
+pe_status pe_replay_attn_static_scratch(pe_cache *c, int32_t seq, int32_t layer, const void *Q, void *out,
+                                        int32_t n_q, int32_t num_q_heads, float softmax_scale, void *stream)
+{
+    // Same computation as pe_replay_attn through the split-KV kernel and its
+    // combine, but the partials go to the library's fixed device array, and
+    // nothing here allocates (parameters live on the stack).
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if ((s = check_attn_args(c, layer, Q, out, num_q_heads, softmax_scale)) != PE_OK) return s;
+    if (n_q < 0) return fail(PE_ERR_INVALID, "negative n_q");
+    if (n_q > c->len[seq])
+        return fail(PE_ERR_RANGE, "n_q = %d exceeds the sequence length %lld", n_q, static_cast<long long>(c->len[seq]));
+    if (n_q == 0) return PE_OK;
+    const pe_cache_config &cf = c->cfg;
+    const int hkv = cf.num_kv_heads, d = cf.head_dim, g = num_q_heads / hkv;
+    const int64_t n_qtiles = ceil_div(static_cast<int64_t>(n_q) * g, kBM);
+    const int64_t ktiles = ceil_div(c->len[seq], kBN);
+    const int64_t row_bytes = static_cast<int64_t>(d) * 4 + 4;   // fp32 partial row + its LSE
+    const int64_t split_bytes = n_qtiles * hkv * kBM * row_bytes;  // one split of every q-tile
+    const int64_t max_splits = kStaticScratchBytes / split_bytes;
+    if (max_splits < 1)
+        return fail(PE_ERR_RANGE,
+                    "static scratch too small: one key split of %d queries x %d heads needs %lld bytes, the fixed "
+                    "array holds %lld",
+                    n_q, num_q_heads, static_cast<long long>(split_bytes),
+                    static_cast<long long>(kStaticScratchBytes));
+    float *scratch = nullptr;
+    cudaError_t e = static_scratch(&scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the static scratch");
+    // split count: about four CTAs per SM, at least 4 key tiles per split, within the array
+    const int64_t pairs = ceil_div(n_qtiles, 2) * hkv;
+    int64_t n_splits = std::max<int64_t>(1, std::min<int64_t>(ceil_div(4LL * c->num_sms, pairs), ceil_div(ktiles, 4)));
+    n_splits = std::min(n_splits, max_splits);
+    const int split_tiles = static_cast<int>(ceil_div(ktiles, n_splits));
+    n_splits = ceil_div(ktiles, split_tiles);
+
+    CUtensorMap tm_q;
+    if ((s = encode_q(&tm_q, Q, n_q, num_q_heads, d, g)) != PE_OK) return s;
+    AttnParams p;
+    std::memset(&p, 0, sizeof p);
+    p.page_table = c->d_table;
+    p.out = out;
+    p.status = c->d_status;
+    p.n_seqs = 1;
+    p.hq = num_q_heads;
+    p.hkv = hkv;
+    p.group = g;
+    p.layer = layer;
+    p.num_pages = cf.num_pages;
+    p.ps = cf.page_size;
+    p.oob_row = static_cast<int32_t>(c->pool_rows);
+    p.split_tiles = split_tiles;
+    p.scale_log2 = softmax_scale * 1.4426950408889634f;
+    AttnSeq &q = p.seqs[0];
+    q.table_row = seq * cf.max_pages_per_seq;
+    q.n_pages = static_cast<int32_t>(c->table[seq].size());
+    q.q_row0 = 0;
+    q.n_q = n_q;
+    q.n_keys = static_cast<int32_t>(c->len[seq]);
+    q.n_qtiles = static_cast<int32_t>(n_qtiles);
+    q.n_splits = static_cast<int32_t>(n_splits);
+    const int64_t prow = n_qtiles * hkv * n_splits * kBM;
+    p.total_items = static_cast<int32_t>(ceil_div(n_qtiles, 2) * hkv * n_splits);
+    p.total_comb = static_cast<int32_t>(n_qtiles * hkv * kBM);
+    p.part_o = scratch;
+    p.part_lse = scratch + prow * d;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, p, st);
+    if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
+    c->launches++;
+    e = launch_splitkv_combine(d, p, st);
+    if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
+    c->launches++;
+    return PE_OK;
+}
+
 pe_status pe_seq_info(const pe_cache *c, int32_t seq, int64_t *len, int64_t *appended_since_crop)
 {
     pe_status s = check_seq(c, seq);

@@ -97,4 +97,10 @@ cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q
                                const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);
 
+// Fixed split-KV scratch compiled into the library (pe_attn.cu), used only by
+// pe_replay_attn_static_scratch.  static_scratch() returns its device address
+// on the current device; the address is looked up once per device.
+constexpr int64_t kStaticScratchBytes = 16ll << 20;
+cudaError_t static_scratch(float **ptr);
+
 }  // namespace pe
