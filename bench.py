@@ -52,6 +52,7 @@ def load_peaks():
 
 
 def make_workload(name):
+    """agent_batch | tiny | short_suffix | long_suffix | tau_sweep_r<ratio> (ratio 0 = full reset)."""
     if name.startswith("tau_sweep_r"):
         return synth.tau_sweep(float(name[len("tau_sweep_r"):]))
     return synth.WORKLOADS[name]()
@@ -150,6 +151,72 @@ def oracle_tokens_per_s(w, budget_s, seed=7):
 
 
 # ------------------------------------------------------------------ GPU arm
+# DRAM traffic per attention launch from one ncu capture (profiles/), valid only
+# while the kernel source is the one that was captured.
+NCU_TRAFFIC = {
+    "agent_batch": {"bytes": 695.840256e6 + 328.223232e6, "profile": "profiles/replay_attn_agent_batch.md",
+                    "src_sha256": "9ffa64956896d561458cf73e334afd33e763c555ae0a4a560f7f043460335b88"},
+}
+ATTN_SRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc", "pe_attn.cu")
+
+
+def _src_sha():
+    """sha256 of the attention kernel's source (from its config struct to the
+    end of the kernel), so that recorded counters lapse when the kernel changes."""
+    import hashlib
+    with open(ATTN_SRC) as f:
+        txt = f.read()
+    try:
+        a = txt.index("template <int HD>\nstruct AttnCfg")
+        b = txt.index("// One warp per output row")
+    except ValueError:
+        return None
+    return hashlib.sha256(txt[a:b].encode()).hexdigest()
+
+
+def traffic_for(workload):
+    t = NCU_TRAFFIC.get(workload)
+    if not t or t["src_sha256"] != _src_sha():
+        return None, None
+    return t["bytes"], t["profile"]
+
+
+def roofline_for(w, flops_launch, bytes_launch, attn_s, peaks, peak_src):
+    """Per-launch roofline of the replay-attention kernel: the slower of its
+    algorithmic FLOPs at the bf16 tensor peak and its algorithmic bytes at HBM
+    bandwidth decides the bound."""
+    tflops = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    gbs = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    t_flop = flops_launch / (tflops * 1e12)
+    t_hbm = bytes_launch / (gbs * 1e9)
+    traffic, prof = traffic_for(w.name)
+    if t_flop >= t_hbm:
+        achieved = flops_launch / attn_s / 1e12
+        r = {"bound": "tensor", "achieved": achieved, "peak": tflops, "unit": "TFLOP/s",
+             "peak_source": f"bf16_tflops (burst) of {peak_src}"}
+    else:
+        achieved = bytes_launch / attn_s / 1e9
+        r = {"bound": "hbm", "achieved": achieved, "peak": gbs, "unit": "GB/s",
+             "peak_source": f"hbm_gbs of {peak_src}"}
+    r["frac"] = r["achieved"] / r["peak"]
+    r["traffic"] = traffic
+    r["traffic_profile"] = prof
+    r["kernel"] = f"replay_attn_kernel<{w.head_dim},{'split' if w.name == 'short_suffix' else 'nosplit'}>"
+    r["attn_ms_per_launch"] = attn_s * 1e3
+    r["algorithmic_flop_per_launch"] = flops_launch
+    r["algorithmic_bytes_per_launch"] = bytes_launch
+    r["roofline_ms_per_launch"] = max(t_flop, t_hbm) * 1e3
+    return r
+
+
+def attn_bytes(w):
+    """Algorithmic bytes of one attention launch (one layer): every cached K/V
+    row of each kv-head read once, Q read, O written (bf16)."""
+    keys = sum(a.T for a in w.agents)
+    q = sum(a.S for a in w.agents)
+    return 2.0 * (2 * keys * w.num_kv_heads * w.head_dim + 2 * q * w.num_q_heads * w.head_dim)
+
+
 def run_pe(args, rank, world, local_rank):
     import torch
 
@@ -203,34 +270,36 @@ def run_pe(args, rank, world, local_rank):
     ms_per_step = elapsed_ms / args.steps
     value = world * tokens_per_step * args.steps / (elapsed_ms / 1e3)
 
-    # ---- crop latency: host call time and device time of the crop kernel
-    crop_host_us, crop_dev_us = [], []
+    # ---- crop latency: host call time and device time of the crop kernel;
+    #      append time of the same steps
+    crop_host_us, crop_dev_us, append_ms = [], [], []
     for _ in range(20):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
         torch.cuda.synchronize(dev)
         e0.record(stream)
         h0 = time.perf_counter()
         drv.crop()
         h1 = time.perf_counter()
         e1.record(stream)
+        drv.append()
+        e2.record(stream)
+        for layer in range(L):
+            drv.attend(layer)
         torch.cuda.synchronize(dev)
         crop_host_us.append((h1 - h0) * 1e6)
         crop_dev_us.append(e0.elapsed_time(e1) * 1e3)
-        drv.append()
-        for layer in range(L):
-            drv.attend(layer)
+        append_ms.append(e1.elapsed_time(e2))
     torch.cuda.synchronize(dev)
 
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(drv, dev, stream, min(args.steps, args.e2e_steps), world, dist)
+        e2e = run_e2e(drv, dev, min(args.steps, args.e2e_steps), world, dist)
 
     peaks, peak_src = load_peaks()
     flops = workload_flops(w) / L  # per attention launch (one per layer)
     attn_avg_s = statistics.mean(attn_ms) / 1e3
-    achieved = flops / attn_avg_s / 1e12
-    peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    roof = roofline_for(w, flops, attn_bytes(w), attn_avg_s, peaks, peak_src)
     result = {
         "metric": METRIC,
         "value": value,
@@ -243,28 +312,22 @@ def run_pe(args, rank, world, local_rank):
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1)/sqrt(128) bf16 Q/K/V; no dataset)",
+        "data": f"synthetic (seeded N(0,{w.std:.4g}^2) bf16 Q/K/V; no dataset)",
         "config": {
             **w.describe(),
             "parallelism": f"replicas x{world} (independent agents, no collective)",
-            "l2": "inputs larger than L2 (KV cache %.0f MB per GPU)" % (
+            "l2": "inputs larger than L2 (KV cache %.0f MB per GPU, L2 129 MB)" % (
                 sum(a.T for a in w.agents) * w.num_kv_heads * w.head_dim * 4 * w.num_layers / 1e6),
         },
-        "roofline": {
-            "bound": "tensor",
-            "kernel": "replay_attn_kernel<128,false>",
-            "achieved": achieved,
-            "peak": peak,
-            "peak_source": f"bf16_tflops (burst) of {peak_src}",
-            "unit": "TFLOP/s",
-            "frac": achieved / peak,
-            "traffic": None,
-            "attn_ms_per_launch": attn_avg_s * 1e3,
-            "algorithmic_flop_per_launch": flops,
-        },
+        "roofline": roof,
         "attn_tflops_step": workload_flops(w) / (ms_per_step / 1e3) / 1e12,
+        "step_breakdown_ms": {"attention_all_layers": attn_avg_s * 1e3 * L,
+                              "append": statistics.median(append_ms),
+                              "crop": statistics.median(crop_dev_us) / 1e3},
         "crop_us": {"host_call_median": statistics.median(crop_host_us),
                     "device_median": statistics.median(crop_dev_us), "agents": len(w.agents)},
+        "recomputed_tokens": tokens_per_step,
+        "session_tokens": sum(a.T for a in w.agents),
         "gpu_launches": launches,
         "clocks": clk,
         "e2e": e2e,
@@ -278,32 +341,55 @@ def run_pe(args, rank, world, local_rank):
         print(json.dumps(result), flush=True)
 
 
-def run_e2e(drv, dev, stream, steps, world, dist):
-    """Same step through the public API with the step's inputs (K', V', Q') in
-    pinned host memory: H2D copies, crop + append + replay, D2H of the output."""
+def run_e2e(drv, dev, steps, world, dist):
+    """The same step through the public API with the step's inputs (K', V', Q')
+    in pinned host memory: every step copies its inputs host->device, runs
+    crop + append + replay and copies its output device->host.  Copies run on
+    their own streams and overlap the previous/next step's compute (two device
+    buffer sets); the timed region spans the first input copy to the last
+    output copy."""
     import torch
-    hK = drv.Kc.cpu().pin_memory()
-    hV = drv.Vc.cpu().pin_memory()
-    hQ = drv.Qc.cpu().pin_memory()
-    hO = torch.empty(drv.out.shape, dtype=drv.out.dtype).pin_memory()
-    h2d = (hK.numel() + hV.numel() + hQ.numel()) * 2
-    d2h = hO.numel() * 2
+    K, V, Q, O = drv.buffers()
+    hK, hV, hQ = K.cpu().pin_memory(), V.cpu().pin_memory(), Q.cpu().pin_memory()
+    hO = [torch.empty(O.shape, dtype=O.dtype).pin_memory() for _ in range(2)]
+    sets = [(K, V, Q, O), tuple(torch.empty_like(x) for x in (K, V, Q, O))]
+    h2d_bytes = (hK.numel() + hV.numel() + hQ.numel()) * 2
+    d2h_bytes = O.numel() * 2
+    comp = torch.cuda.current_stream(dev)
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    free = [torch.cuda.Event() for _ in range(2)]
+    ready = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+    for e in free:
+        e.record(comp)
 
-    def one():
-        drv.Kc.copy_(hK, non_blocking=True)
-        drv.Vc.copy_(hV, non_blocking=True)
-        drv.Qc.copy_(hQ, non_blocking=True)
-        drv.step()
-        hO.copy_(drv.out, non_blocking=True)
+    def one(k):
+        b = k % 2
+        bk, bv, bq, bo = sets[b]
+        s_in.wait_event(free[b])
+        with torch.cuda.stream(s_in):
+            bk.copy_(hK, non_blocking=True)
+            bv.copy_(hV, non_blocking=True)
+            bq.copy_(hQ, non_blocking=True)
+            ready[b].record(s_in)
+        comp.wait_event(ready[b])
+        drv.step(bufs=sets[b])
+        done[b].record(comp)
+        s_out.wait_event(done[b])
+        with torch.cuda.stream(s_out):
+            hO[b].copy_(bo, non_blocking=True)
+            free[b].record(s_out)
 
-    for _ in range(3):
-        one()
+    for k in range(3):
+        one(k)
     torch.cuda.synchronize(dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(steps):
-        one()
-    e1.record(stream)
+    e0.record(comp)
+    s_in.wait_stream(comp)
+    for k in range(steps):
+        one(k)
+    comp.wait_stream(s_out)
+    e1.record(comp)
     torch.cuda.synchronize(dev)
     ms = e0.elapsed_time(e1)
     if dist:
@@ -312,8 +398,9 @@ def run_e2e(drv, dev, stream, steps, world, dist):
         tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
         ms = float(t.item())
     tokens = world * drv.w.total_suffix * steps
-    return {"value": tokens / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "steps": steps, "ms_per_step": ms / steps}
+    return {"value": tokens / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
+            "d2h_bytes_per_step": d2h_bytes, "steps": steps, "ms_per_step": ms / steps,
+            "overlap": "double-buffered: copies of step k+1 / k-1 overlap the compute of step k"}
 
 
 # ------------------------------------------------------------------ reference arm

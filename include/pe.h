@@ -70,7 +70,7 @@ typedef struct {
     void *k_pool;               /* device, nullable: caller-owned K pool, bf16 [L][num_pages][Hkv][ps][d] */
     void *v_pool;               /* device, nullable: caller-owned V pool, same layout.  NULL = the
                                    library allocates (cudaMalloc) and zero-fills both pools */
-    int64_t workspace_bytes;    /* split-KV scratch allocated at create; 0 = 64 MiB */
+    int64_t workspace_bytes;    /* split-KV scratch allocated at create; 0 = 256 MiB */
 } pe_cache_config;
 
 /* Creates a cache.  Sizes are checked (d, ps, positive counts, int32-addressable

@@ -359,28 +359,46 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
 
     // split-KV decision over the whole launch group
     auto plan_group = [&](size_t lo, size_t hi, AttnParams &p, bool &split) -> pe_status {
-        int64_t base_ctas = 0, total_tiles = 0, max_tiles = 0;
+        // C CTAs (pairs of q-tiles x kv-heads), W key tiles per CTA on average.
+        int64_t C = 0, tiles = 0, rows = 0, max_tiles = 0;
         for (size_t i = lo; i < hi; ++i) {
             const AttnItem &it = order[i];
+            const int64_t len = c->len[it.seq];
             const int64_t nqt = ceil_div(static_cast<int64_t>(it.n_q) * g, kBM);
-            base_ctas += ceil_div(nqt, 2) * hkv;  // one CTA per pair of q-tiles
-            const int64_t ktiles = ceil_div(c->len[it.seq], kBN);
-            total_tiles += ktiles * nqt * hkv;
-            max_tiles = std::max(max_tiles, ktiles);
-        }
-        int split_tiles = static_cast<int>(max_tiles);
-        if (c->splitkv == 1 || (c->splitkv == -1 && base_ctas < c->num_sms && max_tiles >= 16)) {
-            if (c->num_splits > 0) {
-                split_tiles = static_cast<int>(ceil_div(max_tiles, c->num_splits));
-            } else {
-                const int64_t target = 4LL * c->num_sms;
-                split_tiles = static_cast<int>(std::max<int64_t>(4, ceil_div(total_tiles, target)));
+            for (int64_t pp = 0; pp < ceil_div(nqt, 2); ++pp) {
+                const int64_t q_last = std::min<int64_t>((std::min(2 * pp + 1, nqt - 1) + 1) * bmq, it.n_q) - 1;
+                tiles += ceil_div(len - it.n_q + q_last + 1, kBN) * hkv;
             }
-            split_tiles = std::max(1, split_tiles);
-            split = true;
-        } else {
-            split = false;
+            C += ceil_div(nqt, 2) * hkv;
+            rows += nqt * hkv * kBM;
+            max_tiles = std::max(max_tiles, ceil_div(len, kBN));
         }
+        // Estimated time with s key splits: the CTAs run in ceil(C s / N) waves of
+        // (W/s + 2) tile times (about 1.5 us per tile, compute- or HBM-bound
+        // alike); splits add their fp32 partials' HBM round trip and a combine launch.
+        const double W = C > 0 ? static_cast<double>(tiles) / C : 0.0;
+        const int64_t row_bytes = static_cast<int64_t>(d) * 4 + 4;
+        auto cost = [&](int64_t sp) {
+            const double waves = std::ceil(static_cast<double>(C * sp) / c->num_sms);
+            double t = waves * (W / sp + 2.0) * 1.5e-6;
+            if (sp > 1) t += static_cast<double>(rows * sp * row_bytes * 2) / 6.0e12 + 5e-6;
+            return t;
+        };
+        int64_t best = 1;
+        if (c->splitkv != 0) {
+            const int64_t s_max = std::min<int64_t>(128, std::max<int64_t>(1, max_tiles / 4));
+            double best_t = c->splitkv == 1 ? 1e30 : cost(1);
+            for (int64_t sp = 2; sp <= s_max; ++sp) {
+                if (rows * sp * row_bytes > c->ws_bytes) break;
+                const double t = cost(sp);
+                if (t < best_t) { best_t = t; best = sp; }
+            }
+            if (c->splitkv == -1 && best > 1 && best_t > 0.95 * cost(1)) best = 1;  // keep the single pass unless clearly faster
+        }
+        if (c->splitkv != 0 && c->num_splits > 0) best = c->num_splits;
+        int split_tiles = static_cast<int>(max_tiles);
+        split = best > 1 || c->splitkv == 1;
+        if (split) split_tiles = static_cast<int>(std::max<int64_t>(1, ceil_div(max_tiles, std::max<int64_t>(best, 1))));
         std::memset(&p, 0, sizeof p);
         p.page_table = c->d_table;
         p.out = out;
@@ -541,7 +559,7 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
     }
     const size_t pool_bytes = static_cast<size_t>(pool_rows) * c.head_dim * 2;
     const size_t table_bytes = static_cast<size_t>(c.max_seqs) * c.max_pages_per_seq * sizeof(int32_t);
-    cc->ws_bytes = c.workspace_bytes > 0 ? c.workspace_bytes : (64ll << 20);
+    cc->ws_bytes = c.workspace_bytes > 0 ? c.workspace_bytes : (256ll << 20);
     pe_status st = PE_OK;
     do {
         if (c.k_pool) {

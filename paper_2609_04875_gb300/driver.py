@@ -68,28 +68,35 @@ class ReplayDriver:
         torch.cuda.synchronize(self.device)
 
     # -- the hot path ------------------------------------------------------------
+    def buffers(self):
+        """The step's device buffers (K', V', Q', out)."""
+        return self.Kc, self.Vc, self.Qc, self.out
+
     def crop(self, stream=None):
         self.cache.crop_batch(self.seqs, self.taus, stream=stream)
 
-    def append(self, stream=None):
-        self.cache.append_kv_batch(self.seqs, self.Kc, self.Vc, self.cu, stream=stream)
+    def append(self, stream=None, bufs=None):
+        K, V = (bufs or self.buffers())[:2]
+        self.cache.append_kv_batch(self.seqs, K, V, self.cu, stream=stream)
 
-    def attend(self, layer, stream=None):
-        self.cache.replay_attn_batch(self.seqs, layer, self.Qc[layer], self.cu, out=self.out[layer],
+    def attend(self, layer, stream=None, bufs=None):
+        Q, out = (bufs or self.buffers())[2:]
+        self.cache.replay_attn_batch(self.seqs, layer, Q[layer], self.cu, out=out[layer],
                                      softmax_scale=self.w.softmax_scale, stream=stream)
 
-    def step(self, stream=None, attn_events=None):
+    def step(self, stream=None, attn_events=None, bufs=None):
         """One forget request for every agent.  attn_events: optional list of
-        (start, end) CUDA event pairs, one per layer, recorded around attention."""
+        (start, end) CUDA event pairs, one per layer, recorded around attention.
+        bufs: optional (K', V', Q', out) device tensors shaped like buffers()."""
         self.crop(stream)
-        self.append(stream)
+        self.append(stream, bufs)
         for layer in range(self.w.num_layers):
             if attn_events is not None:
                 attn_events[layer][0].record(stream)
-            self.attend(layer, stream)
+            self.attend(layer, stream, bufs)
             if attn_events is not None:
                 attn_events[layer][1].record(stream)
-        return self.out
+        return (bufs or self.buffers())[3]
 
     # -- bookkeeping -------------------------------------------------------------
     def algorithmic_flops(self) -> float:
