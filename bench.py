@@ -154,8 +154,8 @@ def oracle_tokens_per_s(w, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "agent_batch": {"bytes": 695.840256e6 + 328.223232e6, "profile": "profiles/replay_attn_agent_batch.md",
-                    "src_sha256": "9ffa64956896d561458cf73e334afd33e763c555ae0a4a560f7f043460335b88"},
+    "agent_batch": {"bytes": 696.202240e6 + 328.267008e6, "profile": "profiles/replay_attn_agent_batch.md",
+                    "src_sha256": "8f464a14b8867cf08b98323c8adbd93a191e4ab164630cb50790aa344dfe764f"},
 }
 ATTN_SRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc", "pe_attn.cu")
 

@@ -26,10 +26,13 @@
 // Key tiles always start at logical key 0 (multiples of 128 keys), whatever
 // the physical pages, so a row's arithmetic depends only on its own keys.
 //
-// Online softmax with a lazily moved reference: a row's reference max m_ref
-// only moves when a new tile's max exceeds it by more than 2^8 (then O and l
-// are rescaled in place); otherwise exp2(x - m_ref) <= 256, exact in the final
-// O / l.  Rows decide independently.
+// Online softmax with a lazily moved reference: a row's reference m_ref is the
+// first tile's max (log2 units) and only moves when a later tile's weights
+// exp2(x - m_ref) sum beyond 2^64 (a logit more than ~64 above m_ref, or
+// inf/NaN); then the tile max is taken, O and l are rescaled in place and the
+// tile's weights recomputed.  Any fixed reference gives the same O / l, and
+// weights up to 2^64 stay far inside fp32/bf16 range, so the tile max is
+// skipped on all other tiles.  Rows decide independently.
 //
 // Every wait is bounded (kWaitNs); on expiry the CTA records a status code,
 // all roles leave their loops, and TMEM is freed before exit.
@@ -43,7 +46,7 @@
 namespace pe {
 
 constexpr uint64_t kWaitNs = 1000000000ull;  // 1 s
-constexpr float kRescaleThreshold = 8.0f;    // log2 units
+constexpr float kTileSumLimit = 1.8446744e19f;  // 2^64: larger tile sums move the reference
 constexpr int kThreads = 320;
 
 template <int HD>
@@ -430,21 +433,49 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int c = 0; c < kBN; ++c)
                     if (kbase + c > pos) s[c] = -INFINITY;
             }
-            // row max: 8 independent chains of 3-input max, then a tree
-            float mx[8];
+            // Exponentials against the row's current reference m_ref; the exact tile
+            // max is needed only on the first tile, or when the tile's sum exceeds
+            // 2^64 (some logit above m_ref + ~64, or inf/NaN): then m_ref moves, O
+            // and l are rescaled, and the tile is recomputed.
+            auto exp_tile = [&](float ref) -> float {
+                const float2 nref = make_float2(-ref, -ref);
+                float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                                 make_float2(0.f, 0.f)};
 #pragma unroll
-            for (int k = 0; k < 8; ++k) mx[k] = fmaxf(s[k], s[8 + k]);
+                for (int ch = 0; ch < kBN / 32; ++ch) {
+                    uint32_t pk[16];
 #pragma unroll
-            for (int c = 16; c < kBN; c += 16)
+                    for (int k = 0; k < 16; ++k) {
+                        const int c = ch * 32 + 2 * k;
+                        const float2 x = fma2(make_float2(s[c], s[c + 1]), sl2x2, nref);
+                        const float2 e = make_float2(ex2(x.x), ex2(x.y));
+                        acc[k & 3] = add2(acc[k & 3], e);
+                        pk[k] = pack_bf16(e.x, e.y);
+                    }
+                    tmem_st16(tS + ch * 16, pk);
+                }
+                const float2 a = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
+                return a.x + a.y;
+            };
+            float rs = 0.f;
+            bool need = j == 0;
+            if (j > 0) {
+                rs = exp_tile(m_ref);
+                need = !(rs <= kTileSumLimit);
+            }
+            if (__any_sync(0xffffffffu, need)) {
+                float mx[8];
 #pragma unroll
-                for (int k = 0; k < 8; ++k) mx[k] = max3(mx[k], s[c + k], s[c + 8 + k]);
-            const float mt = fmaxf(max3(mx[0], mx[1], mx[2]), max3(max3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
-            const float m_new = fmaxf(m_ref, mt * sl2);
-            if (j == 0) {
-                m_ref = (m_new == -INFINITY) ? 0.f : m_new;
-            } else {
-                const bool need = m_new > m_ref + kRescaleThreshold;
-                if (__any_sync(0xffffffffu, need)) {
+                for (int k = 0; k < 8; ++k) mx[k] = fmaxf(s[k], s[8 + k]);
+#pragma unroll
+                for (int c = 16; c < kBN; c += 16)
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) mx[k] = max3(mx[k], s[c + k], s[c + 8 + k]);
+                const float mt = fmaxf(max3(mx[0], mx[1], mx[2]), max3(max3(mx[3], mx[4], mx[5]), mx[6], mx[7]));
+                const float m_new = fmaxf(m_ref, mt * sl2);
+                if (j == 0) {
+                    m_ref = (m_new == -INFINITY) ? 0.f : m_new;
+                } else {
                     // O holds PV of tiles < j once PV(j-1) completed; PV(j) waits for our P
                     if (!wait_bar_warp(b_o, (j - 1) & 1, wctx)) { ok = false; break; }
                     ptx::tc_fence_after();
@@ -458,34 +489,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int k = 0; k < 16; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * alpha);
                         tmem_st16(tO + ch * 16, o);
                     }
-                    ptx::tmem_wait_st();
                     if (need) {
                         l *= alpha;
                         m_ref = m_new;
                     }
                 }
+                ptx::tmem_wait_st();
+                rs = exp_tile(m_ref);
             }
-            // P = exp2(s * scale_log2 - m_ref) as bf16 pairs, written over S's first 64 columns
-            const float2 nref = make_float2(-m_ref, -m_ref);
-            float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                             make_float2(0.f, 0.f)};
-#pragma unroll
-            for (int ch = 0; ch < kBN / 32; ++ch) {
-                uint32_t pk[16];
-#pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    const int c = ch * 32 + 2 * k;
-                    const float2 x = fma2(make_float2(s[c], s[c + 1]), sl2x2, nref);
-                    const float2 e = make_float2(ex2(x.x), ex2(x.y));
-                    acc[k & 3] = add2(acc[k & 3], e);
-                    pk[k] = pack_bf16(e.x, e.y);
-                }
-                tmem_st16(tS + ch * 16, pk);
-            }
-            const float2 a01 = add2(acc[0], acc[1]);
-            const float2 a23 = add2(acc[2], acc[3]);
-            const float2 a = add2(a01, a23);
-            l += a.x + a.y;
+            l += rs;
             ptx::tmem_wait_st();
             ptx::tc_fence_before();
             ptx::mbar_arrive(b_p);

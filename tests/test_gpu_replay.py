@@ -38,15 +38,45 @@ def test_replay_matches_oracle(case):
     assert pair.gpu.device_status() == 0
 
 
-@pytest.mark.parametrize("scale_mult", [4.0, 8.0])
+@pytest.mark.parametrize("scale_mult", [4.0, 8.0, 64.0])
 def test_peaked_logits_exercise_rescaling(scale_mult):
-    """Logit std 4-8: running maxima jump between key tiles, so the lazy rescale
-    of O in TMEM runs.  The output is then close to single value rows (|O| up
-    to max|V|), so the check uses the derived rounding bound."""
+    """Logit std 4 to 64: running maxima jump between key tiles; at 64 later
+    tiles exceed the first tile's max by far more than 2^64 in weight, so the
+    reference moves and O in TMEM is rescaled.  The output is then close to
+    single value rows (|O| up to max|V|), so the check uses the derived
+    rounding bound."""
     d = 128
-    pair, s, outs, refs, inputs = replay_case(1, 32, 8, d, 16, 700, 300, seed=5, scale=scale_mult / math.sqrt(d))
+    pair, s, outs, refs, inputs = replay_case(1, 32, 8, d, 16, 700, 300, seed=5, scale=scale_mult / math.sqrt(d),
+                                              split=0)
     vmax = float(np.abs(synth.bf16_bits_to_f32(np.concatenate([inputs[1], inputs[3]], 1))).max())
     assert_within_rounding_bound(outs[0], refs[0], vmax, f"peaked x{scale_mult}")
+
+
+@pytest.mark.parametrize("split", [0, 1])
+def test_reference_moves_on_large_jump(split):
+    """Keys after the first 128 are scaled by 16 (exact in bf16), so for nearly
+    every row a later tile's logits exceed the first tile's max by far more
+    than 64 in log2 units: the row's reference must move and O be rescaled."""
+    d, hq, hkv, ps, P, S = 128, 32, 8, 16, 600, 100
+    T = P + S
+    npg = -(-T // ps) + 3
+    pair = Pair(1, hkv, d, ps, npg, 1, npg, seed=61)
+    if split:
+        pair.gpu.set_option("splitkv", 1)
+    g = synth.rng(61, 1)
+    f = synth.bf16_bits_to_f32
+    k0 = f(synth.normal_bf16(g, (1, T, hkv, d)))
+    k0[:, 128:] *= 16.0
+    k0 = synth.f32_to_bf16_bits(k0)
+    v0 = synth.normal_bf16(g, (1, T, hkv, d))
+    q = synth.normal_bf16(g, (S, hq, d))
+    s = pair.seq()
+    pair.append(s, k0, v0)
+    scale = 4.0 / math.sqrt(d)
+    out = pair.gpu.replay_attn(s, 0, dev(q), softmax_scale=scale)
+    ref = oracle.replay_attention(pair.orc, s, 0, q, scale)
+    vmax = float(np.abs(f(v0)).max())
+    assert_within_rounding_bound(out, ref, vmax, f"large jump split={split}")
 
 
 def test_multilayer_and_pool_contents():
