@@ -51,11 +51,27 @@ def load_peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
-def make_workload(name):
-    """agent_batch | tiny | short_suffix | long_suffix | tau_sweep_r<ratio> (ratio 0 = full reset)."""
+def make_workload(name, replica=0):
+    """agent_batch | tiny | short_suffix | long_suffix | tau_sweep_r<ratio> (ratio 0 = full reset).
+    replica r > 0 (the rank under torchrun) draws the same shapes from its own seeds."""
     if name.startswith("tau_sweep_r"):
-        return synth.tau_sweep(float(name[len("tau_sweep_r"):]))
-    return synth.WORKLOADS[name]()
+        w = synth.tau_sweep(float(name[len("tau_sweep_r"):]))
+    else:
+        w = synth.WORKLOADS[name]()
+    if replica:
+        w = synth.replica(w, replica)
+    return w
+
+
+def reduce_max(x, dist):
+    """Max over ranks (gloo, on the host) of a float; identity without a process group."""
+    if not dist:
+        return x
+    import torch
+    import torch.distributed as tdist
+    t = torch.tensor([x], dtype=torch.float64)
+    tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+    return float(t.item())
 
 
 def workload_flops(w):
@@ -224,7 +240,7 @@ def run_pe(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     from paper_2609_04875_gb300.driver import ReplayDriver
 
-    w = make_workload(args.workload)
+    w = make_workload(args.workload, replica=rank)
     drv = ReplayDriver(w, device=dev)
     stream = torch.cuda.current_stream(dev)
     L = w.num_layers
@@ -262,11 +278,7 @@ def run_pe(args, rank, world, local_rank):
     clk = clocks.stop() if clocks else None
     elapsed_ms = t_start.elapsed_time(t_end)
     attn_ms = [a.elapsed_time(b) for a, b in attn_ev]
-    if dist:
-        import torch.distributed as tdist
-        t = torch.tensor([elapsed_ms], dtype=torch.float64)
-        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = reduce_max(elapsed_ms, dist)
     ms_per_step = elapsed_ms / args.steps
     value = world * tokens_per_step * args.steps / (elapsed_ms / 1e3)
 
@@ -391,12 +403,7 @@ def run_e2e(drv, dev, steps, world, dist):
     comp.wait_stream(s_out)
     e1.record(comp)
     torch.cuda.synchronize(dev)
-    ms = e0.elapsed_time(e1)
-    if dist:
-        import torch.distributed as tdist
-        t = torch.tensor([ms], dtype=torch.float64)
-        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_max(e0.elapsed_time(e1), dist)
     tokens = world * drv.w.total_suffix * steps
     return {"value": tokens / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
             "d2h_bytes_per_step": d2h_bytes, "steps": steps, "ms_per_step": ms / steps,

@@ -178,6 +178,14 @@ pe_status pe_set_option(pe_cache *cache, const char *key, int64_t value);
  * wait ran out).  clear != 0 resets it.  Returns DEVICE_TIMEOUT if *code != 0. */
 pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *stream);
 
+/* Failure-detection self-test: launches one kernel whose single wait (the same
+ * bounded mbarrier wait the attention kernel uses) is on a barrier nothing
+ * arrives at.  After limit_ns (1 us .. 2 s) the wait gives up, records status
+ * code 1 in the cache's device status word and the kernel returns, leaving the
+ * context usable; pe_device_status then reports DEVICE_TIMEOUT.  The paper has
+ * no counterpart (its failure handling is at the tool level). */
+pe_status pe_selftest_bounded_wait(pe_cache *cache, int64_t limit_ns, void *stream);
+
 /* Number of kernel launches this cache has made so far (crop, append,
  * attention, combine); lets a caller count its device work. */
 pe_status pe_kernel_launches(const pe_cache *cache, int64_t *count);

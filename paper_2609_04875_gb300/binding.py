@@ -27,7 +27,8 @@ EXPORTED = [
     "pe_cache_create", "pe_cache_destroy", "pe_seq_create", "pe_seq_release", "pe_crop", "pe_crop_batch",
     "pe_append_kv", "pe_append_kv_batch", "pe_replay_attn", "pe_replay_attn_batch", "pe_seq_info",
     "pe_seq_page_table", "pe_free_list", "pe_seq_device_page_table", "pe_cache_pools", "pe_set_option",
-    "pe_device_status", "pe_kernel_launches", "pe_replay_attn_static_scratch", "pe_last_error", "pe_version",
+    "pe_device_status", "pe_kernel_launches", "pe_replay_attn_static_scratch", "pe_selftest_bounded_wait",
+    "pe_last_error", "pe_version",
 ]
 
 
@@ -73,6 +74,7 @@ _sigs = {
     "pe_set_option": [_P, ctypes.c_char_p, _I64],
     "pe_device_status": [_P, _I32P, _I32, _P],
     "pe_kernel_launches": [_P, _I64P],
+    "pe_selftest_bounded_wait": [_P, _I64, _P],
     "pe_replay_attn_static_scratch": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
 }
 for _name, _args in _sigs.items():
@@ -304,6 +306,11 @@ class PagedKVCache:
 
     def set_option(self, key: str, value: int):
         _check(_lib.pe_set_option(self._h, key.encode(), int(value)))
+
+    def selftest_bounded_wait(self, limit_ns: int, stream=None):
+        """Launches a kernel whose bounded wait runs out (nothing arrives); the
+        device status word then reads 1.  Tests failure detection without a fault."""
+        _check(_lib.pe_selftest_bounded_wait(self._h, int(limit_ns), self._s(stream)))
 
     def kernel_launches(self) -> int:
         n = ctypes.c_int64()

@@ -75,14 +75,15 @@ struct WaitCtx {
 
 // Bounded mbarrier wait.  Returns false (and stops the CTA's pipeline) when the
 // wait ran out or another role already gave up.
-__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, const WaitCtx &w)
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, const WaitCtx &w,
+                                         uint64_t limit_ns = kWaitNs)
 {
     if (ptx::mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = ptx::globaltimer();
     for (;;) {
         if (ptx::mbar_try_wait(bar, parity)) return true;
         if (*w.abort) return false;
-        if (ptx::globaltimer() - t0 > kWaitNs) {
+        if (ptx::globaltimer() - t0 > limit_ns) {
             *w.abort = 1;
             atomicCAS(w.status, 0, kStatusWaitTimeout);
             return false;
@@ -562,6 +563,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, C::kTmemCols);
     }
+}
+
+// Exercises the bounded wait on its own: one thread waits on an mbarrier that
+// nothing arrives at; after limit_ns the wait gives up, records the status code
+// and the kernel returns normally, leaving the context usable.
+__global__ void bounded_wait_selftest_kernel(int32_t *status, uint64_t limit_ns)
+{
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x != 0) return;
+    const uint32_t b = ptx::smem_addr(&bar);
+    ptx::mbar_init(b, 1);
+    abort_flag = 0;
+    ptx::fence_barrier_init();
+    const WaitCtx w{&abort_flag, status};
+    (void)wait_bar(b, 0, w, limit_ns);
+}
+
+cudaError_t launch_bounded_wait_selftest(int32_t *status, uint64_t limit_ns, cudaStream_t st)
+{
+    bounded_wait_selftest_kernel<<<1, 32, 0, st>>>(status, limit_ns);
+    return cudaGetLastError();
 }
 
 // One warp per output row: LSE-weighted merge of the split partials.

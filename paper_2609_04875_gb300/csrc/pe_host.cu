@@ -891,6 +891,18 @@ pe_status pe_set_option(pe_cache *c, const char *key, int64_t value)
     return PE_OK;
 }
 
+pe_status pe_selftest_bounded_wait(pe_cache *c, int64_t limit_ns, void *stream)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (c->host_only) return fail(PE_ERR_UNSUPPORTED, "host-only cache has no device");
+    if (limit_ns < 1000 || limit_ns > 2000000000ll) return fail(PE_ERR_RANGE, "limit_ns must be in [1 us, 2 s]");
+    cudaError_t e = launch_bounded_wait_selftest(c->d_status, static_cast<uint64_t>(limit_ns),
+                                                 static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "self-test launch");
+    c->launches++;
+    return PE_OK;
+}
+
 pe_status pe_kernel_launches(const pe_cache *c, int64_t *count)
 {
     if (!c || !count) return fail(PE_ERR_INVALID, "null argument");

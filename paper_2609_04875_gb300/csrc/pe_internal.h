@@ -96,6 +96,7 @@ cudaError_t launch_crop(const CropParams &p, cudaStream_t st);
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
                                const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);
+cudaError_t launch_bounded_wait_selftest(int32_t *status, uint64_t limit_ns, cudaStream_t st);
 
 // Fixed split-KV scratch compiled into the library (pe_attn.cu), used only by
 // pe_replay_attn_static_scratch.  static_scratch() returns its device address

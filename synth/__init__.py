@@ -186,9 +186,9 @@ def tiny() -> Workload:
     return _finish(w)
 
 
-def agent_batch(n_agents: int = 16) -> Workload:
+def agent_batch(n_agents: int = 16, seed: int = BASE_SEED + 2) -> Workload:
     """16 agents, 1 layer, GQA 32/8, d=128, ps=16; T ~ U{2048..8192}, tau/T ~ U[0.2, 0.9]; N(0,1)/sqrt(128)."""
-    w = Workload("agent_batch", BASE_SEED + 2, 1, 32, 8, 128, 16, 1.0 / math.sqrt(128))
+    w = Workload("agent_batch", seed, 1, 32, 8, 128, 16, 1.0 / math.sqrt(128))
     g = rng(w.seed, STREAM_LENGTHS)
     for i in range(n_agents):
         T = int(g.integers(2048, 8192, endpoint=True))
@@ -210,6 +210,19 @@ def long_suffix(n_agents: int = 4, prefix: int = 4096, suffix: int = 16384) -> W
     w = Workload("long_suffix", BASE_SEED + 4, 1, 64, 8, 128, 64, 1.0 / math.sqrt(128))
     w.agents = [Agent(T=prefix + suffix, tau=prefix + 1, index=i) for i in range(n_agents)]
     return _finish(w)
+
+
+def replica(w: Workload, r: int) -> Workload:
+    """The same workload shape drawn from replica r's own seeds (one replica per
+    GPU under weak scaling): the base seed moves by 1000 * r.  The agent batch
+    redraws its agents' lengths and injection steps too."""
+    seed = w.seed + 1000 * r
+    if w.name == "agent_batch":
+        return agent_batch(len(w.agents), seed=seed)
+    import copy
+    w2 = copy.deepcopy(w)
+    w2.seed = seed
+    return w2
 
 
 TAU_SWEEP_RATIOS = (0.1, 0.3, 0.5, 0.7, 0.9)
