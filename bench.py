@@ -170,21 +170,23 @@ def oracle_tokens_per_s(w, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "agent_batch": {"bytes": 696.202240e6 + 328.267008e6, "profile": "profiles/replay_attn_agent_batch.md",
-                    "src_sha256": "8f464a14b8867cf08b98323c8adbd93a191e4ab164630cb50790aa344dfe764f"},
+    "agent_batch": {"bytes": 697.009152e6 + 328.204544e6, "profile": "profiles/replay_attn_agent_batch.md",
+                    "src_sha256": "6c7f02193ba40db6058212f482f1f89251554b8b4166af8e998283581fc845c3"},
+    "short_suffix": {"bytes": 1.076274e9 + 21.424384e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
+                     "src_sha256": "6c7f02193ba40db6058212f482f1f89251554b8b4166af8e998283581fc845c3"},
 }
 ATTN_SRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc", "pe_attn.cu")
 
 
 def _src_sha():
-    """sha256 of the attention kernel's source (from its config struct to the
-    end of the kernel), so that recorded counters lapse when the kernel changes."""
+    """sha256 of the attention kernel function's source, so that recorded
+    counters lapse when the kernel changes."""
     import hashlib
     with open(ATTN_SRC) as f:
         txt = f.read()
     try:
-        a = txt.index("template <int HD>\nstruct AttnCfg")
-        b = txt.index("// One warp per output row")
+        a = txt.index("template <int HD, bool SPLIT>\n__global__")
+        b = txt.index("// Exercises the bounded wait on its own")
     except ValueError:
         return None
     return hashlib.sha256(txt[a:b].encode()).hexdigest()
@@ -197,7 +199,7 @@ def traffic_for(workload):
     return t["bytes"], t["profile"]
 
 
-def roofline_for(w, flops_launch, bytes_launch, attn_s, peaks, peak_src):
+def roofline_for(w, flops_launch, bytes_launch, attn_s, peaks, peak_src, plan=(False, 1, 0)):
     """Per-launch roofline of the replay-attention kernel: the slower of its
     algorithmic FLOPs at the bf16 tensor peak and its algorithmic bytes at HBM
     bandwidth decides the bound."""
@@ -217,7 +219,8 @@ def roofline_for(w, flops_launch, bytes_launch, attn_s, peaks, peak_src):
     r["frac"] = r["achieved"] / r["peak"]
     r["traffic"] = traffic
     r["traffic_profile"] = prof
-    r["kernel"] = f"replay_attn_kernel<{w.head_dim},{'split' if w.name == 'short_suffix' else 'nosplit'}>"
+    r["kernel"] = f"replay_attn_kernel<{w.head_dim},{'split' if plan[0] else 'single'}>"
+    r["plan"] = {"split_kv": plan[0], "key_splits": plan[1], "ctas": plan[2]}
     r["attn_ms_per_launch"] = attn_s * 1e3
     r["algorithmic_flop_per_launch"] = flops_launch
     r["algorithmic_bytes_per_launch"] = bytes_launch
@@ -311,7 +314,7 @@ def run_pe(args, rank, world, local_rank):
     peaks, peak_src = load_peaks()
     flops = workload_flops(w) / L  # per attention launch (one per layer)
     attn_avg_s = statistics.mean(attn_ms) / 1e3
-    roof = roofline_for(w, flops, attn_bytes(w), attn_avg_s, peaks, peak_src)
+    roof = roofline_for(w, flops, attn_bytes(w), attn_avg_s, peaks, peak_src, drv.cache.last_attn_plan())
     result = {
         "metric": METRIC,
         "value": value,

@@ -186,6 +186,11 @@ pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *
  * no counterpart (its failure handling is at the tool level). */
 pe_status pe_selftest_bounded_wait(pe_cache *cache, int64_t limit_ns, void *stream);
 
+/* Plan of the most recent replay-attention launch group on this cache: split
+ * = 1 when the split-KV path (with its combine launch) ran, n_splits = key
+ * splits of its first sequence, ctas = attention CTAs launched. */
+pe_status pe_last_attn_plan(const pe_cache *cache, int32_t *split, int32_t *n_splits, int32_t *ctas);
+
 /* Number of kernel launches this cache has made so far (crop, append,
  * attention, combine); lets a caller count its device work. */
 pe_status pe_kernel_launches(const pe_cache *cache, int64_t *count);

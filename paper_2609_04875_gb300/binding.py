@@ -28,7 +28,7 @@ EXPORTED = [
     "pe_append_kv", "pe_append_kv_batch", "pe_replay_attn", "pe_replay_attn_batch", "pe_seq_info",
     "pe_seq_page_table", "pe_free_list", "pe_seq_device_page_table", "pe_cache_pools", "pe_set_option",
     "pe_device_status", "pe_kernel_launches", "pe_replay_attn_static_scratch", "pe_selftest_bounded_wait",
-    "pe_last_error", "pe_version",
+    "pe_last_attn_plan", "pe_last_error", "pe_version",
 ]
 
 
@@ -75,6 +75,7 @@ _sigs = {
     "pe_device_status": [_P, _I32P, _I32, _P],
     "pe_kernel_launches": [_P, _I64P],
     "pe_selftest_bounded_wait": [_P, _I64, _P],
+    "pe_last_attn_plan": [_P, _I32P, _I32P, _I32P],
     "pe_replay_attn_static_scratch": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
 }
 for _name, _args in _sigs.items():
@@ -311,6 +312,12 @@ class PagedKVCache:
         """Launches a kernel whose bounded wait runs out (nothing arrives); the
         device status word then reads 1.  Tests failure detection without a fault."""
         _check(_lib.pe_selftest_bounded_wait(self._h, int(limit_ns), self._s(stream)))
+
+    def last_attn_plan(self):
+        """(split path used, key splits, attention CTAs) of the last attention launch."""
+        a, b, c = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+        _check(_lib.pe_last_attn_plan(self._h, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
+        return bool(a.value), b.value, c.value
 
     def kernel_launches(self) -> int:
         n = ctypes.c_int64()

@@ -87,6 +87,7 @@ struct pe_cache {
     // options
     int splitkv = -1, num_splits = 0, debug_poison = 0;
     int64_t launches = 0;
+    int32_t last_split = 0, last_splits = 0, last_ctas = 0;  // plan of the last attention launch
 };
 
 namespace {
@@ -375,12 +376,13 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         }
         // Estimated time with s key splits: the CTAs run in ceil(C s / N) waves of
         // (W/s + 2) tile times (about 1.5 us per tile, compute- or HBM-bound
-        // alike); splits add their fp32 partials' HBM round trip and a combine launch.
+        // alike), and never faster than the longest CTA (max_tiles/s + 2);
+        // splits add their fp32 partials' HBM round trip and a combine launch.
         const double W = C > 0 ? static_cast<double>(tiles) / C : 0.0;
         const int64_t row_bytes = static_cast<int64_t>(d) * 4 + 4;
         auto cost = [&](int64_t sp) {
             const double waves = std::ceil(static_cast<double>(C * sp) / c->num_sms);
-            double t = waves * (W / sp + 2.0) * 1.5e-6;
+            double t = std::max(waves * (W / sp + 2.0), static_cast<double>(max_tiles) / sp + 2.0) * 1.5e-6;
             if (sp > 1) t += static_cast<double>(rows * sp * row_bytes * 2) / 6.0e12 + 5e-6;
             return t;
         };
@@ -462,6 +464,9 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         bool split = false;
         s = plan_group(lo, hi, p, split);
         if (s != PE_OK) return s;
+        c->last_split = split ? 1 : 0;
+        c->last_splits = split ? p.seqs[0].n_splits : 1;
+        c->last_ctas = p.total_items;
         cudaError_t e = launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, p, st);
         if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
         c->launches++;
@@ -900,6 +905,15 @@ pe_status pe_selftest_bounded_wait(pe_cache *c, int64_t limit_ns, void *stream)
                                                  static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "self-test launch");
     c->launches++;
+    return PE_OK;
+}
+
+pe_status pe_last_attn_plan(const pe_cache *c, int32_t *split, int32_t *n_splits, int32_t *ctas)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (split) *split = c->last_split;
+    if (n_splits) *n_splits = c->last_splits;
+    if (ctas) *ctas = c->last_ctas;
     return PE_OK;
 }
 

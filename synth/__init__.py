@@ -198,6 +198,16 @@ def agent_batch(n_agents: int = 16, seed: int = BASE_SEED + 2) -> Workload:
     return _finish(w)
 
 
+def decode_batch(n_agents: int = 16, seed: int = BASE_SEED + 6) -> Workload:
+    """Decode after replay: the 16 agents of the agent batch each generate one
+    token (S = 1, P = T - 1): the last position is cropped and recomputed, so
+    steps repeat without growing the caches."""
+    base = agent_batch(n_agents, seed=seed - 4)  # the agent batch's lengths (seed + 2 <-> + 6)
+    w = Workload("decode_batch", seed, 1, 32, 8, 128, 16, 1.0 / math.sqrt(128))
+    w.agents = [Agent(T=a.T, tau=a.T, index=i) for i, a in enumerate(base.agents)]
+    return _finish(w)
+
+
 def short_suffix(n_agents: int = 8, prefix: int = 32768, suffix: int = 16) -> Workload:
     """8 agents, GQA 32/8, d=128, ps=16; prefix 32k, suffix 16; N(0,1)/sqrt(128)."""
     w = Workload("short_suffix", BASE_SEED + 3, 1, 32, 8, 128, 16, 1.0 / math.sqrt(128))
@@ -219,6 +229,8 @@ def replica(w: Workload, r: int) -> Workload:
     seed = w.seed + 1000 * r
     if w.name == "agent_batch":
         return agent_batch(len(w.agents), seed=seed)
+    if w.name == "decode_batch":
+        return decode_batch(len(w.agents), seed=seed)
     import copy
     w2 = copy.deepcopy(w)
     w2.seed = seed
@@ -242,6 +254,7 @@ def tau_sweep(ratio: float, T: int = 16384, num_layers: int = 32) -> Workload:
 WORKLOADS = {
     "tiny": tiny,
     "agent_batch": agent_batch,
+    "decode_batch": decode_batch,
     "short_suffix": short_suffix,
     "long_suffix": long_suffix,
 }

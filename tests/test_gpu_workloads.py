@@ -109,6 +109,18 @@ def test_agent_batch():
     _check_bookkeeping(drv, steps=2)
 
 
+def test_decode_batch():
+    """Decode after replay: one new token per agent (n_q = 1) over the full cache."""
+    w = synth.decode_batch()
+    drv, inputs = _run(w)
+    _check_bookkeeping(drv)
+    _check_attention(drv, inputs, range(len(w.agents)), [0], n_random=0)
+    first = drv.out.clone()
+    drv.step()
+    torch.cuda.synchronize()
+    assert torch.equal(first, drv.out)
+
+
 def test_short_suffix_splitkv():
     w = synth.short_suffix()
     drv, inputs = _run(w)
