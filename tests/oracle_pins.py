@@ -317,3 +317,135 @@ def pin_bookkeeping(orc, n_ops=400):
             except orc.OracleError:
                 pass
         check_invariants(c, num_pages)
+
+
+# ---------------------------------------------------------------------------
+def load_fork_trace():
+    with open(os.path.join(GOLDEN, "fork_trace.json")) as f:
+        return json.load(f)
+
+
+def run_fork_trace(orc, trace):
+    """Replays the hand-derived fork / copy-on-write / checkpoint trace."""
+    cfg = trace["config"]
+    c = orc.OracleKVCache(cfg["num_layers"], cfg["num_kv_heads"], cfg["head_dim"], cfg["page_size"],
+                          cfg["num_pages"], cfg["max_seqs"], cfg["max_pages_per_seq"],
+                          init_free_order=cfg["init_free_order"])
+    hkv, d = cfg["num_kv_heads"], cfg["head_dim"]
+    codes = {}  # seq -> per-token value code currently expected at that position
+    for idx, st in enumerate(trace["steps"]):
+        op, seq = st["op"], st.get("seq")
+        try:
+            if op == "create":
+                s = c.seq_create()
+                assert s == st["expect_seq"], f"step {idx}"
+                codes[s] = []
+                continue
+            if op == "append":
+                n = st["n"]
+                base = c.length[seq]
+                code = (1000 * idx + base + np.arange(n)).astype(np.uint16)
+                kb = np.broadcast_to(code[None, :, None, None], (1, n, hkv, d)).copy()
+                c.append(seq, kb, kb ^ np.uint16(0x4000))
+                codes[seq] = codes[seq][:base] + [int(x) for x in code]
+            elif op == "checkpoint":
+                for b in st["offsets"]:
+                    c.checkpoint_add(seq, b)
+                continue
+            elif op == "fork":
+                s = c.seq_fork(seq)
+                assert s == st["expect_seq"], f"step {idx}"
+                codes[s] = list(codes[seq])
+            elif op == "crop":
+                freed = c.crop(seq, st["tau"])
+                assert freed == st["expect_freed"], f"step {idx}: freed {freed}"
+                codes[seq] = codes[seq][: st["tau"] - 1]
+            elif op == "restore":
+                b, freed = c.restore(seq, st["tau"])
+                assert b == st["expect_offset"], f"step {idx}: offset {b}"
+                assert freed == st["expect_freed"], f"step {idx}: freed {freed}"
+                codes[seq] = codes[seq][:b]
+            elif op == "release":
+                freed = c.seq_release(seq)
+                assert freed == st["expect_freed"], f"step {idx}: freed {freed}"
+                assert c.free_list() == st["expect_free"], f"step {idx}"
+                del codes[seq]
+                continue
+        except orc.OracleError as e:
+            assert st.get("expect_error") == e.kind, f"step {idx}: unexpected {e.kind}"
+            continue
+        assert "expect_error" not in st, f"step {idx}"
+        ex = st.get("expect", {})
+        s = ex.get("seq", seq)
+        if "table" in ex:
+            assert c.page_table(s) == ex["table"], f"step {idx}: table {c.page_table(s)}"
+        if "len" in ex:
+            assert c.length[s] == ex["len"], f"step {idx}"
+        if "free" in ex:
+            assert c.free_list() == ex["free"], f"step {idx}: free {c.free_list()}"
+        for pg, r in ex.get("refs", {}).items():
+            assert c.refs[int(pg)] == r, f"step {idx}: refs[{pg}] = {c.refs[int(pg)]}"
+        if "checkpoints" in ex:
+            assert c.checkpoints[s] == ex["checkpoints"], f"step {idx}"
+        for tok, page, slot, _ in st.get("slots", []):
+            assert c.page_table(seq)[tok // cfg["page_size"]] == page, f"step {idx}: token {tok}"
+            assert np.all(c.k_pool[0, page, :, slot, :] == codes[seq][tok]), f"step {idx}: slot of {tok}"
+        for q, cq in codes.items():   # every branch still reads its own tokens
+            k, _ = c.gather(q, 0)
+            assert np.array_equal(k[:, 0, 0], np.array(cq, dtype=np.uint16)), f"step {idx}: seq {q} content"
+    return c
+
+
+def check_ref_invariants(c, num_pages):
+    counts = [0] * num_pages
+    for s in c.table:
+        for p in c.table[s]:
+            counts[p] += 1
+    assert counts == list(c.refs), "reference counts != table occurrences"
+    assert sorted(c.free) == [p for p in range(num_pages) if counts[p] == 0], "free list != unreferenced pages"
+    for s in c.table:
+        assert len(c.table[s]) == c.pages_for(c.length[s]), "table size != ceil(len / ps)"
+
+
+def pin_fork(orc, n_ops=400):
+    run_fork_trace(orc, load_fork_trace())
+    g = synth.rng(5151, 0)
+    ps, num_pages, L, hkv, d = 4, 48, 1, 1, 1
+    c = orc.OracleKVCache(L, hkv, d, ps, num_pages, 6, 40, init_free_order=synth.page_permutation(5151, num_pages))
+    codes = {}
+    s0 = c.seq_create()
+    codes[s0] = []
+    step = 0
+    for _ in range(n_ops):
+        step += 1
+        live = list(c.table)
+        s = live[int(g.integers(0, len(live)))]
+        r = g.random()
+        try:
+            if r < 0.2 and len(live) < 6:
+                t = c.seq_fork(s)
+                codes[t] = list(codes[s])
+            elif r < 0.45:
+                tau = int(g.integers(1, c.length[s] + 2))
+                c.crop(s, tau)
+                codes[s] = codes[s][: tau - 1]
+            elif r < 0.55:
+                c.checkpoint_add(s, int(g.integers(0, c.length[s] + 1)))
+            elif r < 0.62 and c.checkpoints[s]:
+                b, _ = c.restore(s, int(g.integers(1, c.length[s] + 2)))
+                codes[s] = codes[s][:b]
+            elif r < 0.68 and len(live) > 1:
+                c.seq_release(s)
+                del codes[s]
+            else:
+                n = int(g.integers(0, 9))
+                base = c.length[s]
+                code = ((step * 37 + base + np.arange(n)) % 60000).astype(np.uint16)
+                c.append(s, code[None, :, None, None].copy(), code[None, :, None, None].copy())
+                codes[s] = codes[s][:base] + [int(x) for x in code]
+        except orc.OracleError:
+            pass
+        check_ref_invariants(c, num_pages)
+        for q in c.table:
+            k, v = c.gather(q, 0)
+            assert np.array_equal(k[:, 0, 0], np.array(codes[q], dtype=np.uint16)), "a branch lost its content"

@@ -21,11 +21,16 @@ MUTANTS = [
     ("value_from_keys", "attention.c", "const uint16_t *vrow = jb->v +", "const uint16_t *vrow = jb->k +"),
     ("unnormalised", "attention.c", "o[c] /= den;", "o[c] /= 1.0;"),
     ("crop_keeps_tau", "kvcache.py", "new_len = tau - 1\n", "new_len = min(tau, n)\n"),
-    ("push_ascending", "kvcache.py", "for p in reversed(freed):          # descending", "for p in freed:  #"),
+    ("push_ascending", "kvcache.py", "for p in reversed(pages):", "for p in pages:"),
     ("slot_shift", "kvcache.py", "page, slot = tbl[pos // self.ps], pos % self.ps",
      "page, slot = tbl[pos // self.ps], (pos + 1) % self.ps"),
-    ("counter_not_reset", "kvcache.py", "self.appended[seq] = 0\n        return list(freed)",
-     "return list(freed)"),
+    ("counter_not_reset", "kvcache.py", "self.length[seq] = new_len\n        self.appended[seq] = 0\n",
+     "self.length[seq] = new_len\n"),
+    ("cow_skipped", "kvcache.py", "cow = n > 0 and old % self.ps != 0 and self.refs[tbl[-1]] > 1",
+     "cow = False"),
+    ("fork_no_ref", "kvcache.py", "        for p in self.table[s]:\n            self.refs[p] += 1\n", ""),
+    ("checkpoint_le_tau", "kvcache.py", "cands = [b for b in self.checkpoints[seq] if b < tau]",
+     "cands = [b for b in self.checkpoints[seq] if b <= tau]"),
 ]
 
 
@@ -47,7 +52,7 @@ def _load_mutant(tmp_path, name, fname, old, new):
 def _pins_fail(mod):
     checks = [lambda: pins.pin_bruteforce(mod, full=False), lambda: pins.pin_closed_forms(mod),
               lambda: pins.pin_splice(mod), lambda: pins.pin_corollary(mod),
-              lambda: pins.pin_bookkeeping(mod, n_ops=150)]
+              lambda: pins.pin_bookkeeping(mod, n_ops=150), lambda: pins.pin_fork(mod, n_ops=150)]
     caught = 0
     for chk in checks:
         try:

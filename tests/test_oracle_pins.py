@@ -51,3 +51,7 @@ def test_error_rules():
         c.append(s2, n_tokens=1)    # pool exhausted
     assert e.value.kind == "oom"
     assert c.seq_info(s2) == (8, 8) and len(c.free) == 0
+
+
+def test_fork_copy_on_write_checkpoints():
+    pins.pin_fork(oracle)
