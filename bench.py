@@ -306,6 +306,20 @@ def run_pe(args, rank, world, local_rank):
         append_ms.append(e1.elapsed_time(e2))
     torch.cuda.synchronize(dev)
 
+    # ---- branching from the base (fork + release of every agent) and checkpoint restore
+    fork_us, rel_us = [], []
+    for _ in range(10):
+        torch.cuda.synchronize(dev)
+        h0 = time.perf_counter()
+        forks = [drv.cache.seq_fork(s) for s in drv.seqs]
+        h1 = time.perf_counter()
+        for f in forks:
+            drv.cache.seq_release(f)
+        h2 = time.perf_counter()
+        fork_us.append((h1 - h0) * 1e6 / len(forks))
+        rel_us.append((h2 - h1) * 1e6 / len(forks))
+    torch.cuda.synchronize(dev)
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -341,6 +355,8 @@ def run_pe(args, rank, world, local_rank):
                               "crop": statistics.median(crop_dev_us) / 1e3},
         "crop_us": {"host_call_median": statistics.median(crop_host_us),
                     "device_median": statistics.median(crop_dev_us), "agents": len(w.agents)},
+        "fork_us": {"host_per_fork_median": statistics.median(fork_us),
+                    "host_per_release_median": statistics.median(rel_us)},
         "recomputed_tokens": tokens_per_step,
         "session_tokens": sum(a.T for a in w.agents),
         "gpu_launches": launches,

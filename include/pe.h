@@ -32,7 +32,8 @@
  *     concurrently.
  *   - Allocation policy: the free list is a LIFO stack whose initial pop order
  *     is `init_free_order`; an append pops one page per new logical page; crop
- *     and release push the removed pages in descending logical order, so a
+ *     and release drop one reference per removed page in descending logical
+ *     order and push the pages whose last reference goes, so (without forks) a
  *     crop followed by an append of the same length restores the same table.
  */
 #ifndef PE_H
@@ -86,13 +87,38 @@ pe_status pe_seq_release(pe_cache *cache, int32_t seq, void *stream);
 
 /* Crop = restore (Sec. 3.4(b); Alg. 1 Restore).  Keeps the first tau-1 tokens:
  * pages at logical index >= ceil((tau-1)/ps) are removed from the table and
- * pushed on the free list; the device table entries are set to -1 by a kernel
- * on `stream`.  Resets the recomputation counter to 0.  tau = len+1 keeps
- * every token.  freed_out (host, nullable) receives the freed page ids in
+ * lose one reference each (visited in descending logical order); a page whose
+ * last reference goes is pushed on the free list.  The device table entries
+ * are set to -1 by a kernel on `stream`.  Resets the recomputation counter to
+ * 0 and drops checkpoints past the new length.  tau = len+1 keeps every token.
+ * freed_out (host, nullable) receives the pages returned to the free list in
  * ascending logical order; n_freed (nullable) their number.
  * Errors: INVALID (tau < 1, unknown seq), RANGE (tau-1 > len, freed_cap too small). */
 pe_status pe_crop(pe_cache *cache, int32_t seq, int64_t tau, int32_t *freed_out, int32_t freed_cap,
                   int32_t *n_freed, void *stream);
+
+/* Branching from one base state (Sec. 4.1: every method starts from the same
+ * contaminated base, the cache cloned).  The new sequence (lowest free slot)
+ * shares every page of `seq` (reference counts), its length, counter and
+ * checkpoints; no K/V is copied.  An append into a shared, partially filled
+ * last page first copies that page's valid slots into a fresh page on
+ * `stream` (copy-on-write); full shared pages are never written.
+ * Errors: INVALID (unknown seq), OOM (no sequence slot). */
+pe_status pe_seq_fork(pe_cache *cache, int32_t seq, int32_t *new_seq, void *stream);
+
+/* Metadata-only checkpoints (Sec. 3.4(b), Sec. 4.6): a checkpoint is a token
+ * offset b, the state after the first b tokens.  pe_checkpoint_add records one
+ * (0 <= b <= len; duplicates ignored; RANGE otherwise).  pe_checkpoint_select
+ * returns c* = the largest recorded offset b < tau (Alg. 1: the last boundary
+ * before the target's entry; RANGE when none, INVALID when tau < 1).
+ * pe_restore = select + crop to keep c* tokens (Alg. 1 Restore); the caller
+ * then replays positions c*+1 .. T.  pe_seq_checkpoints lists the offsets
+ * (ascending). */
+pe_status pe_checkpoint_add(pe_cache *cache, int32_t seq, int64_t offset);
+pe_status pe_checkpoint_select(const pe_cache *cache, int32_t seq, int64_t tau, int64_t *offset);
+pe_status pe_restore(pe_cache *cache, int32_t seq, int64_t tau, int64_t *offset, int32_t *freed_out,
+                     int32_t freed_cap, int32_t *n_freed, void *stream);
+pe_status pe_seq_checkpoints(const pe_cache *cache, int32_t seq, int64_t *out, int32_t cap, int32_t *n);
 
 /* Crops n sequences (host arrays seqs[n], taus[n]) with one device launch.
  * All-or-nothing: every (seq, tau) is validated before any state changes;
@@ -158,6 +184,8 @@ pe_status pe_replay_attn_static_scratch(pe_cache *cache, int32_t seq, int32_t la
 pe_status pe_seq_info(const pe_cache *cache, int32_t seq, int64_t *len, int64_t *appended_since_crop);
 pe_status pe_seq_page_table(const pe_cache *cache, int32_t seq, int32_t *out, int32_t cap, int32_t *n);
 pe_status pe_free_list(const pe_cache *cache, int32_t *out, int32_t cap, int32_t *n); /* top of stack first */
+/* Reference count of every page (out[num_pages]; 0 = on the free list). */
+pe_status pe_page_refs(const pe_cache *cache, int32_t *out, int32_t cap);
 
 /* Synchronous copy of a sequence's DEVICE page-table row (first `cap` entries)
  * into host `out`, after all work on `stream`; for checking the mirror. */

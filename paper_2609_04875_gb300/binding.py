@@ -28,7 +28,8 @@ EXPORTED = [
     "pe_append_kv", "pe_append_kv_batch", "pe_replay_attn", "pe_replay_attn_batch", "pe_seq_info",
     "pe_seq_page_table", "pe_free_list", "pe_seq_device_page_table", "pe_cache_pools", "pe_set_option",
     "pe_device_status", "pe_kernel_launches", "pe_replay_attn_static_scratch", "pe_selftest_bounded_wait",
-    "pe_last_attn_plan", "pe_last_error", "pe_version",
+    "pe_last_attn_plan", "pe_seq_fork", "pe_checkpoint_add", "pe_checkpoint_select", "pe_restore",
+    "pe_seq_checkpoints", "pe_page_refs", "pe_last_error", "pe_version",
 ]
 
 
@@ -76,6 +77,12 @@ _sigs = {
     "pe_kernel_launches": [_P, _I64P],
     "pe_selftest_bounded_wait": [_P, _I64, _P],
     "pe_last_attn_plan": [_P, _I32P, _I32P, _I32P],
+    "pe_seq_fork": [_P, _I32, _I32P, _P],
+    "pe_checkpoint_add": [_P, _I32, _I64],
+    "pe_checkpoint_select": [_P, _I32, _I64, _I64P],
+    "pe_restore": [_P, _I32, _I64, _I64P, _I32P, _I32, _I32P, _P],
+    "pe_seq_checkpoints": [_P, _I32, _I64P, _I32, _I32P],
+    "pe_page_refs": [_P, _I32P, _I32],
     "pe_replay_attn_static_scratch": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
 }
 for _name, _args in _sigs.items():
@@ -196,6 +203,42 @@ class PagedKVCache:
 
     def seq_release(self, seq, stream=None):
         _check(_lib.pe_seq_release(self._h, seq, self._s(stream)))
+
+    def seq_fork(self, seq, stream=None) -> int:
+        """New sequence sharing all of ``seq``'s pages (copy-on-write on append)."""
+        out = ctypes.c_int32()
+        _check(_lib.pe_seq_fork(self._h, seq, ctypes.byref(out), self._s(stream)))
+        return out.value
+
+    # -- checkpoints (metadata only) --------------------------------------------
+    def checkpoint_add(self, seq, offset):
+        _check(_lib.pe_checkpoint_add(self._h, seq, int(offset)))
+
+    def checkpoint_select(self, seq, tau) -> int:
+        out = ctypes.c_int64()
+        _check(_lib.pe_checkpoint_select(self._h, seq, int(tau), ctypes.byref(out)))
+        return out.value
+
+    def checkpoints(self, seq):
+        n = ctypes.c_int32()
+        _check(_lib.pe_seq_checkpoints(self._h, seq, None, 0, ctypes.byref(n)))
+        buf = (ctypes.c_int64 * max(1, n.value))()
+        _check(_lib.pe_seq_checkpoints(self._h, seq, buf, n.value, ctypes.byref(n)))
+        return list(buf[: n.value])
+
+    def restore(self, seq, tau, stream=None):
+        """Restore(c*): crop to the last checkpoint before tau; returns (offset, freed pages)."""
+        cap = self.max_pages_per_seq
+        buf = (ctypes.c_int32 * cap)()
+        n = ctypes.c_int32()
+        off = ctypes.c_int64()
+        _check(_lib.pe_restore(self._h, seq, int(tau), ctypes.byref(off), buf, cap, ctypes.byref(n), self._s(stream)))
+        return off.value, list(buf[: n.value])
+
+    def page_refs(self):
+        buf = (ctypes.c_int32 * self.num_pages)()
+        _check(_lib.pe_page_refs(self._h, buf, self.num_pages))
+        return list(buf)
 
     # -- crop (restore) --------------------------------------------------------
     def crop(self, seq, tau, stream=None):

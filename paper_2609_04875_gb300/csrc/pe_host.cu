@@ -72,6 +72,8 @@ struct pe_cache {
     std::vector<std::vector<int32_t>> table;       // per sequence slot
     std::vector<int64_t> len, appended;
     std::vector<uint8_t> alive;
+    std::vector<int32_t> refs;                     // sequences holding each page (0 = free)
+    std::vector<std::vector<int64_t>> ckpt;        // per sequence: checkpoint token offsets, ascending
     // device state
     int device = 0;
     int num_sms = 148;
@@ -149,29 +151,47 @@ void free_device(pe_cache *c)
     c->d_ws = nullptr;
 }
 
-// ---- crop bookkeeping shared by pe_crop, pe_crop_batch and pe_seq_release
+// ---- crop bookkeeping shared by pe_crop, pe_crop_batch, pe_restore and pe_seq_release
 struct CropPlan {
     int32_t seq;
     int32_t keep, old_n;
     int64_t new_len;
+    int32_t n_freed;                 // pages whose last reference this crop drops
+    std::vector<int32_t> freed;      // filled by apply_crop, ascending logical order
+    int32_t tail_page = -1;          // last kept page when this sequence is its only holder
 };
 
-void apply_crop(pe_cache *c, const CropPlan &pl, int32_t *freed_out)
+// Drops one reference per removed page (descending logical order); a page whose
+// last reference goes is pushed onto the free list.
+void apply_crop(pe_cache *c, CropPlan &pl, int32_t *freed_out)
 {
     std::vector<int32_t> &t = c->table[pl.seq];
-    for (int32_t e = pl.keep; e < pl.old_n; ++e)
-        if (freed_out) freed_out[e - pl.keep] = t[e];
-    for (int32_t e = pl.old_n - 1; e >= pl.keep; --e)  // descending logical order onto the stack
-        c->free_stack.push_back(t[e]);
+    std::vector<int32_t> freed_desc;
+    for (int32_t e = pl.old_n - 1; e >= pl.keep; --e) {
+        const int32_t pg = t[e];
+        if (--c->refs[pg] == 0) {
+            c->free_stack.push_back(pg);
+            freed_desc.push_back(pg);
+        }
+    }
+    pl.freed.assign(freed_desc.rbegin(), freed_desc.rend());
+    if (freed_out) std::copy(pl.freed.begin(), pl.freed.end(), freed_out);
     t.resize(pl.keep);
     c->len[pl.seq] = pl.new_len;
     c->appended[pl.seq] = 0;
+    std::vector<int64_t> &ck = c->ckpt[pl.seq];
+    while (!ck.empty() && ck.back() > pl.new_len) ck.pop_back();
+    pl.tail_page = (pl.keep > 0 && pl.new_len % c->cfg.page_size != 0 && c->refs[t[pl.keep - 1]] == 1)
+                       ? t[pl.keep - 1]
+                       : -1;
 }
 
 pe_status launch_crops(pe_cache *c, const std::vector<CropPlan> &plans, cudaStream_t st)
 {
     if (c->host_only) return PE_OK;
-    CropParams p{};
+    std::vector<char> buf(sizeof(CropParams));
+    CropParams &p = *reinterpret_cast<CropParams *>(buf.data());
+    std::memset(&p, 0, sizeof p);
     p.page_table = c->d_table;
     p.seq_len = c->d_len;
     p.k_pool = static_cast<uint4 *>(c->k_pool);
@@ -185,14 +205,23 @@ pe_status launch_crops(pe_cache *c, const std::vector<CropPlan> &plans, cudaStre
     size_t i = 0;
     while (i < plans.size()) {
         p.n = 0;
+        int32_t nf = 0;
         while (i < plans.size() && p.n < kMaxCropSegs) {
-            const CropPlan &pl = plans[i++];
+            const CropPlan &pl = plans[i];
+            const int32_t want = c->debug_poison ? static_cast<int32_t>(pl.freed.size()) : 0;
+            if (p.n > 0 && nf + want > kMaxCropFreed) break;  // next launch
+            ++i;
             CropSeg &sg = p.segs[p.n++];
             sg.table_row = pl.seq * c->cfg.max_pages_per_seq;
             sg.keep = pl.keep;
             sg.old_n = pl.old_n;
             sg.seq = pl.seq;
             sg.new_len = pl.new_len;
+            sg.freed0 = nf;
+            sg.n_freed = std::min(want, kMaxCropFreed - nf);
+            for (int32_t k = 0; k < sg.n_freed; ++k) p.freed[nf + k] = pl.freed[k];
+            nf += sg.n_freed;
+            sg.tail_page = pl.tail_page;
         }
         cudaError_t e = launch_crop(p, st);
         if (e != cudaSuccess) return cuda_fail(e, "crop kernel launch");
@@ -213,6 +242,8 @@ pe_status plan_crop(const pe_cache *c, int32_t seq, int64_t tau, CropPlan *pl)
     pl->new_len = tau - 1;
     pl->keep = static_cast<int32_t>(ceil_div(tau - 1, c->cfg.page_size));
     pl->old_n = static_cast<int32_t>(c->table[seq].size());
+    pl->n_freed = 0;
+    for (int32_t e = pl->keep; e < pl->old_n; ++e) pl->n_freed += c->refs[c->table[seq][e]] == 1 ? 1 : 0;
     return PE_OK;
 }
 
@@ -221,7 +252,8 @@ struct AppendPlan {
     int32_t seq;
     int32_t tok0;  // offset in the packed K/V
     int32_t n;
-    int32_t need;  // pages to pop
+    int32_t need;  // pages to pop (including the copy-on-write page)
+    bool cow;      // the partial last page is shared: copy it before writing
 };
 
 pe_status plan_append(const pe_cache *c, int32_t seq, int64_t n, AppendPlan *pl)
@@ -237,7 +269,32 @@ pe_status plan_append(const pe_cache *c, int32_t seq, int64_t n, AppendPlan *pl)
     if (new_len > INT32_MAX) return fail(PE_ERR_RANGE, "sequence length exceeds int32");
     pl->seq = seq;
     pl->n = static_cast<int32_t>(n);
-    pl->need = static_cast<int32_t>(pages - static_cast<int64_t>(c->table[seq].size()));
+    const std::vector<int32_t> &t = c->table[seq];
+    pl->cow = n > 0 && c->len[seq] % c->cfg.page_size != 0 && c->refs[t.back()] > 1;
+    pl->need = static_cast<int32_t>(pages - static_cast<int64_t>(t.size())) + (pl->cow ? 1 : 0);
+    return PE_OK;
+}
+
+// Copy-on-write of a sequence's shared, partially filled last page: pop a
+// fresh page, copy the valid slots on the device, drop one reference.
+pe_status apply_cow(pe_cache *c, int32_t seq, cudaStream_t st)
+{
+    std::vector<int32_t> &t = c->table[seq];
+    const int32_t src = t.back();
+    const int32_t dst = c->free_stack.back();
+    c->free_stack.pop_back();
+    c->refs[dst] = 1;
+    c->refs[src] -= 1;
+    t.back() = dst;
+    if (!c->host_only) {
+        const int32_t slots = static_cast<int32_t>(c->len[seq] % c->cfg.page_size);
+        int32_t *entry = c->d_table + static_cast<int64_t>(seq) * c->cfg.max_pages_per_seq + (t.size() - 1);
+        cudaError_t e = launch_cow_copy(static_cast<uint4 *>(c->k_pool), static_cast<uint4 *>(c->v_pool), src, dst,
+                                        slots, c->cfg.num_layers, c->cfg.num_kv_heads, c->cfg.page_size,
+                                        c->cfg.head_dim / 8, c->cfg.num_pages, entry, st);
+        if (e != cudaSuccess) return cuda_fail(e, "copy-on-write launch");
+        c->launches++;
+    }
     return PE_OK;
 }
 
@@ -281,6 +338,10 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
     };
     int32_t pages_in_launch = 0;
     for (const AppendPlan &pl : plans) {
+        if (pl.cow) {
+            pe_status s = apply_cow(c, pl.seq, st);
+            if (s != PE_OK) return s;
+        }
         int32_t done = 0;
         while (done < pl.n) {
             const int64_t len0 = c->len[pl.seq];
@@ -315,6 +376,7 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
             for (int32_t i = 0; i < need; ++i) {
                 const int32_t pg = c->free_stack.back();
                 c->free_stack.pop_back();
+                c->refs[pg] = 1;
                 t.push_back(pg);
                 if (!c->host_only) p->new_pages[pages_in_launch + i] = pg;
             }
@@ -361,7 +423,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     // split-KV decision over the whole launch group
     auto plan_group = [&](size_t lo, size_t hi, AttnParams &p, bool &split) -> pe_status {
         // C CTAs (pairs of q-tiles x kv-heads), W key tiles per CTA on average.
-        int64_t C = 0, tiles = 0, rows = 0, max_tiles = 0;
+        int64_t C = 0, tiles = 0, rows = 0, valid_rows = 0, max_tiles = 0;
         for (size_t i = lo; i < hi; ++i) {
             const AttnItem &it = order[i];
             const int64_t len = c->len[it.seq];
@@ -371,7 +433,8 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
                 tiles += ceil_div(len - it.n_q + q_last + 1, kBN) * hkv;
             }
             C += ceil_div(nqt, 2) * hkv;
-            rows += nqt * hkv * kBM;
+            rows += nqt * hkv * kBM;                               // workspace slots (whole tiles)
+            valid_rows += static_cast<int64_t>(it.n_q) * g * hkv;  // partial rows written and read
             max_tiles = std::max(max_tiles, ceil_div(len, kBN));
         }
         // Estimated time with s key splits: the CTAs run in ceil(C s / N) waves of
@@ -383,7 +446,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         auto cost = [&](int64_t sp) {
             const double waves = std::ceil(static_cast<double>(C * sp) / c->num_sms);
             double t = std::max(waves * (W / sp + 2.0), static_cast<double>(max_tiles) / sp + 2.0) * 1.5e-6;
-            if (sp > 1) t += static_cast<double>(rows * sp * row_bytes * 2) / 6.0e12 + 5e-6;
+            if (sp > 1) t += static_cast<double>(valid_rows * sp * row_bytes * 2) / 6.0e12 + 5e-6;
             return t;
         };
         int64_t best = 1;
@@ -543,6 +606,8 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
     cc->len.assign(c.max_seqs, 0);
     cc->appended.assign(c.max_seqs, 0);
     cc->alive.assign(c.max_seqs, 0);
+    cc->refs.assign(c.num_pages, 0);
+    cc->ckpt.resize(c.max_seqs);
     cc->pool_rows = pool_rows;
     if (cc->host_only) {
         *out = cc;
@@ -618,6 +683,7 @@ pe_status pe_seq_create(pe_cache *c, int32_t *seq_out)
             c->table[s].clear();
             c->len[s] = 0;
             c->appended[s] = 0;
+            c->ckpt[s].clear();
             *seq_out = s;
             return PE_OK;
         }
@@ -627,25 +693,112 @@ pe_status pe_seq_create(pe_cache *c, int32_t *seq_out)
 
 pe_status pe_seq_release(pe_cache *c, int32_t seq, void *stream)
 {
-    CropPlan pl{};
-    pe_status s = plan_crop(c, seq, 1, &pl);
+    std::vector<CropPlan> pl(1);
+    pe_status s = plan_crop(c, seq, 1, &pl[0]);
     if (s != PE_OK) return s;
-    apply_crop(c, pl, nullptr);
+    apply_crop(c, pl[0], nullptr);
     c->alive[seq] = 0;
-    return launch_crops(c, {pl}, static_cast<cudaStream_t>(stream));
+    c->ckpt[seq].clear();
+    return launch_crops(c, pl, static_cast<cudaStream_t>(stream));
+}
+
+pe_status pe_seq_fork(pe_cache *c, int32_t seq, int32_t *new_seq, void *stream)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if (!new_seq) return fail(PE_ERR_INVALID, "null new_seq");
+    int32_t ns = -1;
+    for (int32_t q = 0; q < c->cfg.max_seqs; ++q)
+        if (!c->alive[q]) { ns = q; break; }
+    if (ns < 0) return fail(PE_ERR_OOM, "no free sequence slot (max_seqs = %d)", c->cfg.max_seqs);
+    c->alive[ns] = 1;
+    c->table[ns] = c->table[seq];
+    for (int32_t pg : c->table[ns]) c->refs[pg] += 1;
+    c->len[ns] = c->len[seq];
+    c->appended[ns] = c->appended[seq];
+    c->ckpt[ns] = c->ckpt[seq];
+    *new_seq = ns;
+    if (!c->host_only) {
+        cudaError_t e = launch_table_copy(c->d_table, seq * c->cfg.max_pages_per_seq, ns * c->cfg.max_pages_per_seq,
+                                          static_cast<int32_t>(c->table[ns].size()), c->d_len, ns, c->len[ns],
+                                          static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "fork table copy launch");
+        c->launches++;
+    }
+    return PE_OK;
+}
+
+pe_status pe_checkpoint_add(pe_cache *c, int32_t seq, int64_t offset)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if (offset < 0 || offset > c->len[seq])
+        return fail(PE_ERR_RANGE, "checkpoint offset %lld outside [0, %lld]", static_cast<long long>(offset),
+                    static_cast<long long>(c->len[seq]));
+    std::vector<int64_t> &ck = c->ckpt[seq];
+    auto it = std::lower_bound(ck.begin(), ck.end(), offset);
+    if (it == ck.end() || *it != offset) ck.insert(it, offset);
+    return PE_OK;
+}
+
+pe_status pe_checkpoint_select(const pe_cache *c, int32_t seq, int64_t tau, int64_t *offset)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    if (tau < 1) return fail(PE_ERR_INVALID, "tau = %lld < 1", static_cast<long long>(tau));
+    const std::vector<int64_t> &ck = c->ckpt[seq];
+    auto it = std::lower_bound(ck.begin(), ck.end(), tau);  // first offset >= tau
+    if (it == ck.begin()) return fail(PE_ERR_RANGE, "no checkpoint before tau = %lld", static_cast<long long>(tau));
+    if (offset) *offset = *(it - 1);
+    return PE_OK;
+}
+
+pe_status pe_seq_checkpoints(const pe_cache *c, int32_t seq, int64_t *out, int32_t cap, int32_t *n)
+{
+    pe_status s = check_seq(c, seq);
+    if (s != PE_OK) return s;
+    const std::vector<int64_t> &ck = c->ckpt[seq];
+    if (n) *n = static_cast<int32_t>(ck.size());
+    if (out) {
+        if (cap < static_cast<int32_t>(ck.size())) return fail(PE_ERR_RANGE, "cap %d < %zu checkpoints", cap, ck.size());
+        std::copy(ck.begin(), ck.end(), out);
+    }
+    return PE_OK;
+}
+
+pe_status pe_restore(pe_cache *c, int32_t seq, int64_t tau, int64_t *offset, int32_t *freed_out, int32_t freed_cap,
+                     int32_t *n_freed, void *stream)
+{
+    int64_t b = 0;
+    pe_status s = pe_checkpoint_select(c, seq, tau, &b);
+    if (s != PE_OK) return s;
+    if (tau - 1 > c->len[seq])
+        return fail(PE_ERR_RANGE, "tau - 1 = %lld exceeds the sequence length %lld", static_cast<long long>(tau - 1),
+                    static_cast<long long>(c->len[seq]));
+    s = pe_crop(c, seq, b + 1, freed_out, freed_cap, n_freed, stream);
+    if (s == PE_OK && offset) *offset = b;
+    return s;
+}
+
+pe_status pe_page_refs(const pe_cache *c, int32_t *out, int32_t cap)
+{
+    if (!c || !out) return fail(PE_ERR_INVALID, "null argument");
+    if (cap < c->cfg.num_pages) return fail(PE_ERR_RANGE, "cap %d < %d pages", cap, c->cfg.num_pages);
+    std::copy(c->refs.begin(), c->refs.end(), out);
+    return PE_OK;
 }
 
 pe_status pe_crop(pe_cache *c, int32_t seq, int64_t tau, int32_t *freed_out, int32_t freed_cap, int32_t *n_freed,
                   void *stream)
 {
-    CropPlan pl{};
-    pe_status s = plan_crop(c, seq, tau, &pl);
+    std::vector<CropPlan> pl(1);
+    pe_status s = plan_crop(c, seq, tau, &pl[0]);
     if (s != PE_OK) return s;
-    const int32_t nf = pl.old_n - pl.keep;
+    const int32_t nf = pl[0].n_freed;
     if (freed_out && freed_cap < nf) return fail(PE_ERR_RANGE, "freed_cap %d < %d freed pages", freed_cap, nf);
-    apply_crop(c, pl, freed_out);
+    apply_crop(c, pl[0], freed_out);
     if (n_freed) *n_freed = nf;
-    return launch_crops(c, {pl}, static_cast<cudaStream_t>(stream));
+    return launch_crops(c, pl, static_cast<cudaStream_t>(stream));
 }
 
 pe_status pe_crop_batch(pe_cache *c, int32_t n, const int32_t *seqs, const int64_t *taus, void *stream)
@@ -660,7 +813,7 @@ pe_status pe_crop_batch(pe_cache *c, int32_t n, const int32_t *seqs, const int64
         if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice in the batch", seqs[i]);
         seen[seqs[i]] = 1;
     }
-    for (const CropPlan &pl : plans) apply_crop(c, pl, nullptr);
+    for (CropPlan &pl : plans) apply_crop(c, pl, nullptr);
     return launch_crops(c, plans, static_cast<cudaStream_t>(stream));
 }
 

@@ -44,12 +44,18 @@ struct AppendParams {
 };
 
 // ---------------------------------------------------------------- crop
+constexpr int kMaxCropFreed = 2048;  // freed page ids carried by one crop launch (debug poison)
+
 struct CropSeg {
     int32_t table_row;
     int32_t keep;          // pages kept
     int32_t old_n;         // pages before the crop
     int32_t seq;
     int64_t new_len;
+    int32_t freed0;        // debug poison: this sequence's pages whose last reference went,
+    int32_t n_freed;       //   as a range of CropParams::freed
+    int32_t tail_page;     // debug poison: last kept page when this sequence is its only holder, else -1
+    int32_t pad_;
 };
 
 struct CropParams {
@@ -59,6 +65,7 @@ struct CropParams {
     uint4 *v_pool;
     int32_t n, poison, L, hkv, ps, dvec, num_pages;
     CropSeg segs[kMaxCropSegs];
+    int32_t freed[kMaxCropFreed];
 };
 
 // ---------------------------------------------------------------- attention
@@ -93,6 +100,15 @@ struct AttnParams {
 // Launchers (defined in the .cu files).
 cudaError_t launch_append(const AppendParams &p, int64_t chunks, cudaStream_t st);
 cudaError_t launch_crop(const CropParams &p, cudaStream_t st);
+// Fork: copies n device page-table entries from row src_row to dst_row and sets
+// the new sequence's device length.
+cudaError_t launch_table_copy(int32_t *page_table, int32_t src_row, int32_t dst_row, int32_t n, int64_t *seq_len,
+                              int32_t dst_seq, int64_t len, cudaStream_t st);
+// Copy-on-write: copies slots [0, slots) of page src to page dst (every layer
+// and kv-head, K and V) and points the device table entry at dst.
+cudaError_t launch_cow_copy(uint4 *k_pool, uint4 *v_pool, int32_t src, int32_t dst, int32_t slots, int32_t L,
+                            int32_t hkv, int32_t ps, int32_t dvec, int32_t num_pages, int32_t *table_entry,
+                            cudaStream_t st);
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
                                const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);

@@ -80,10 +80,10 @@ cudaError_t launch_append(const AppendParams &p, int64_t chunks, cudaStream_t st
     return cudaGetLastError();
 }
 
-// One block per cropped sequence.  Debug poison first overwrites the freed
-// pages (every layer, head, slot, K and V) and the stale tail of the last kept
-// page, reading the page ids from the device table before this block
-// invalidates them; then the table entries [keep, old_n) become -1.
+// One block per cropped sequence.  Debug poison first overwrites the pages
+// whose last reference this crop dropped (every layer, head, slot, K and V) and
+// the stale tail of the last kept page when no other sequence holds it; then
+// the table entries [keep, old_n) of this sequence become -1.
 __global__ void __launch_bounds__(256) crop_kernel(const __grid_constant__ CropParams p)
 {
     const CropSeg &sg = p.segs[blockIdx.x];
@@ -92,8 +92,8 @@ __global__ void __launch_bounds__(256) crop_kernel(const __grid_constant__ CropP
         const uint4 poison = make_uint4(kPoisonPair, kPoisonPair, kPoisonPair, kPoisonPair);
         const int slot_chunks = p.dvec;                          // chunks per (page, head, slot)
         const int page_chunks = p.hkv * p.ps * slot_chunks;      // per (layer, page)
-        for (int e = sg.keep; e < sg.old_n; ++e) {
-            const int page = row[e];
+        for (int e = 0; e < sg.n_freed; ++e) {
+            const int page = p.freed[sg.freed0 + e];
             if (page < 0 || page >= p.num_pages) continue;
             for (int l = 0; l < p.L; ++l) {
                 const int64_t base = (static_cast<int64_t>(l) * p.num_pages + page) * page_chunks;
@@ -104,21 +104,18 @@ __global__ void __launch_bounds__(256) crop_kernel(const __grid_constant__ CropP
             }
         }
         const int tail = static_cast<int>(sg.new_len % p.ps);
-        if (tail != 0 && sg.keep > 0) {
-            const int page = row[sg.keep - 1];
-            if (page >= 0 && page < p.num_pages) {
-                const int per_head = (p.ps - tail) * slot_chunks;
-                for (int l = 0; l < p.L; ++l)
-                    for (int h = 0; h < p.hkv; ++h) {
-                        const int64_t base =
-                            (((static_cast<int64_t>(l) * p.num_pages + page) * p.hkv + h) * p.ps + tail) *
-                            slot_chunks;
-                        for (int i = threadIdx.x; i < per_head; i += blockDim.x) {
-                            p.k_pool[base + i] = poison;
-                            p.v_pool[base + i] = poison;
-                        }
+        const int page = sg.tail_page;
+        if (tail != 0 && page >= 0 && page < p.num_pages) {
+            const int per_head = (p.ps - tail) * slot_chunks;
+            for (int l = 0; l < p.L; ++l)
+                for (int h = 0; h < p.hkv; ++h) {
+                    const int64_t base =
+                        (((static_cast<int64_t>(l) * p.num_pages + page) * p.hkv + h) * p.ps + tail) * slot_chunks;
+                    for (int i = threadIdx.x; i < per_head; i += blockDim.x) {
+                        p.k_pool[base + i] = poison;
+                        p.v_pool[base + i] = poison;
                     }
-            }
+                }
         }
         __syncthreads();
     }
@@ -132,6 +129,44 @@ cudaError_t launch_crop(const CropParams &p, cudaStream_t st)
 {
     if (p.n <= 0) return cudaSuccess;
     crop_kernel<<<p.n, 256, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
+__global__ void __launch_bounds__(256) table_copy_kernel(int32_t *page_table, int32_t src_row, int32_t dst_row,
+                                                         int32_t n, int64_t *seq_len, int32_t dst_seq, int64_t len)
+{
+    for (int i = threadIdx.x; i < n; i += blockDim.x) page_table[dst_row + i] = page_table[src_row + i];
+    if (threadIdx.x == 0) seq_len[dst_seq] = len;
+}
+
+cudaError_t launch_table_copy(int32_t *page_table, int32_t src_row, int32_t dst_row, int32_t n, int64_t *seq_len,
+                              int32_t dst_seq, int64_t len, cudaStream_t st)
+{
+    table_copy_kernel<<<1, 256, 0, st>>>(page_table, src_row, dst_row, n, seq_len, dst_seq, len);
+    return cudaGetLastError();
+}
+
+// Grid: (layer x kv-head) blocks; each copies `slots` rows of d (16-byte chunks).
+__global__ void __launch_bounds__(256) cow_copy_kernel(uint4 *k_pool, uint4 *v_pool, int32_t src, int32_t dst,
+                                                       int32_t slots, int32_t hkv, int32_t ps, int32_t dvec,
+                                                       int32_t num_pages, int32_t *table_entry)
+{
+    const int l = blockIdx.x / hkv;
+    const int h = blockIdx.x % hkv;
+    const int64_t s_base = ((static_cast<int64_t>(l) * num_pages + src) * hkv + h) * ps * dvec;
+    const int64_t d_base = ((static_cast<int64_t>(l) * num_pages + dst) * hkv + h) * ps * dvec;
+    for (int i = threadIdx.x; i < slots * dvec; i += blockDim.x) {
+        k_pool[d_base + i] = k_pool[s_base + i];
+        v_pool[d_base + i] = v_pool[s_base + i];
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) *table_entry = dst;
+}
+
+cudaError_t launch_cow_copy(uint4 *k_pool, uint4 *v_pool, int32_t src, int32_t dst, int32_t slots, int32_t L,
+                            int32_t hkv, int32_t ps, int32_t dvec, int32_t num_pages, int32_t *table_entry,
+                            cudaStream_t st)
+{
+    cow_copy_kernel<<<L * hkv, 256, 0, st>>>(k_pool, v_pool, src, dst, slots, hkv, ps, dvec, num_pages, table_entry);
     return cudaGetLastError();
 }
 

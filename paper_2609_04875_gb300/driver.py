@@ -32,7 +32,8 @@ class ReplayDriver:
         self.w = w
         self.device = torch.device(device)
         L, hq, hkv, d = w.num_layers, w.num_q_heads, w.num_kv_heads, w.head_dim
-        self.cache = PagedKVCache(L, hkv, d, w.page_size, w.num_pages, max_seqs=len(w.agents),
+        # twice the agents' sequence slots: room for one branch (fork) of every agent
+        self.cache = PagedKVCache(L, hkv, d, w.page_size, w.num_pages, max_seqs=2 * len(w.agents),
                                   max_pages_per_seq=w.max_pages_per_seq, init_free_order=w.init_free_order(),
                                   **(cache_kwargs or {}))
         self.seqs = [self.cache.seq_create() for _ in w.agents]
@@ -40,6 +41,7 @@ class ReplayDriver:
         S = [a.S for a in w.agents]
         self.cu = [0] + list(np.cumsum(S).astype(int))
         n = self.cu[-1]
+        # (twice the agents' sequence slots: room for a branch of every agent)
         # sanitized suffix inputs, packed over agents: K'/V' [L][sum S][Hkv][d], Q' [L][sum S][Hq][d]
         self.Kc = torch.empty((L, n, hkv, d), dtype=torch.bfloat16, device=self.device)
         self.Vc = torch.empty_like(self.Kc)

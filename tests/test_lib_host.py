@@ -181,3 +181,103 @@ def test_error_codes():
     with pytest.raises(binding.PEError) as e:
         pe.PagedKVCache(1, 1, 64, 16, 4, 2, 4, init_free_order=[0, 1, 1, 2], host_only=True)
     assert e.value.kind == "invalid"
+
+
+def test_golden_fork_trace():
+    """The hand-derived fork / copy-on-write / checkpoint trace on libpe
+    (ps = 4 in the trace, 8 here: token counts, taus and offsets doubled)."""
+    trace = pins.load_fork_trace()
+    cfg = trace["config"]
+    c = _mk(cfg)
+    f = 8 // cfg["page_size"]
+    for idx, st in enumerate(trace["steps"]):
+        op, seq = st["op"], st.get("seq")
+        try:
+            if op == "create":
+                assert c.seq_create() == st["expect_seq"]
+                continue
+            if op == "append":
+                c.append_kv(seq, n_tokens=st["n"] * f)
+            elif op == "checkpoint":
+                for b in st["offsets"]:
+                    c.checkpoint_add(seq, b * f)
+                continue
+            elif op == "fork":
+                assert c.seq_fork(seq) == st["expect_seq"], f"step {idx}"
+            elif op == "crop":
+                assert c.crop(seq, (st["tau"] - 1) * f + 1) == st["expect_freed"], f"step {idx}"
+            elif op == "restore":
+                b, freed = c.restore(seq, (st["tau"] - 1) * f + 1)
+                assert (b, freed) == (st["expect_offset"] * f, st["expect_freed"]), f"step {idx}"
+            elif op == "release":
+                c.seq_release(seq)
+                assert c.free_list() == st["expect_free"], f"step {idx}"
+                continue
+        except binding.PEError as e:
+            assert st.get("expect_error") == e.kind, f"step {idx}: {e}"
+            continue
+        assert "expect_error" not in st, f"step {idx}"
+        ex = st.get("expect", {})
+        s = ex.get("seq", seq)
+        if "table" in ex:
+            assert c.page_table(s) == ex["table"], f"step {idx}: {c.page_table(s)}"
+        if "len" in ex:
+            assert c.seq_info(s)[0] == ex["len"] * f, f"step {idx}"
+        if "free" in ex:
+            assert c.free_list() == ex["free"], f"step {idx}"
+        refs = c.page_refs()
+        for pg, r in ex.get("refs", {}).items():
+            assert refs[int(pg)] == r, f"step {idx}: refs[{pg}]"
+        if "checkpoints" in ex:
+            assert c.checkpoints(s) == [b * f for b in ex["checkpoints"]], f"step {idx}"
+
+
+@pytest.mark.parametrize("ps", [8, 16])
+def test_random_fork_ops_match_oracle(ps):
+    num_pages, max_pages, max_seqs = 64, 30, 6
+    order = synth.page_permutation(77 + ps, num_pages)
+    lib = pe.PagedKVCache(1, 1, 64, ps, num_pages, max_seqs, max_pages, init_free_order=order, host_only=True)
+    orc = oracle.OracleKVCache(1, 1, 64, ps, num_pages, max_seqs, max_pages, init_free_order=order,
+                               store_values=False)
+    assert lib.seq_create() == orc.seq_create()
+    g = synth.rng(31, ps)
+    for step in range(1500):
+        live = sorted(orc.table)
+        s = live[int(g.integers(0, len(live)))]
+        r = g.random()
+
+        def both(f_orc, f_lib):
+            try:
+                want = f_orc()
+            except oracle.OracleError as e:
+                with pytest.raises(binding.PEError) as pe_err:
+                    f_lib()
+                assert pe_err.value.kind == e.kind, f"step {step}"
+                return
+            got = f_lib()
+            if got is not None:
+                assert got == want, f"step {step}"
+
+        n = orc.length[s]
+        if r < 0.15:
+            both(lambda: orc.seq_fork(s), lambda: lib.seq_fork(s))
+        elif r < 0.35:
+            tau = int(g.integers(0, n + 3))
+            both(lambda: orc.crop(s, tau), lambda: lib.crop(s, tau))
+        elif r < 0.45:
+            b = int(g.integers(-1, n + 2))
+            both(lambda: orc.checkpoint_add(s, b), lambda: lib.checkpoint_add(s, b))
+        elif r < 0.55:
+            tau = int(g.integers(0, n + 3))
+            both(lambda: orc.restore(s, tau), lambda: lib.restore(s, tau))
+        elif r < 0.62 and len(live) > 1:
+            both(lambda: orc.seq_release(s), lambda: lib.seq_release(s))
+        else:
+            k = int(g.integers(0, 3 * ps))
+            both(lambda: orc.append(s, n_tokens=k), lambda: lib.append_kv(s, n_tokens=k))
+        assert lib.free_list() == orc.free_list(), f"step {step}"
+        assert lib.page_refs() == list(orc.refs), f"step {step}"
+        for q in orc.table:
+            assert lib.page_table(q) == orc.page_table(q), f"step {step}"
+            assert lib.seq_info(q) == orc.seq_info(q), f"step {step}"
+            assert lib.checkpoints(q) == orc.checkpoints[q], f"step {step}"
