@@ -66,3 +66,50 @@ def _pins_fail(mod):
 def test_pins_catch_planted_mistake(tmp_path, name, fname, old, new):
     mod = _load_mutant(tmp_path, name, fname, old, new)
     assert _pins_fail(mod) >= 1, f"no pin caught mutant {name}"
+
+
+PROV_MUTANTS = [
+    ("edges_reversed", "for p in rec[\"parents\"]:\n                ch[p].append(a)",
+     "for p in rec[\"parents\"]:\n                ch[a].append(p)"),
+    ("closure_without_source", "seen = {s}\n        frontier = [s]", "seen = set()\n        frontier = [s]"),
+    ("tau_zero_based", "return min(self.art[a][\"begin\"] for a in self.taint_closure(s)) + 1",
+     "return min(self.art[a][\"begin\"] for a in self.taint_closure(s))"),
+    ("source_not_root", "return min(roots, key=lambda a: (self.art[a][\"begin\"], a))",
+     "return max(carriers, key=lambda a: (self.art[a][\"begin\"], a))"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", PROV_MUTANTS, ids=[m[0] for m in PROV_MUTANTS])
+def test_provenance_pins_catch_planted_mistake(tmp_path, name, old, new):
+    import test_oracle_provenance as tp
+    src = open(os.path.join(ORACLE_DIR, "provenance.py")).read()
+    assert old in src, name
+    path = tmp_path / f"prov_mut_{name}.py"
+    path.write_text(src.replace(old, new))
+    spec = importlib.util.spec_from_file_location(f"prov_mut_{name}", path)
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    caught = 0
+    for chk in (lambda: _prov_episode(tp, mod), lambda: _prov_random(tp, mod)):
+        try:
+            chk()
+        except Exception:
+            caught += 1
+    assert caught >= 1, f"no pin caught provenance mutant {name}"
+
+
+def _prov_episode(tp, mod):
+    ep = tp.load_episode()
+    g = tp.build(mod.OracleProvenance(), ep["artifacts"])
+    q = ep["query"]
+    s = g.locate_source(q["z"])
+    assert s == q["source"] and g.taint_closure(s) == q["closure"] and g.first_entry(s) == q["tau"]
+
+
+def _prov_random(tp, mod):
+    for seed in range(6):
+        arts = tp.random_dag(seed, 60)
+        g = tp.build(mod.OracleProvenance(), arts)
+        s = g.locate_source(9)
+        assert g.taint_closure(s) == tp.brute_closure(arts, s)
+        assert not any(9 in g.art[p]["sources"] for p in g.art[s]["parents"])
