@@ -320,6 +320,19 @@ def run_pe(args, rank, world, local_rank):
         rel_us.append((h2 - h1) * 1e6 / len(forks))
     torch.cuda.synchronize(dev)
 
+    # ---- provenance queries on a 100k-artifact session graph (host)
+    from paper_2609_04875_gb300 import ProvenanceGraph
+    arts = synth.provenance_dag(w.seed, 100000)
+    pg = ProvenanceGraph()
+    for a in arts:
+        pg.add(a["id"], a["type"], a["parents"], a["sources"], a["begin"], a["end"], a["turn"], a["committed"])
+    h0 = time.perf_counter()
+    src = pg.locate_source(9)
+    closure, _ = pg.taint_closure(src)
+    tau_q = pg.first_entry(src)
+    prov_us = (time.perf_counter() - h0) * 1e6
+    pg.close()
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -357,6 +370,8 @@ def run_pe(args, rank, world, local_rank):
                     "device_median": statistics.median(crop_dev_us), "agents": len(w.agents)},
         "fork_us": {"host_per_fork_median": statistics.median(fork_us),
                     "host_per_release_median": statistics.median(rel_us)},
+        "provenance_query_us": {"artifacts": len(arts), "closure": len(closure), "tau": tau_q,
+                                "locate_closure_first_entry": prov_us},
         "recomputed_tokens": tokens_per_step,
         "session_tokens": sum(a.T for a in w.agents),
         "gpu_launches": launches,

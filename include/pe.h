@@ -223,6 +223,33 @@ pe_status pe_last_attn_plan(const pe_cache *cache, int32_t *split, int32_t *n_sp
  * attention, combine); lets a caller count its device work. */
 pe_status pe_kernel_launches(const pe_cache *cache, int64_t *count);
 
+/* ---- Provenance graph (Sec. 3.4(a); Alg. 1 lines 1-3), host only ----------
+ * The runtime records artifacts in execution order: id (unique), type,
+ * parents (ids already added; edges run parent -> child), the source ids the
+ * artifact carries (e.g. a forget target z and the artifacts derived while z
+ * was resident), its token span [token_begin, token_end) in the session, its
+ * turn, and whether it committed an external side effect.
+ *   pe_prov_locate_source: LocateSource(z), the artifact through which z
+ *     entered: a carrier of z none of whose parents carries z (earliest
+ *     token_begin, then smallest id); RANGE when nothing carries z.
+ *   pe_prov_taint_closure: TaintClosure(s) = I(z), the artifacts reachable
+ *     from s (s included), ids ascending into out[cap]; *n their number and
+ *     *n_committed how many committed side effects (Theorem 1's assumption A3
+ *     needs 0 for an exact replay).  RANGE when s is unknown or cap < *n.
+ *   pe_prov_first_entry: FirstEntry(s) = tau, the 1-based position of the
+ *     closure's first token; pe_crop(seq, tau) then keeps the clean prefix.
+ * Errors of pe_prov_add: INVALID (duplicate id, unknown parent, bad span). */
+typedef struct pe_prov pe_prov;
+pe_status pe_prov_create(pe_prov **out);
+pe_status pe_prov_destroy(pe_prov *graph);
+pe_status pe_prov_add(pe_prov *graph, int64_t id, int32_t type, const int64_t *parents, int32_t n_parents,
+                      const int64_t *source_ids, int32_t n_sources, int64_t token_begin, int64_t token_end,
+                      int32_t turn, int32_t committed);
+pe_status pe_prov_locate_source(const pe_prov *graph, int64_t z, int64_t *source);
+pe_status pe_prov_taint_closure(const pe_prov *graph, int64_t source, int64_t *out, int32_t cap, int32_t *n,
+                                int32_t *n_committed);
+pe_status pe_prov_first_entry(const pe_prov *graph, int64_t source, int64_t *tau);
+
 /* Thread-local description of the last error on this thread ("" if none). */
 const char *pe_last_error(void);
 /* Library version string. */

@@ -29,7 +29,8 @@ EXPORTED = [
     "pe_seq_page_table", "pe_free_list", "pe_seq_device_page_table", "pe_cache_pools", "pe_set_option",
     "pe_device_status", "pe_kernel_launches", "pe_replay_attn_static_scratch", "pe_selftest_bounded_wait",
     "pe_last_attn_plan", "pe_seq_fork", "pe_checkpoint_add", "pe_checkpoint_select", "pe_restore",
-    "pe_seq_checkpoints", "pe_page_refs", "pe_last_error", "pe_version",
+    "pe_seq_checkpoints", "pe_page_refs", "pe_prov_create", "pe_prov_destroy", "pe_prov_add",
+    "pe_prov_locate_source", "pe_prov_taint_closure", "pe_prov_first_entry", "pe_last_error", "pe_version",
 ]
 
 
@@ -83,6 +84,12 @@ _sigs = {
     "pe_restore": [_P, _I32, _I64, _I64P, _I32P, _I32, _I32P, _P],
     "pe_seq_checkpoints": [_P, _I32, _I64P, _I32, _I32P],
     "pe_page_refs": [_P, _I32P, _I32],
+    "pe_prov_create": [ctypes.POINTER(_P)],
+    "pe_prov_destroy": [_P],
+    "pe_prov_add": [_P, _I64, _I32, _I64P, _I32, _I64P, _I32, _I64, _I64, _I32, _I32],
+    "pe_prov_locate_source": [_P, _I64, _I64P],
+    "pe_prov_taint_closure": [_P, _I64, _I64P, _I32, _I32P, _I32P],
+    "pe_prov_first_entry": [_P, _I64, _I64P],
     "pe_replay_attn_static_scratch": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
 }
 for _name, _args in _sigs.items():
@@ -373,3 +380,48 @@ class PagedKVCache:
         if rc not in (PE_OK, -6):
             _check(rc)
         return code.value
+
+
+class ProvenanceGraph:
+    """Artifact DAG of one session (Sec. 3.4(a)) and the queries of Alg. 1,
+    lines 1-3: locate_source(z), taint_closure(s), first_entry(s) -> tau."""
+
+    def __init__(self):
+        h = ctypes.c_void_p()
+        _check(_lib.pe_prov_create(ctypes.byref(h)))
+        self._h = h
+
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            _check(_lib.pe_prov_destroy(self._h))
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def add(self, aid, type_=0, parents=(), source_ids=(), token_begin=0, token_end=0, turn=0, committed=False):
+        par = _i64_array(parents)
+        src = _i64_array(source_ids)
+        _check(_lib.pe_prov_add(self._h, int(aid), int(type_), par, len(parents), src, len(source_ids),
+                                int(token_begin), int(token_end), int(turn), 1 if committed else 0))
+
+    def locate_source(self, z) -> int:
+        out = ctypes.c_int64()
+        _check(_lib.pe_prov_locate_source(self._h, int(z), ctypes.byref(out)))
+        return out.value
+
+    def taint_closure(self, s):
+        """(ids ascending, number that committed a side effect)"""
+        n, nc = ctypes.c_int32(), ctypes.c_int32()
+        _check(_lib.pe_prov_taint_closure(self._h, int(s), None, 0, ctypes.byref(n), ctypes.byref(nc)))
+        buf = (ctypes.c_int64 * max(1, n.value))()
+        _check(_lib.pe_prov_taint_closure(self._h, int(s), buf, n.value, ctypes.byref(n), ctypes.byref(nc)))
+        return list(buf[: n.value]), nc.value
+
+    def first_entry(self, s) -> int:
+        out = ctypes.c_int64()
+        _check(_lib.pe_prov_first_entry(self._h, int(s), ctypes.byref(out)))
+        return out.value

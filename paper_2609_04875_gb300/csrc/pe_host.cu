@@ -64,6 +64,12 @@ EncodeTiledFn encode_fn()
 
 }  // namespace
 
+int32_t pe::report_error(int32_t code, const char *msg)
+{
+    g_err = msg;
+    return code;
+}
+
 struct pe_cache {
     pe_cache_config cfg{};
     bool host_only = false;

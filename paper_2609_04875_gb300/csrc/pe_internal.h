@@ -97,6 +97,9 @@ struct AttnParams {
     AttnSeq seqs[kMaxSegs];
 };
 
+// Records `msg` as this thread's last error (pe_last_error) and returns code.
+int32_t report_error(int32_t code, const char *msg);
+
 // Launchers (defined in the .cu files).
 cudaError_t launch_append(const AppendParams &p, int64_t chunks, cudaStream_t st);
 cudaError_t launch_crop(const CropParams &p, cudaStream_t st);

@@ -271,3 +271,25 @@ def sample_rows(seed: int, n_q: int, n_random: int, tile_rows: int = 128, index:
     if n_q > 0 and n_random > 0:
         rows.update(int(x) for x in g.integers(0, n_q, size=n_random))
     return np.array(sorted(r for r in rows if 0 <= r < n_q), dtype=np.int64)
+
+
+def provenance_dag(seed: int, n: int, z: int = 9):
+    """A session's artifacts in execution order: random parents (up to 3 earlier
+    artifacts), token spans of 1-39 tokens laid end to end, one artifact where
+    the target z enters, and z inherited by each descendant of a carrier with
+    probability 0.7; about 10% of artifacts committed a side effect."""
+    g = rng(seed, 0)
+    arts, begin, carriers = [], 0, set()
+    entry = int(g.integers(0, n))
+    for i in range(n):
+        k = int(g.integers(0, min(i, 3) + 1))
+        parents = sorted({int(x) for x in g.integers(0, i, size=k)}) if i > 0 and k > 0 else []
+        length = int(g.integers(1, 40))
+        src = []
+        if i == entry or (any(p in carriers for p in parents) and g.random() < 0.7):
+            src = [z]
+            carriers.add(i)
+        arts.append(dict(id=i, type=0, parents=parents, sources=src, begin=begin, end=begin + length, turn=i,
+                         committed=int(g.random() < 0.1)))
+        begin += length
+    return arts

@@ -24,24 +24,7 @@ def build(g, arts):
 
 
 def random_dag(seed, n, z=9):
-    """Artifacts in execution order with random parents, token spans and a
-    target z entering at a random artifact and propagating to a random share
-    of its descendants."""
-    g = synth.rng(seed, 0)
-    arts, begin, carriers = [], 0, set()
-    entry = int(g.integers(0, n))
-    for i in range(n):
-        k = int(g.integers(0, min(i, 3) + 1))
-        parents = sorted({int(x) for x in g.integers(0, i, size=k)}) if i > 0 and k > 0 else []
-        length = int(g.integers(1, 40))
-        src = []
-        if i == entry or (any(p in carriers for p in parents) and g.random() < 0.7):
-            src = [z]
-            carriers.add(i)
-        arts.append(dict(id=i, type=0, parents=parents, sources=src, begin=begin, end=begin + length, turn=i,
-                         committed=int(g.random() < 0.1)))
-        begin += length
-    return arts
+    return synth.provenance_dag(seed, n, z)
 
 
 def brute_closure(arts, s):
