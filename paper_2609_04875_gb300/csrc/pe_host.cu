@@ -548,12 +548,14 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     return PE_OK;
 }
 
-pe_status check_attn_args(const pe_cache *c, int32_t layer, const void *Q, const void *out, int32_t hq, float scale)
+// Pointers are only checked when the call has queries (an empty tensor may be null).
+pe_status check_attn_args(const pe_cache *c, int32_t layer, const void *Q, const void *out, int32_t hq, float scale,
+                          bool has_rows = true)
 {
     if (c->host_only) return fail(PE_ERR_UNSUPPORTED, "attention on a host-only cache");
     if (layer < 0 || layer >= c->cfg.num_layers) return fail(PE_ERR_RANGE, "layer %d out of range", layer);
-    if (!Q || !out) return fail(PE_ERR_INVALID, "null Q or out");
-    if (!aligned16(Q) || !aligned16(out)) return fail(PE_ERR_INVALID, "Q and out must be 16-byte aligned");
+    if (has_rows && (!Q || !out)) return fail(PE_ERR_INVALID, "null Q or out");
+    if (has_rows && (!aligned16(Q) || !aligned16(out))) return fail(PE_ERR_INVALID, "Q and out must be 16-byte aligned");
     if (hq <= 0 || hq % c->cfg.num_kv_heads != 0)
         return fail(PE_ERR_INVALID, "num_q_heads %d is not a multiple of num_kv_heads %d", hq, c->cfg.num_kv_heads);
     const int g = hq / c->cfg.num_kv_heads;
@@ -872,7 +874,7 @@ pe_status pe_replay_attn(pe_cache *c, int32_t seq, int32_t layer, const void *Q,
 {
     pe_status s = check_seq(c, seq);
     if (s != PE_OK) return s;
-    if ((s = check_attn_args(c, layer, Q, out, num_q_heads, softmax_scale)) != PE_OK) return s;
+    if ((s = check_attn_args(c, layer, Q, out, num_q_heads, softmax_scale, n_q > 0)) != PE_OK) return s;
     if (n_q < 0) return fail(PE_ERR_INVALID, "negative n_q");
     if (n_q > c->len[seq])
         return fail(PE_ERR_RANGE, "n_q = %d exceeds the sequence length %lld", n_q, static_cast<long long>(c->len[seq]));
@@ -887,7 +889,7 @@ pe_status pe_replay_attn_batch(pe_cache *c, int32_t n, const int32_t *seqs, int3
     if (!c) return fail(PE_ERR_INVALID, "null cache");
     if (n < 0 || (n > 0 && (!seqs || !cu_q))) return fail(PE_ERR_INVALID, "bad batch arguments");
     if (n == 0) return PE_OK;
-    pe_status s = check_attn_args(c, layer, Q_packed, out, num_q_heads, softmax_scale);
+    pe_status s = check_attn_args(c, layer, Q_packed, out, num_q_heads, softmax_scale, cu_q[n] > 0);
     if (s != PE_OK) return s;
     if (cu_q[0] != 0) return fail(PE_ERR_INVALID, "cu_q[0] must be 0");
     std::vector<AttnItem> items(n);
