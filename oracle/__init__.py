@@ -12,6 +12,10 @@ Contents
     over rows; see attention.c).
   * ``replay_attention`` -- gathers a sequence through the oracle cache's page
     table and runs ``causal_attention`` on its last n_q positions.
+  * ``schedule`` -- which suffix positions a replay re-prefills and which it
+    re-decodes (selective replay vs full reset with a prefix cache), the
+    lockstep rounds over many agents, and ``execute_rounds`` on the oracle cache.
+  * ``provenance.OracleProvenance`` -- the artifact graph queries.
 """
 from __future__ import annotations
 
@@ -23,6 +27,7 @@ import threading
 import numpy as np
 
 from .kvcache import OracleError, OracleKVCache  # noqa: F401
+from . import schedule  # noqa: F401
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "attention.c")
@@ -100,3 +105,10 @@ def replay_attention(cache: OracleKVCache, seq: int, layer: int, q_bits, scale, 
     if q_bits.shape[0] > n_keys:
         raise OracleError("range", "more queries than cached tokens")
     return causal_attention(q_bits, k, v, scale, rows=rows, nthreads=nthreads)
+
+
+def execute_rounds(cache: OracleKVCache, seqs, take, k_bits, v_bits, q_bits, cu_tok, scale, nthreads=0):
+    """``schedule.execute_rounds`` with this package's replay attention."""
+    def attend(c, seq, layer, q, sc):
+        return replay_attention(c, seq, layer, q, sc, nthreads=nthreads)
+    return schedule.execute_rounds(cache, seqs, take, k_bits, v_bits, q_bits, cu_tok, scale, attend)

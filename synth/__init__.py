@@ -29,6 +29,14 @@ STREAM_Q_CF = 4          # Q' of the counterfactual suffix
 STREAM_Q_PREFIX = 5      # Q of the prefix positions (full-reset comparator)
 STREAM_LENGTHS = 6       # per-agent T and tau/T (agent batch)
 STREAM_SAMPLE = 7        # query rows sampled for large-size checks
+STREAM_TURNS = 8         # per-agent turn lengths of the suffix (turn-structured workload)
+STREAM_LABELS = 9        # which model turns are independent of the target
+
+# Turn kinds of a turn-structured suffix (labels of the synthetic session; the
+# replay policy that reads them lives in the library and in the oracle).
+TURN_INPUT = 0           # user message, tool observation or loaded document
+TURN_MODEL_INDEP = 1     # model turn causally independent of the target
+TURN_MODEL_DEP = 2       # model turn that depends on the target
 
 
 def rng(seed: int, stream: int, index: int = 0) -> np.random.Generator:
@@ -94,6 +102,7 @@ class Agent:
     T: int            # session length (tokens) before the forget request
     tau: int          # 1-based position of the first tainted token
     index: int        # agent index inside the workload (stream index)
+    turns: tuple = ()  # optional suffix turns ((n_tokens, kind), ...) summing to S
 
     @property
     def P(self) -> int:
@@ -222,6 +231,39 @@ def long_suffix(n_agents: int = 4, prefix: int = 4096, suffix: int = 16384) -> W
     return _finish(w)
 
 
+INDEP_MODEL_TURNS = 4    # model turns in the suffix; the last (the answer) always depends on z
+
+
+def indep_split(indep: float = 1.0, n_agents: int = 16, seed: int = BASE_SEED + 7) -> Workload:
+    """16 agents, 1 layer, GQA 32/8, d=128, ps=16, N(0,1)/sqrt(128); turn-structured suffixes.
+
+    Each agent keeps a clean prefix P ~ U{1024..4096}.  Its suffix starts with
+    the (sanitized) acquisition input and alternates model and input turns:
+    input, model, input, model, input, model, input, model (the final answer).
+    Inputs are U{32..256} tokens, model turns U{64..192}.  Of the three model
+    turns before the answer, round(3 * indep) are independent of the target,
+    chosen by a seeded per-agent order, so the independent sets grow with
+    indep and the lengths do not change."""
+    w = Workload(f"indep_split_{indep:g}", seed, 1, 32, 8, 128, 16, 1.0 / math.sqrt(128))
+    g = rng(seed, STREAM_LENGTHS)
+    n_indep = int(round((INDEP_MODEL_TURNS - 1) * float(indep)))
+    if not 0 <= n_indep <= INDEP_MODEL_TURNS - 1:
+        raise ValueError("indep must lie in [0, 1]")
+    for i in range(n_agents):
+        P = int(g.integers(1024, 4096, endpoint=True))
+        gt = rng(seed, STREAM_TURNS, i)
+        order = rng(seed, STREAM_LABELS, i).permutation(INDEP_MODEL_TURNS - 1)
+        indep_turns = set(int(x) for x in order[:n_indep])
+        turns = []
+        for m in range(INDEP_MODEL_TURNS):
+            turns.append((int(gt.integers(32, 256, endpoint=True)), TURN_INPUT))
+            kind = TURN_MODEL_INDEP if m in indep_turns else TURN_MODEL_DEP
+            turns.append((int(gt.integers(64, 192, endpoint=True)), kind))
+        S = sum(n for n, _ in turns)
+        w.agents.append(Agent(T=P + S, tau=P + 1, index=i, turns=tuple(turns)))
+    return _finish(w)
+
+
 def replica(w: Workload, r: int) -> Workload:
     """The same workload shape drawn from replica r's own seeds (one replica per
     GPU under weak scaling): the base seed moves by 1000 * r.  The agent batch
@@ -231,6 +273,8 @@ def replica(w: Workload, r: int) -> Workload:
         return agent_batch(len(w.agents), seed=seed)
     if w.name == "decode_batch":
         return decode_batch(len(w.agents), seed=seed)
+    if w.name.startswith("indep_split_"):
+        return indep_split(float(w.name[len("indep_split_"):]), len(w.agents), seed=seed)
     import copy
     w2 = copy.deepcopy(w)
     w2.seed = seed
@@ -257,6 +301,7 @@ WORKLOADS = {
     "decode_batch": decode_batch,
     "short_suffix": short_suffix,
     "long_suffix": long_suffix,
+    "indep_split": indep_split,
 }
 
 

@@ -113,3 +113,32 @@ def _prov_random(tp, mod):
         s = g.locate_source(9)
         assert g.taint_closure(s) == tp.brute_closure(arts, s)
         assert not any(9 in g.art[p]["sources"] for p in g.art[s]["parents"])
+
+
+SCHED_MUTANTS = [
+    ("independent_turns_decoded", "_KNOWN = {SELECTIVE: (0, 1), PREFIX_CACHE: (0,)}",
+     "_KNOWN = {SELECTIVE: (0,), PREFIX_CACHE: (0,)}"),
+    ("trailing_run_dropped", "    if run > 0:\n        units.append(run)\n    return units", "    return units"),
+    ("decode_turn_one_pass", "units.extend([1] * n)", "units.append(n)"),
+    ("known_turns_not_merged",
+     "            run += n                      # known tokens extend the current prefill run\n",
+     "            if run > 0:\n                units.append(run)\n            run = n\n"),
+    ("values_from_keys", "cache.append(seqs[i], k_bits[:, lo:hi], v_bits[:, lo:hi])",
+     "cache.append(seqs[i], k_bits[:, lo:hi], k_bits[:, lo:hi])"),
+    ("progress_ignored", "lo = int(cu_tok[i]) + done[i]", "lo = int(cu_tok[i])"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", SCHED_MUTANTS, ids=[m[0] for m in SCHED_MUTANTS])
+def test_schedule_pins_catch_planted_mistake(tmp_path, name, old, new):
+    import test_oracle_schedule as ts
+    mod = _load_mutant(tmp_path, name, "schedule.py", old, new)
+    caught = 0
+    for chk in (lambda: ts.pin_golden(mod.schedule), lambda: ts.pin_bruteforce_and_count(mod.schedule),
+                lambda: ts.pin_degenerate(mod.schedule), lambda: ts.pin_workload_monotone(mod.schedule),
+                lambda: ts.pin_execution(mod, seeds=range(3))):
+        try:
+            chk()
+        except Exception:
+            caught += 1
+    assert caught >= 1, f"no pin caught schedule mutant {name}"
