@@ -158,6 +158,50 @@ pe_status pe_replay_attn_batch(pe_cache *cache, int32_t n, const int32_t *seqs, 
                                const void *Q_packed, const int32_t *cu_q, void *out, int32_t num_q_heads,
                                float softmax_scale, void *stream);
 
+/* ---- Replay with the indep split (Sec. 4.5, the T - tau + 1 paragraph;
+ * Sec. 4.1 methods B7 and B5').  Post-target turns whose content is the same
+ * in the counterfactual world are re-prefilled, many positions per pass;
+ * turns that depend on the target are re-decoded, one position per pass.
+ * Selective replay (B7) counts model turns independent of the target as
+ * known; full reset with a prefix cache (B5') re-decodes every model turn of
+ * the suffix.  Both recompute the same T - tau + 1 positions (Corollary 1) and
+ * coincide when no model turn is independent. */
+enum { PE_TURN_INPUT = 0, PE_TURN_MODEL_INDEP = 1, PE_TURN_MODEL_DEP = 2 };
+enum { PE_POLICY_SELECTIVE = 0, PE_POLICY_PREFIX_CACHE = 1 };
+
+/* Plans the passes of n agents' suffix replays (host only, no cache).
+ * Agent i's suffix is turns [cu_turns[i], cu_turns[i+1]) of turn_len /
+ * turn_kind (host arrays; cu_turns host [n+1], from 0, non-decreasing).
+ * A unit is a maximal run of consecutive known positions (one prefill pass)
+ * or one position to decode; empty turns contribute nothing.  Agents advance
+ * in lockstep rounds: round r runs every agent's r-th unit.
+ * take (host int32 [n_rounds][n], row-major, nullable when take_cap == 0)
+ * receives the positions agent i appends and attends in round r (0 = idle);
+ * *n_rounds (required) the number of rounds; *decode_tokens (nullable) the
+ * positions decoded over all agents.  Call with take = NULL, take_cap = 0 to
+ * learn the size.
+ * Errors: INVALID (bad arrays, kind or policy, negative length, an agent's
+ * suffix above INT32_MAX), RANGE (n_rounds * n > take_cap; *n_rounds is set). */
+pe_status pe_replay_schedule(int32_t n, const int32_t *cu_turns, const int32_t *turn_len, const int32_t *turn_kind,
+                             int32_t policy, int32_t *take, int64_t take_cap, int32_t *n_rounds,
+                             int64_t *decode_tokens);
+
+/* Runs the rounds of a replay on the cache: in round r, every agent i with
+ * take[r*n + i] > 0 appends its next take[r*n + i] positions (K/V of all
+ * layers, as pe_append_kv_batch), then for each layer attends those positions'
+ * queries (as pe_replay_attn_batch).  Agent i's positions are rows
+ * [cu_tok[i], cu_tok[i+1]) of K, V (device bf16 [L][N][Hkv][d]) and of Q, out
+ * (device bf16 [L][N][Hq][d]), N = cu_tok[n]; cu_tok host [n+1], from 0.
+ * The rounds must cover each agent's rows exactly (sum over r of take = its
+ * row count).  Every argument, the pages all rounds need (checked up front,
+ * including copy-on-write) and the page-table capacity are checked before any
+ * state changes; a CUDA error (CUDA) may leave the earlier rounds applied.
+ * On a host-only cache only the bookkeeping runs (Q, out unused).
+ * Errors: INVALID, RANGE, OOM, UNSUPPORTED, CUDA. */
+pe_status pe_replay_rounds(pe_cache *cache, int32_t n, const int32_t *seqs, int32_t n_rounds, const int32_t *take,
+                           const int32_t *cu_tok, const void *K, const void *V, const void *Q, void *out,
+                           int32_t num_q_heads, float softmax_scale, void *stream);
+
 /* Variant of pe_replay_attn for callers that cannot allocate device memory at
  * the time they run attention: code inside a stream host callback or a
  * latency-critical serving loop where cudaMalloc (which may synchronise the

@@ -5,6 +5,6 @@ replayed suffix K/V and causal replay attention over the cropped cache -- is
 the C-ABI library libpe.so (include/pe.h), built from the CUDA sources in
 csrc/.  This package only binds it.
 """
-from .binding import PagedKVCache, PEError, ProvenanceGraph, version  # noqa: F401
+from .binding import PagedKVCache, PEError, ProvenanceGraph, replay_schedule, version  # noqa: F401
 
-__all__ = ["PagedKVCache", "PEError", "ProvenanceGraph", "version"]
+__all__ = ["PagedKVCache", "PEError", "ProvenanceGraph", "replay_schedule", "version"]

@@ -30,8 +30,13 @@ EXPORTED = [
     "pe_device_status", "pe_kernel_launches", "pe_replay_attn_static_scratch", "pe_selftest_bounded_wait",
     "pe_last_attn_plan", "pe_seq_fork", "pe_checkpoint_add", "pe_checkpoint_select", "pe_restore",
     "pe_seq_checkpoints", "pe_page_refs", "pe_prov_create", "pe_prov_destroy", "pe_prov_add",
-    "pe_prov_locate_source", "pe_prov_taint_closure", "pe_prov_first_entry", "pe_last_error", "pe_version",
+    "pe_prov_locate_source", "pe_prov_taint_closure", "pe_prov_first_entry", "pe_replay_schedule",
+    "pe_replay_rounds", "pe_last_error", "pe_version",
 ]
+
+# Turn kinds and replay policies of pe_replay_schedule (pe.h).
+TURN_INPUT, TURN_MODEL_INDEP, TURN_MODEL_DEP = 0, 1, 2
+POLICY_SELECTIVE, POLICY_PREFIX_CACHE = 0, 1
 
 
 class PEError(RuntimeError):
@@ -91,6 +96,8 @@ _sigs = {
     "pe_prov_taint_closure": [_P, _I64, _I64P, _I32, _I32P, _I32P],
     "pe_prov_first_entry": [_P, _I64, _I64P],
     "pe_replay_attn_static_scratch": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
+    "pe_replay_schedule": [_I32, _I32P, _I32P, _I32P, _I32, _I32P, _I64, _I32P, _I64P],
+    "pe_replay_rounds": [_P, _I32, _I32P, _I32, _I32P, _I32P, _P, _P, _P, _P, _I32, ctypes.c_float, _P],
 }
 for _name, _args in _sigs.items():
     _fn = getattr(_lib, _name)
@@ -123,6 +130,29 @@ def _i32_array(vals):
 def _i64_array(vals):
     vals = [int(v) for v in vals]
     return (ctypes.c_int64 * max(1, len(vals)))(*vals)
+
+
+def replay_schedule(agents_turns, policy):
+    """pe_replay_schedule: agents_turns[i] = ((n_tokens, kind), ...).  Returns
+    (take, decode_tokens): take is int32 numpy [rounds][agents] (positions each
+    agent appends and attends per round); decode_tokens the positions decoded."""
+    import numpy as np
+    cu, lens, kinds = [0], [], []
+    for turns in agents_turns:
+        for n, k in turns:
+            lens.append(int(n))
+            kinds.append(int(k))
+        cu.append(len(lens))
+    n = len(agents_turns)
+    rounds, dec = ctypes.c_int32(), ctypes.c_int64()
+    cu_a, len_a, kind_a = _i32_array(cu), _i32_array(lens), _i32_array(kinds)
+    _check(_lib.pe_replay_schedule(n, cu_a, len_a, kind_a, int(policy), None, 0, ctypes.byref(rounds),
+                                   ctypes.byref(dec)))
+    take = np.zeros((rounds.value, n), dtype=np.int32)
+    if take.size:
+        _check(_lib.pe_replay_schedule(n, cu_a, len_a, kind_a, int(policy), take.ctypes.data_as(_I32P), take.size,
+                                       ctypes.byref(rounds), ctypes.byref(dec)))
+    return take, dec.value
 
 
 def _stream(stream):
@@ -314,6 +344,37 @@ class PagedKVCache:
         _check(_lib.pe_replay_attn_batch(self._h, len(seqs), _i32_array(seqs), layer, _dev_ptr(Q, "Q"),
                                          _i32_array(cu_q), _dev_ptr(out, "out"), Q.shape[1], scale,
                                          self._s(stream)))
+        return out
+
+    def replay_rounds(self, seqs, take, cu_tok, K=None, V=None, Q=None, out=None, softmax_scale=None,
+                      num_q_heads=None, stream=None):
+        """pe_replay_rounds: round r appends take[r][i] positions of agent i and
+        attends them, all layers.  K, V: CUDA bf16 [L][N][Hkv][d]; Q, out:
+        [L][N][Hq][d]; agent i owns rows cu_tok[i]:cu_tok[i+1].  Host-only
+        caches take no tensors (bookkeeping only)."""
+        import numpy as np
+        import torch
+        take = np.ascontiguousarray(take, dtype=np.int32)
+        n_rounds = int(take.shape[0]) if take.ndim == 2 else 0
+        if take.size and take.shape[1] != len(seqs):
+            raise ValueError("take must be [rounds][len(seqs)]")
+        take_p = take.ctypes.data_as(_I32P) if take.size else None
+        scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
+        if self.host_only:
+            hq = num_q_heads or self.num_kv_heads
+            _check(_lib.pe_replay_rounds(self._h, len(seqs), _i32_array(seqs), n_rounds, take_p, _i32_array(cu_tok),
+                                         None, None, None, None, hq, scale, self._s(stream)))
+            return None
+        self._check_kv(K, V)
+        if Q.dim() != 4 or Q.shape[0] != self.num_layers or Q.shape[1] != K.shape[1] or Q.shape[3] != self.head_dim:
+            raise ValueError("Q must be [L][N][Hq][d] with the rows of K")
+        if K.shape[1] != cu_tok[-1]:
+            raise ValueError("K row count does not match cu_tok")
+        if out is None:
+            out = torch.empty_like(Q)
+        _check(_lib.pe_replay_rounds(self._h, len(seqs), _i32_array(seqs), n_rounds, take_p, _i32_array(cu_tok),
+                                     _dev_ptr(K, "K"), _dev_ptr(V, "V"), _dev_ptr(Q, "Q"), _dev_ptr(out, "out"),
+                                     Q.shape[2], scale, self._s(stream)))
         return out
 
     def replay_attn_static_scratch(self, seq, layer, Q, out=None, softmax_scale=None, stream=None):

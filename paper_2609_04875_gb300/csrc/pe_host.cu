@@ -907,6 +907,83 @@ pe_status pe_replay_attn_batch(pe_cache *c, int32_t n, const int32_t *seqs, int3
                          static_cast<cudaStream_t>(stream));
 }
 
+pe_status pe_replay_rounds(pe_cache *c, int32_t n, const int32_t *seqs, int32_t n_rounds, const int32_t *take,
+                           const int32_t *cu_tok, const void *K, const void *V, const void *Q, void *out,
+                           int32_t num_q_heads, float softmax_scale, void *stream)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (n < 0 || n_rounds < 0 || (n > 0 && (!seqs || !cu_tok)) || (n > 0 && n_rounds > 0 && !take))
+        return fail(PE_ERR_INVALID, "bad rounds arguments");
+    if (n == 0) return PE_OK;
+    if (cu_tok[0] != 0) return fail(PE_ERR_INVALID, "cu_tok[0] must be 0");
+    const int64_t N = cu_tok[n];
+    pe_status s;
+    if (c->host_only) {
+        if (num_q_heads <= 0 || num_q_heads % c->cfg.num_kv_heads != 0)
+            return fail(PE_ERR_INVALID, "num_q_heads %d is not a multiple of num_kv_heads", num_q_heads);
+    } else if ((s = check_attn_args(c, 0, Q, out, num_q_heads, softmax_scale, N > 0)) != PE_OK) {
+        return s;
+    }
+    if (!c->host_only && N > 0) {
+        if (!K || !V) return fail(PE_ERR_INVALID, "null K or V");
+        if (!aligned16(K) || !aligned16(V)) return fail(PE_ERR_INVALID, "K and V must be 16-byte aligned");
+    }
+    // every agent: a live, distinct sequence whose rounds cover its rows exactly,
+    // and room for all of its positions (pages counted once, up front)
+    std::vector<uint8_t> seen(c->cfg.max_seqs, 0);
+    int64_t need = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        if (cu_tok[i + 1] < cu_tok[i]) return fail(PE_ERR_INVALID, "cu_tok must be non-decreasing");
+        AppendPlan pl{};
+        if ((s = plan_append(c, seqs[i], cu_tok[i + 1] - cu_tok[i], &pl)) != PE_OK) return s;
+        if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice", seqs[i]);
+        seen[seqs[i]] = 1;
+        need += pl.need;
+        int64_t sum = 0;
+        for (int32_t r = 0; r < n_rounds; ++r) {
+            const int32_t t = take[static_cast<int64_t>(r) * n + i];
+            if (t < 0) return fail(PE_ERR_INVALID, "negative take in round %d", r);
+            sum += t;
+        }
+        if (sum != cu_tok[i + 1] - cu_tok[i])
+            return fail(PE_ERR_INVALID, "agent %d: rounds cover %lld of its %d rows", i, static_cast<long long>(sum),
+                        cu_tok[i + 1] - cu_tok[i]);
+    }
+    if (need > static_cast<int64_t>(c->free_stack.size()))
+        return fail(PE_ERR_OOM, "the rounds need %lld pages, %zu free", static_cast<long long>(need),
+                    c->free_stack.size());
+
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int64_t row_bytes = static_cast<int64_t>(num_q_heads) * c->cfg.head_dim * 2;  // one bf16 [Hq][d] row
+    std::vector<int32_t> done(n, 0);
+    std::vector<AppendPlan> plans;
+    std::vector<AttnItem> items;
+    for (int32_t r = 0; r < n_rounds; ++r) {
+        plans.clear();
+        items.clear();
+        for (int32_t i = 0; i < n; ++i) {
+            const int32_t t = take[static_cast<int64_t>(r) * n + i];
+            if (t == 0) continue;
+            AppendPlan pl{};
+            plan_append(c, seqs[i], t, &pl);  // checked above for the whole suffix
+            pl.tok0 = cu_tok[i] + done[i];
+            plans.push_back(pl);
+            items.push_back(AttnItem{seqs[i], cu_tok[i] + done[i], t});
+            done[i] += t;
+        }
+        if (plans.empty()) continue;
+        if ((s = apply_appends(c, plans, K, V, N, st)) != PE_OK) return s;
+        if (c->host_only) continue;
+        for (int32_t layer = 0; layer < c->cfg.num_layers; ++layer) {
+            const int64_t off = static_cast<int64_t>(layer) * N * row_bytes;
+            s = run_attention(c, items, layer, static_cast<const char *>(Q) + off, N, static_cast<char *>(out) + off,
+                              num_q_heads, softmax_scale, st);
+            if (s != PE_OK) return s;
+        }
+    }
+    return PE_OK;
+}
+
 pe_status pe_replay_attn_static_scratch(pe_cache *c, int32_t seq, int32_t layer, const void *Q, void *out,
                                         int32_t n_q, int32_t num_q_heads, float softmax_scale, void *stream)
 {

@@ -9,6 +9,10 @@ all agents at once:
   3. replay attention of the suffix queries Q', per layer    -> pe_replay_attn_batch
 After a step every agent again holds T tokens, so steps repeat without reset.
 All inputs are device-resident bf16 tensors; the driver only orders the calls.
+
+`RoundsDriver` replays turn-structured suffixes instead: after the crop, one
+pe_replay_rounds call runs the lockstep rounds of a replay policy (known turns
+re-prefilled, the others re-decoded one position per round; Sec. 4.5).
 """
 from __future__ import annotations
 
@@ -41,7 +45,6 @@ class ReplayDriver:
         S = [a.S for a in w.agents]
         self.cu = [0] + list(np.cumsum(S).astype(int))
         n = self.cu[-1]
-        # (twice the agents' sequence slots: room for a branch of every agent)
         # sanitized suffix inputs, packed over agents: K'/V' [L][sum S][Hkv][d], Q' [L][sum S][Hq][d]
         self.Kc = torch.empty((L, n, hkv, d), dtype=torch.bfloat16, device=self.device)
         self.Vc = torch.empty_like(self.Kc)
@@ -124,3 +127,94 @@ class ReplayDriver:
         per_layer = 2.0 * (2 * P * w.num_kv_heads * w.head_dim + 4 * S * w.num_kv_heads * w.head_dim
                            + 2 * S * w.num_q_heads * w.head_dim)
         return per_layer * w.num_layers
+
+
+class RoundsDriver(ReplayDriver):
+    """Replay of a turn-structured workload (agents carry ``turns``) with the
+    indep split (Sec. 4.5): one step crops every agent to tau and then runs
+    the rounds of ``policy`` (selective replay or the prefix-cache comparator)
+    through pe_replay_rounds, all layers, in one library call."""
+
+    def __init__(self, w, policy, device="cuda", **kw):
+        super().__init__(w, device, **kw)
+        self.set_policy(policy)
+
+    def set_policy(self, policy):
+        from .binding import replay_schedule
+        self.policy = policy
+        self.take, self.decode_tokens = replay_schedule([a.turns for a in self.w.agents], policy)
+
+    @property
+    def rounds(self) -> int:
+        return int(self.take.shape[0])
+
+    def step(self, stream=None, attn_events=None, bufs=None):
+        K, V, Q, out = bufs or self.buffers()
+        self.crop(stream)
+        self.cache.replay_rounds(self.seqs, self.take, self.cu, K, V, Q, out, softmax_scale=self.w.softmax_scale,
+                                 stream=stream)
+        return out
+
+    # -- the same rounds through the per-round public calls, for timing attention alone
+    def round_buffers(self):
+        """Per round: (seqs, cu, K, V, Q, out) with the round's rows gathered and packed."""
+        done = [0] * len(self.seqs)
+        per_round = []
+        for r in range(self.rounds):
+            seqs, cu, idx = [], [0], []
+            for i, s in enumerate(self.seqs):
+                t = int(self.take[r, i])
+                if t == 0:
+                    continue
+                lo = self.cu[i] + done[i]
+                idx.extend(range(lo, lo + t))
+                seqs.append(s)
+                cu.append(cu[-1] + t)
+                done[i] += t
+            ix = torch.tensor(idx, dtype=torch.long, device=self.device)
+            per_round.append((seqs, cu, self.Kc.index_select(1, ix).contiguous(),
+                              self.Vc.index_select(1, ix).contiguous(), self.Qc.index_select(1, ix).contiguous(),
+                              torch.empty((self.w.num_layers, len(idx), self.w.num_q_heads, self.w.head_dim),
+                                          dtype=torch.bfloat16, device=self.device)))
+        return per_round
+
+    def step_per_round(self, per_round, stream=None, attn_events=None, gate_cycles=0):
+        """crop, then per round: pe_append_kv_batch and one pe_replay_attn_batch per
+        layer; attn_events[r] = (start, end) recorded around round r's attention.
+        gate_cycles > 0 enqueues a fixed-length busy kernel (torch.cuda._sleep)
+        before each start event, so that the host has queued the round's
+        launches before the GPU reaches them and the events time the kernels,
+        not the host."""
+        self.crop(stream)
+        for r, (seqs, cu, K, V, Q, out) in enumerate(per_round):
+            self.cache.append_kv_batch(seqs, K, V, cu, stream=stream)
+            if attn_events is not None:
+                if gate_cycles > 0:
+                    with torch.cuda.stream(stream or torch.cuda.current_stream(self.device)):
+                        torch.cuda._sleep(int(gate_cycles))
+                attn_events[r][0].record(stream)
+            for layer in range(self.w.num_layers):
+                self.cache.replay_attn_batch(seqs, layer, Q[layer], cu, out=out[layer],
+                                             softmax_scale=self.w.softmax_scale, stream=stream)
+            if attn_events is not None:
+                attn_events[r][1].record(stream)
+
+    def round_work(self):
+        """Per round: (algorithmic FLOPs, algorithmic bytes) of its attention,
+        all layers: unmasked (query, key) pairs x 4d x Hq; every key of the
+        round's agents read once per kv-head, their Q read and O written."""
+        w = self.w
+        lens = [a.P for a in w.agents]
+        work = []
+        for r in range(self.rounds):
+            fl = by = 0.0
+            for i in range(len(self.seqs)):
+                t = int(self.take[r, i])
+                if t == 0:
+                    continue
+                lens[i] += t
+                n = lens[i]
+                fl += 4.0 * w.head_dim * w.num_q_heads * (t * (n - t) + t * (t + 1) / 2)
+                by += 2.0 * (2 * n * w.num_kv_heads * w.head_dim + 2 * t * w.num_q_heads * w.head_dim)
+            work.append((fl * w.num_layers, by * w.num_layers))
+        return work
