@@ -256,27 +256,71 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 4);
     const WaitCtx wctx{abort_flag, p.status};
 
-    if (threadIdx.x == 0) {
-        ptx::mbar_init(b_q_full, 1);
-        for (int s = 0; s < C::kStages; ++s) {
-            ptx::mbar_init(b_k_full + 8 * s, 1);
-            ptx::mbar_init(b_k_empty + 8 * s, 1);
-            ptx::mbar_init(b_v_full + 8 * s, 1);
-            ptx::mbar_init(b_v_empty + 8 * s, 1);
+    // The producer warp initialises the barriers and starts the Q loads and the
+    // first key tile's loads before the CTA-wide sync, while the MMA warp
+    // allocates TMEM; no other thread touches a barrier before the sync.
+    const int ppt = kBN / p.ps;                 // pages per key tile
+    const int n_ops = ppt * C::kRegions;        // TMA boxes per K (or V) tile, <= 32
+    const int op_page = lane / C::kRegions;     // this lane's box: page index and half
+    const int op_reg = lane % C::kRegions;
+    const bool op_on = lane < n_ops;
+    const uint32_t op_off = op_reg * C::kRegionBytes + op_page * p.ps * 128;
+    auto page_of = [&](int i) -> int {          // this lane's page id of key tile i (or -1)
+        const int lp = (kt0 + i) * ppt + lane;
+        return (lane < ppt && lp < sq.n_pages) ? p.page_table[sq.table_row + lp] : -1;
+    };
+    auto issue_kv = [&](int i, int page) {      // all lanes: TMA boxes of key tile i into stage i % S
+        const int s = i % C::kStages;
+        const int pg = __shfl_sync(0xffffffffu, page, op_page & 31);
+        // rows of pages past the sequence read as zeros (out-of-bounds box)
+        const int y = pg >= 0 ? ((p.layer * p.num_pages + pg) * p.hkv + kvh) * p.ps : p.oob_row;
+        if (i >= C::kStages && !wait_bar_warp(b_k_empty + 8 * s, ((i / C::kStages) - 1) & 1, wctx)) return false;
+        if (lane == 0) ptx::mbar_arrive_expect_tx(b_k_full + 8 * s, C::kTileBytes);
+        __syncwarp();
+        if (op_on) ptx::tma_load_2d(k_smem0 + s * C::kTileBytes + op_off, &tm_k, op_reg * 64, y, b_k_full + 8 * s);
+        if (i >= C::kStages && !wait_bar_warp(b_v_empty + 8 * s, ((i / C::kStages) - 1) & 1, wctx)) return false;
+        if (lane == 0) ptx::mbar_arrive_expect_tx(b_v_full + 8 * s, C::kTileBytes);
+        __syncwarp();
+        if (op_on) ptx::tma_load_2d(v_smem0 + s * C::kTileBytes + op_off, &tm_v, op_reg * 64, y, b_v_full + 8 * s);
+        return true;
+    };
+    int page_next = -1;
+    if (warp == 8) {
+        if (n_all > 0) page_next = page_of(0);   // global load in flight during the set-up
+        if (lane == 0) {
+            ptx::mbar_init(b_q_full, 1);
+            for (int s = 0; s < C::kStages; ++s) {
+                ptx::mbar_init(b_k_full + 8 * s, 1);
+                ptx::mbar_init(b_k_empty + 8 * s, 1);
+                ptx::mbar_init(b_v_full + 8 * s, 1);
+                ptx::mbar_init(b_v_empty + 8 * s, 1);
+            }
+            for (int t = 0; t < 2; ++t) {
+                ptx::mbar_init(b_s_full + 8 * t, 1);
+                ptx::mbar_init(b_p_full + 8 * t, 128);
+                ptx::mbar_init(b_o_done + 8 * t, 1);
+            }
+            *abort_flag = 0;
+            ptx::fence_barrier_init();
+            ptx::fence_proxy_async_smem();
+            ptx::prefetch_tensormap(&tm_q);
+            ptx::prefetch_tensormap(&tm_k);
+            ptx::prefetch_tensormap(&tm_v);
+            if (n_all > 0) {
+                const int nq = geo[1].qt >= 0 ? 2 : 1;
+                ptx::mbar_arrive_expect_tx(b_q_full, nq * C::kTileBytes);
+                for (int t = 0; t < nq; ++t)
+                    for (int r = 0; r < C::kRegions; ++r)
+                        ptx::tma_load_3d(q_smem + t * C::kTileBytes + r * C::kRegionBytes, &tm_q, r * 64, kvh * g,
+                                         sq.q_row0 + geo[t].q_first, b_q_full);
+            }
         }
-        for (int t = 0; t < 2; ++t) {
-            ptx::mbar_init(b_s_full + 8 * t, 1);
-            ptx::mbar_init(b_p_full + 8 * t, 128);
-            ptx::mbar_init(b_o_done + 8 * t, 1);
+        __syncwarp();
+        if (n_all > 0) {
+            const int page = page_next;
+            if (n_all > 1) page_next = page_of(1);
+            issue_kv(0, page);  // tile 0 never waits (its stage is fresh)
         }
-        *abort_flag = 0;
-        ptx::fence_barrier_init();
-        ptx::fence_proxy_async_smem();
-    }
-    if (warp == 8 && lane == 0) {
-        ptx::prefetch_tensormap(&tm_q);
-        ptx::prefetch_tensormap(&tm_k);
-        ptx::prefetch_tensormap(&tm_v);
     }
     if (warp == 9) {
         ptx::tmem_alloc(ptx::smem_addr(tmem_slot), C::kTmemCols);
@@ -288,44 +332,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *tmem_slot;
 
     if (warp == 8 && n_all > 0) {
-        // =================================================== producer (TMA)
-        if (lane == 0) {
-            const int nq = geo[1].qt >= 0 ? 2 : 1;
-            ptx::mbar_arrive_expect_tx(b_q_full, nq * C::kTileBytes);
-            for (int t = 0; t < nq; ++t)
-                for (int r = 0; r < C::kRegions; ++r)
-                    ptx::tma_load_3d(q_smem + t * C::kTileBytes + r * C::kRegionBytes, &tm_q, r * 64, kvh * g,
-                                     sq.q_row0 + geo[t].q_first, b_q_full);
-        }
-        const int ppt = kBN / p.ps;                 // pages per key tile
-        const int n_ops = ppt * C::kRegions;        // TMA boxes per K (or V) tile, <= 32
-        const int op_page = lane / C::kRegions;     // this lane's box: page index and half
-        const int op_reg = lane % C::kRegions;
-        const bool op_on = lane < n_ops;
-        const uint32_t op_off = op_reg * C::kRegionBytes + op_page * p.ps * 128;
-        int page_next = -1;
-        {
-            const int lp = kt0 * ppt + lane;
-            if (lane < ppt && lp < sq.n_pages) page_next = p.page_table[sq.table_row + lp];
-        }
-        for (int i = 0; i < n_all; ++i) {
-            const int s = i % C::kStages;
+        // =================================================== producer (TMA), tiles 1..
+        for (int i = 1; i < n_all; ++i) {
             const int page = page_next;
-            if (i + 1 < n_all) {  // prefetch the next tile's page ids
-                const int lp = (kt0 + i + 1) * ppt + lane;
-                page_next = (lane < ppt && lp < sq.n_pages) ? p.page_table[sq.table_row + lp] : -1;
-            }
-            const int pg = __shfl_sync(0xffffffffu, page, op_page & 31);
-            // rows of pages past the sequence read as zeros (out-of-bounds box)
-            const int y = pg >= 0 ? ((p.layer * p.num_pages + pg) * p.hkv + kvh) * p.ps : p.oob_row;
-            if (i >= C::kStages && !wait_bar_warp(b_k_empty + 8 * s, ((i / C::kStages) - 1) & 1, wctx)) break;
-            if (lane == 0) ptx::mbar_arrive_expect_tx(b_k_full + 8 * s, C::kTileBytes);
-            __syncwarp();
-            if (op_on) ptx::tma_load_2d(k_smem0 + s * C::kTileBytes + op_off, &tm_k, op_reg * 64, y, b_k_full + 8 * s);
-            if (i >= C::kStages && !wait_bar_warp(b_v_empty + 8 * s, ((i / C::kStages) - 1) & 1, wctx)) break;
-            if (lane == 0) ptx::mbar_arrive_expect_tx(b_v_full + 8 * s, C::kTileBytes);
-            __syncwarp();
-            if (op_on) ptx::tma_load_2d(v_smem0 + s * C::kTileBytes + op_off, &tm_v, op_reg * 64, y, b_v_full + 8 * s);
+            if (i + 1 < n_all) page_next = page_of(i + 1);  // prefetch the next tile's page ids
+            if (!issue_kv(i, page)) break;
         }
         __syncwarp();
         if (*abort_flag && lane == 0) {
