@@ -173,10 +173,10 @@ def oracle_tokens_per_s(w, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "agent_batch": {"bytes": 697.009152e6 + 328.204544e6, "profile": "profiles/replay_attn_agent_batch.md",
-                    "src_sha256": "6c7f02193ba40db6058212f482f1f89251554b8b4166af8e998283581fc845c3"},
-    "short_suffix": {"bytes": 1.076274e9 + 21.424384e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
-                     "src_sha256": "6c7f02193ba40db6058212f482f1f89251554b8b4166af8e998283581fc845c3"},
+    "agent_batch": {"bytes": 695.853056e6 + 328.461824e6, "profile": "profiles/replay_attn_agent_batch.md",
+                    "src_sha256": "41d26fc6835fb329162de834ec0cfa144301682912a9d2651026e677a1f7a4e1"},
+    "short_suffix": {"bytes": 1.076216e9 + 21.185280e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
+                     "src_sha256": "41d26fc6835fb329162de834ec0cfa144301682912a9d2651026e677a1f7a4e1"},
 }
 ATTN_SRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc", "pe_attn.cu")
 
