@@ -242,12 +242,20 @@ pe_status pe_cache_pools(const pe_cache *cache, void **k_pool, void **v_pool);
  * "num_splits" = 0 (auto) or the split count; "debug_poison" = 0/1: crop
  * fills freed pages and the stale tail of the last kept page with a finite
  * sentinel (bf16 2^100), so that a kernel reading them unmasked gives a
- * visibly wrong result. */
+ * visibly wrong result; "decode_kernel" = 1 (default) / 2 / 0: sequences
+ * whose n_q x (Hq/Hkv) query rows fit in 16 take a decode kernel with the
+ * split-KV merge done in-kernel -- 1: tcgen05 with keys on the MMA's M side
+ * for d = 128, CUDA cores for d = 64; 2: CUDA cores for both; 0: no decode
+ * kernel (the prefill kernel serves every call).  Split
+ * partials and the decode kernel's merge counters live in the cache's
+ * workspace, so attention calls on one cache must not overlap on the GPU
+ * (issue them on one stream, or order the streams). */
 pe_status pe_set_option(pe_cache *cache, const char *key, int64_t value);
 
 /* Synchronises `stream` and reads the device status word.  *code = 0 when no
  * kernel reported a problem, else the first recorded code (1 = a bounded
- * wait ran out).  clear != 0 resets it.  Returns DEVICE_TIMEOUT if *code != 0. */
+ * wait ran out; 2 = the decode kernel met a page id outside the pool and
+ * skipped it).  clear != 0 resets it.  Returns DEVICE_TIMEOUT if *code != 0. */
 pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *stream);
 
 /* Failure-detection self-test: launches one kernel whose single wait (the same
@@ -259,8 +267,9 @@ pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *
 pe_status pe_selftest_bounded_wait(pe_cache *cache, int64_t limit_ns, void *stream);
 
 /* Plan of the most recent replay-attention launch group on this cache: split
- * = 1 when the split-KV path (with its combine launch) ran, n_splits = key
- * splits of its first sequence, ctas = attention CTAs launched. */
+ * = 1 when the split-KV path ran (the tensor-core kernel's combine launch, or
+ * the decode kernel's in-kernel merge), n_splits = key splits of its first
+ * sequence, ctas = attention CTAs launched. */
 pe_status pe_last_attn_plan(const pe_cache *cache, int32_t *split, int32_t *n_splits, int32_t *ctas);
 
 /* Number of kernel launches this cache has made so far (crop, append,

@@ -1,0 +1,899 @@
+// Decode attention over a paged KV cache on sm_103a.
+//
+// What it computes (Alg. 1 replay loop for positions that are generated again
+// one per pass; Sec. 4.5: target-dependent turns are re-decoded): the n_q x g
+// query rows of one kv-head -- at most 16, e.g. one new position of a GQA
+// group -- attend the sequence's keys, query i at position len-n_q+i seeing
+// keys 0..len-n_q+i:
+//     O = softmax(scale * q K^T) V      (bf16 in, fp32 accumulate, bf16 out)
+//
+// With so few rows per key this is a stream over the sequence's K/V, bound by
+// HBM, not by a contraction: CUDA cores do the arithmetic and the design keeps
+// HBM busy.  One CTA = (sequence, kv-head, key split):
+//   warp 8       producer: reads page ids one tile ahead; its lanes issue one
+//                TMA box per (page, 64-column half) of K and of V into a
+//                3-stage ring of 64-key tiles (128-byte swizzle, so that
+//                reads along a key and along a column are both conflict-free).
+//                Boxes past the sequence read zeros.
+//   warps 0-7    consumers, each an independent online-softmax worker over
+//                its own keys [8w, 8w+8) of every tile (no CTA barrier per
+//                tile):
+//     1. scores: lane l takes key 8w + l/4 and the d-quarter l%4; its partial
+//        dots with the RB query rows (fp32, shared memory) are summed over the
+//        key's four lanes by a reduce-scatter, leaving each lane RB/4 rows;
+//     2. softmax over the warp's 8 keys per row: running max m and sum l in
+//        registers, weights P (exp2) to a warp-private shared buffer;
+//     3. O[r][cols] = alpha_r O[r][cols] + sum_k P[k][r] V[k][cols], lane l
+//        taking the columns [l*d/32, (l+1)*d/32).
+//   After the last tile the 8 warps' (m, l, O) are merged through shared
+//   memory.  With one split the rows are normalised and written.  With several,
+//   each split writes (O, m, l) to the workspace and the last split of a
+//   (sequence, kv-head) to finish -- a ticket counter -- merges them, so no
+//   second launch is needed; it resets the counter for the next launch.
+// Keys past the sequence or past a row's query position get weight 0.  Every
+// wait is bounded.
+#include "dev_common.cuh"
+
+namespace pe {
+namespace {
+
+constexpr int kDecWarps = 8;                       // consumer warps
+constexpr int kConsumers = 32 * kDecWarps;
+constexpr int kDecThreads = kConsumers + 32;       // + producer warp
+constexpr int kDecStages = 3;
+constexpr int kBarConsumers = 1;                   // named barrier of the consumer warps
+constexpr int kStatusBadPage = 2;                  // device status: page id outside the pool
+
+// Every split of a (sequence, kv-head) has written its partial (O, m, l) for
+// the RB rows: O unnormalised [RB][HD], m the running max (log2 units), l the
+// sum of exp2(x - m).  Each split takes a ticket (also after an abort, so the
+// counter returns to 0); the last one merges the partials into the bf16
+// output, O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s, and resets the
+// counter for the next launch.  Called by `nthreads` threads (whole warps,
+// thread ids 0..nthreads-1) that share named barrier `bar`.
+template <int RB, int HD>
+__device__ __forceinline__ void split_merge(const DecodeParams &p, const DecodeSeq &sq, int si, int kvh, int n_rows,
+                                            int tid, int nthreads, int bar, int *s_ticket)
+{
+    const float *pm = p.part + static_cast<int64_t>(p.total_ctas) * RB * HD;
+    const float *pl = pm + static_cast<int64_t>(p.total_ctas) * RB;
+    const int g = p.group;
+    __threadfence();
+    ptx::bar_sync(bar, nthreads);
+    int32_t *ticket = p.tickets + si * p.hkv + kvh;
+    if (tid == 0) *s_ticket = atomicAdd(ticket, 1);
+    ptx::bar_sync(bar, nthreads);
+    if (*s_ticket != sq.n_splits - 1) return;
+    __threadfence();
+    const int64_t c0 = sq.cta0 + static_cast<int64_t>(kvh) * sq.n_splits;
+    for (int e = tid; e < RB * HD / 2; e += nthreads) {
+        const int r = (2 * e) / HD;
+        const int col = (2 * e) % HD;
+        if (r >= n_rows) continue;
+        float mx = -INFINITY;
+        for (int sp = 0; sp < sq.n_splits; ++sp) mx = fmaxf(mx, __ldcg(pm + (c0 + sp) * RB + r));
+        float den = 0.f, o0 = 0.f, o1 = 0.f;
+        if (mx != -INFINITY) {
+            for (int sp = 0; sp < sq.n_splits; ++sp) {
+                const float ms = __ldcg(pm + (c0 + sp) * RB + r);
+                if (ms == -INFINITY) continue;
+                const float w = ex2(ms - mx);
+                den += w * __ldcg(pl + (c0 + sp) * RB + r);
+                const float2 x =
+                    __ldcg(reinterpret_cast<const float2 *>(p.part + ((c0 + sp) * RB + r) * HD + col));
+                o0 += w * x.x;
+                o1 += w * x.y;
+            }
+        }
+        const float inv = den > 0.f ? 1.0f / den : 0.f;
+        __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(p.out) +
+                             (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD + col;
+        *reinterpret_cast<uint32_t *>(dst) = pack_bf16(o0 * inv, o1 * inv);
+    }
+    if (tid == 0) *ticket = 0;
+}
+
+template <int HD, int RB>
+struct DecCfg {
+    static constexpr int kRegions = HD / 64;                 // 128-byte swizzle atoms along d
+    static constexpr int kRegionBytes = kDecKeys * 128;      // 64 keys x 64 columns (bf16)
+    static constexpr int kTileBytes = kRegions * kRegionBytes;
+    static constexpr int kStageBytes = 2 * kTileBytes;       // K then V
+    static constexpr int kQuarter = HD / 4;                  // d-columns per scoring lane
+    static constexpr int kQChunks = kQuarter / 8;            // 16-byte chunks per quarter row
+    static constexpr int kQStride = kQuarter + 4;            // floats per (row, quarter) of q: spreads banks
+    static constexpr int kRPL = RB / 4;                      // score rows per lane
+    static constexpr int kCW = HD / 32;                      // d-columns per lane in P V
+    static constexpr int kOffQ = kDecStages * kStageBytes;   // q [RB][4][kQStride] fp32, log2 units
+    static constexpr int kOffPw = kOffQ + RB * 4 * kQStride * 4;   // per warp: P [8 keys][RB], alpha [RB]
+    static constexpr int kPwFloats = 8 * RB + RB;
+    static constexpr int kOffML = kOffPw + kDecWarps * kPwFloats * 4;  // merge: m, l [8 warps][RB]
+    static constexpr int kOffBar = kOffML + 2 * kDecWarps * RB * 4;    // full[S], empty[S]
+    static constexpr int kOffMisc = kOffBar + 2 * kDecStages * 8;  // abort flag, ticket, tiles issued
+    static constexpr int kSmem = kOffMisc + 16;
+    static constexpr int kDynSmem = kSmem + 1024;            // the stages start 1024-byte aligned
+    static constexpr int kMinBlocks = RB <= 8 ? 2 : 1;
+    static_assert(RB == 4 || RB == 8 || RB == 16, "row capacity");
+    static_assert(kDecWarps * RB * HD * 4 <= kDecStages * kStageBytes, "the O merge reuses the stages");
+    static_assert(kOffBar % 8 == 0, "mbarrier alignment");
+};
+
+template <int HD, int RB>
+__global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
+    decode_attn_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                       const __grid_constant__ DecodeParams p)
+{
+    using C = DecCfg<HD, RB>;
+    constexpr int CW = C::kCW;
+    constexpr int RPL = C::kRPL;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    int si = 0;
+    while (si + 1 < p.n_seqs && static_cast<int>(blockIdx.x) >= p.seqs[si + 1].cta0) ++si;
+    const DecodeSeq &sq = p.seqs[si];
+    const int local = static_cast<int>(blockIdx.x) - sq.cta0;
+    const int kvh = local / sq.n_splits;
+    const int split = local - kvh * sq.n_splits;
+    const int g = p.group;
+    const int n_rows = sq.n_q * g;
+    const int n_tiles_all = (sq.n_keys + kDecKeys - 1) / kDecKeys;
+    const int t0 = split * p.split_tiles;
+    const int nt = max(0, min(t0 + p.split_tiles, n_tiles_all) - t0);
+    const int qpos0 = sq.n_keys - sq.n_q;  // position of query 0
+
+    float *s_q = reinterpret_cast<float *>(smem + C::kOffQ);
+    float *s_ml = reinterpret_cast<float *>(smem + C::kOffML);
+    const uint32_t bar0 = ptx::smem_addr(smem + C::kOffBar);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc);
+    int *s_ticket = reinterpret_cast<int *>(smem + C::kOffMisc + 4);
+    volatile int *s_issued = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 8);
+    const WaitCtx wctx{abort_flag, p.status};
+    auto full = [&](int s) { return bar0 + 8u * s; };
+    auto empty = [&](int s) { return bar0 + 8u * (kDecStages + s); };
+
+    if (threadIdx.x == kConsumers) {
+        for (int s = 0; s < kDecStages; ++s) {
+            ptx::mbar_init(full(s), 1);
+            ptx::mbar_init(empty(s), kDecWarps);
+        }
+        *abort_flag = 0;
+        *s_issued = 0;
+        ptx::fence_barrier_init();
+        ptx::fence_proxy_async_smem();
+        ptx::prefetch_tensormap(&tm_k);
+        ptx::prefetch_tensormap(&tm_v);
+    }
+    // this kv-head's query rows, scaled to log2 units (rows past n_q x g are zero)
+    for (int e = threadIdx.x; e < RB * HD; e += kDecThreads) {
+        const int r = e / HD;
+        const int col = e % HD;
+        float x = 0.f;
+        if (r < n_rows) {
+            const __nv_bfloat16 *src = static_cast<const __nv_bfloat16 *>(p.q) +
+                                       (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD;
+            x = __bfloat162float(src[col]) * p.scale_log2;
+        }
+        s_q[(r * 4 + col / C::kQuarter) * C::kQStride + col % C::kQuarter] = x;
+    }
+    __syncthreads();
+
+    if (warp == kDecWarps) {
+        // ============================================================ producer
+        const int kpc = p.ps < kDecKeys ? p.ps : kDecKeys;  // keys per box (the tensor maps' box height)
+        const int n_ops = (kDecKeys / kpc) * C::kRegions;   // boxes per tile and operand, <= 16
+        const int op_slot = lane / C::kRegions;             // this lane's page slot in the tile
+        const int op_reg = lane % C::kRegions;              // and 64-column half
+        const bool op_on = lane < n_ops;
+        auto page_of = [&](int t) -> int {  // this lane's page of tile t, -1 past the sequence
+            const int key0 = t * kDecKeys + op_slot * kpc;
+            if (!op_on || key0 >= sq.n_keys) return -1;
+            const int pg = p.page_table[sq.table_row + key0 / p.ps];
+            if (pg < 0 || pg >= p.num_pages) {
+                atomicCAS(p.status, 0, kStatusBadPage);
+                return -1;
+            }
+            return pg;
+        };
+        int page_next = nt > 0 ? page_of(t0) : -1;
+        for (int i = 0; i < nt; ++i) {
+            const int t = t0 + i;
+            const int s = i % kDecStages;
+            const int page = page_next;
+            if (i + 1 < nt) page_next = page_of(t + 1);
+            if (i >= kDecStages && !wait_bar_warp(empty(s), ((i / kDecStages) - 1) & 1, wctx)) break;
+            if (lane == 0) ptx::mbar_arrive_expect_tx(full(s), 2u * C::kTileBytes);
+            __syncwarp();
+            if (op_on) {
+                const int key0 = t * kDecKeys + op_slot * kpc;
+                const int y = page >= 0
+                                  ? ((p.layer * p.num_pages + page) * p.hkv + kvh) * p.ps + (key0 % p.ps)
+                                  : p.oob_row;  // past the sequence: zeros
+                const uint32_t dst =
+                    ptx::smem_addr(smem + s * C::kStageBytes) + op_reg * C::kRegionBytes + op_slot * kpc * 128;
+                ptx::tma_load_2d(dst, &tm_k, op_reg * 64, y, full(s));
+                ptx::tma_load_2d(dst + C::kTileBytes, &tm_v, op_reg * 64, y, full(s));
+            }
+            __syncwarp();
+            if (lane == 0) *s_issued = i + 1;
+        }
+    } else {
+        // ============================================================ consumers
+        float *s_pw = reinterpret_cast<float *>(smem + C::kOffPw) + warp * C::kPwFloats;  // P [8][RB], alpha [RB]
+        const int kl = lane >> 2;                  // this lane's key among the warp's 8
+        const int quarter = lane & 3;              // and d-quarter while scoring
+        const int col0 = quarter * C::kQuarter;
+        const int reg1 = col0 / 64;
+        const int lc0 = (col0 % 64) / 8;           // first 16-byte chunk of the quarter in its row
+        const int row0 = ((lane >> 1) & 1) * (RB / 2) + (lane & 1) * (RB / 4);  // rows [row0, row0 + RPL) after the reduce
+        const float *qbase = s_q + quarter * C::kQStride;
+        float m_run[RPL], l_run[RPL];
+#pragma unroll
+        for (int j = 0; j < RPL; ++j) {
+            m_run[j] = -INFINITY;
+            l_run[j] = 0.f;
+        }
+        float2 acc[RB][CW / 2];
+#pragma unroll
+        for (int r = 0; r < RB; ++r)
+#pragma unroll
+            for (int c = 0; c < CW / 2; ++c) acc[r][c] = make_float2(0.f, 0.f);
+
+        for (int i = 0; i < nt; ++i) {
+            const int s = i % kDecStages;
+            if (!wait_bar_warp(full(s), (i / kDecStages) & 1, wctx)) break;
+            const uint8_t *Ks = smem + s * C::kStageBytes;
+            const uint8_t *Vs = Ks + C::kTileBytes;
+            const int key = (t0 + i) * kDecKeys + warp * 8 + kl;
+
+            // 1. partial scores of this lane's key over its quarter, all RB rows
+            float v[RB];
+            {
+                float2 sa[RB], sb[RB];
+#pragma unroll
+                for (int r = 0; r < RB; ++r) {
+                    sa[r] = make_float2(0.f, 0.f);
+                    sb[r] = make_float2(0.f, 0.f);
+                }
+                const int krow = warp * 8 + kl;
+                const uint8_t *kp = Ks + reg1 * C::kRegionBytes + krow * 128;
+#pragma unroll
+                for (int c = 0; c < C::kQChunks; ++c) {
+                    const uint4 u = *reinterpret_cast<const uint4 *>(kp + (((lc0 + c) ^ (krow & 7)) << 4));
+                    const float2 k0 = make_float2(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u));
+                    const float2 k1 = make_float2(__uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+                    const float2 k2 = make_float2(__uint_as_float(u.z << 16), __uint_as_float(u.z & 0xffff0000u));
+                    const float2 k3 = make_float2(__uint_as_float(u.w << 16), __uint_as_float(u.w & 0xffff0000u));
+#pragma unroll
+                    for (int r = 0; r < RB; ++r) {
+                        const float4 qa = *reinterpret_cast<const float4 *>(qbase + r * 4 * C::kQStride + c * 8);
+                        const float4 qb = *reinterpret_cast<const float4 *>(qbase + r * 4 * C::kQStride + c * 8 + 4);
+                        sa[r] = fma2(make_float2(qa.x, qa.y), k0, sa[r]);
+                        sb[r] = fma2(make_float2(qa.z, qa.w), k1, sb[r]);
+                        sa[r] = fma2(make_float2(qb.x, qb.y), k2, sa[r]);
+                        sb[r] = fma2(make_float2(qb.z, qb.w), k3, sb[r]);
+                    }
+                }
+#pragma unroll
+                for (int r = 0; r < RB; ++r) v[r] = (sa[r].x + sa[r].y) + (sb[r].x + sb[r].y);
+            }
+            // sum over the key's four lanes: reduce-scatter on lane bits 1 then 0
+#pragma unroll
+            for (int lvl = 0; lvl < 2; ++lvl) {
+                const int n = RB >> lvl;
+                const int off = 2 >> lvl;
+                const bool upper = (lane & off) != 0;
+#pragma unroll
+                for (int j = 0; j < n / 2; ++j) {
+                    const float send = upper ? v[j] : v[j + n / 2];
+                    const float keep = upper ? v[j + n / 2] : v[j];
+                    v[j] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+                }
+            }
+            // 2. online softmax over the warp's 8 keys (lanes with equal lane % 4 share rows)
+            float alpha[RPL];
+#pragma unroll
+            for (int j = 0; j < RPL; ++j) {
+                const int r = row0 + j;
+                const int qpos = r < n_rows ? qpos0 + r / g : sq.n_keys - 1;
+                const float x = (key < sq.n_keys && key <= qpos) ? v[j] : -INFINITY;
+                float tm = x;
+#pragma unroll
+                for (int off = 4; off <= 16; off <<= 1) tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, off));
+                const float m_new = fmaxf(m_run[j], tm);
+                float pj = 0.f;
+                alpha[j] = 1.f;
+                if (m_new != -INFINITY) {
+                    alpha[j] = ex2(m_run[j] - m_new);
+                    pj = ex2(x - m_new);
+                }
+                float sum = pj;
+#pragma unroll
+                for (int off = 4; off <= 16; off <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+                m_run[j] = m_new;
+                l_run[j] = alpha[j] * l_run[j] + sum;
+                s_pw[kl * RB + r] = pj;
+                if (kl == 0) s_pw[8 * RB + r] = alpha[j];
+            }
+            __syncwarp();
+
+            // 3. O = alpha O + P V over the warp's 8 keys
+#pragma unroll
+            for (int r4 = 0; r4 < RB / 4; ++r4) {
+                const float4 a4 = *reinterpret_cast<const float4 *>(s_pw + 8 * RB + 4 * r4);
+                const float al[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+                for (int h = 0; h < 4; ++h)
+#pragma unroll
+                    for (int c = 0; c < CW / 2; ++c)
+                        acc[4 * r4 + h][c] = make_float2(acc[4 * r4 + h][c].x * al[h], acc[4 * r4 + h][c].y * al[h]);
+            }
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+                const int k = warp * 8 + kk;
+                float2 vf[CW / 2];
+                if constexpr (CW == 4) {
+                    // lane: columns 4l..4l+3 = half (l & 1) of chunk ((l & 15) >> 1) in region (l >> 4)
+                    const uint8_t *row = Vs + (lane >> 4) * C::kRegionBytes + k * 128;
+                    const uint2 u =
+                        *reinterpret_cast<const uint2 *>(row + ((((lane & 15) >> 1) ^ (k & 7)) << 4) + (lane & 1) * 8);
+                    vf[0] = make_float2(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u));
+                    vf[1] = make_float2(__uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+                } else {
+                    // lane: columns 2l, 2l+1 = quarter (l & 3) of chunk (l >> 2)
+                    const uint8_t *row = Vs + k * 128;
+                    const uint32_t u =
+                        *reinterpret_cast<const uint32_t *>(row + (((lane >> 2) ^ (k & 7)) << 4) + (lane & 3) * 4);
+                    vf[0] = make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+                }
+                const float4 *pk = reinterpret_cast<const float4 *>(s_pw + kk * RB);
+#pragma unroll
+                for (int r4 = 0; r4 < RB / 4; ++r4) {
+                    const float4 w = pk[r4];
+                    const float wr[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                    for (int h = 0; h < 4; ++h)
+#pragma unroll
+                        for (int c = 0; c < CW / 2; ++c)
+                            acc[4 * r4 + h][c] = fma2(make_float2(wr[h], wr[h]), vf[c], acc[4 * r4 + h][c]);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(empty(s));
+        }
+
+        // ---------------------------------------------------------- epilogue
+        // merge the 8 warps: O = sum_w 2^(m_w - M) O_w, l = sum_w 2^(m_w - M) l_w
+        const bool stopped = ptx::bar_sync_or(kBarConsumers, kConsumers, *abort_flag != 0);  // stages are free
+        float *red = reinterpret_cast<float *>(smem);  // [8][RB][HD]
+        if (kl == 0) {
+#pragma unroll
+            for (int j = 0; j < RPL; ++j) {
+                s_ml[warp * RB + row0 + j] = m_run[j];
+                s_ml[kDecWarps * RB + warp * RB + row0 + j] = l_run[j];
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < RB; ++r) {
+            float *dst = red + (warp * RB + r) * HD + lane * CW;
+            if constexpr (CW == 4) {
+                *reinterpret_cast<float4 *>(dst) = make_float4(acc[r][0].x, acc[r][0].y, acc[r][1].x, acc[r][1].y);
+            } else {
+                *reinterpret_cast<float2 *>(dst) = acc[r][0];
+            }
+        }
+        ptx::bar_sync(kBarConsumers, kConsumers);
+        const bool single = sq.n_splits == 1;
+        float *po = nullptr, *pm = nullptr, *pl = nullptr;
+        if (!single) {
+            po = p.part + static_cast<int64_t>(blockIdx.x) * RB * HD;
+            pm = p.part + static_cast<int64_t>(p.total_ctas) * RB * HD;
+            pl = pm + static_cast<int64_t>(p.total_ctas) * RB;
+        }
+        for (int e = threadIdx.x; e < RB * HD / 2; e += kConsumers) {
+            const int r = (2 * e) / HD;
+            const int col = (2 * e) % HD;
+            float mx = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kDecWarps; ++w) mx = fmaxf(mx, s_ml[w * RB + r]);
+            float o0 = 0.f, o1 = 0.f, den = 0.f;
+            if (mx != -INFINITY) {
+#pragma unroll
+                for (int w = 0; w < kDecWarps; ++w) {
+                    const float mw = s_ml[w * RB + r];
+                    if (mw == -INFINITY) continue;
+                    const float wgt = ex2(mw - mx);
+                    const float2 x = *reinterpret_cast<const float2 *>(red + (w * RB + r) * HD + col);
+                    o0 += wgt * x.x;
+                    o1 += wgt * x.y;
+                    den += wgt * s_ml[kDecWarps * RB + w * RB + r];
+                }
+            }
+            if (single) {
+                if (r < n_rows && !stopped) {
+                    const float inv = den > 0.f ? 1.0f / den : 0.f;
+                    __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(p.out) +
+                                         (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD + col;
+                    *reinterpret_cast<uint32_t *>(dst) = pack_bf16(o0 * inv, o1 * inv);
+                }
+            } else {
+                *reinterpret_cast<float2 *>(po + r * HD + col) = make_float2(o0, o1);
+                if (col == 0) {
+                    pm[static_cast<int64_t>(blockIdx.x) * RB + r] = mx;
+                    pl[static_cast<int64_t>(blockIdx.x) * RB + r] = den;
+                }
+            }
+        }
+        if (!single) split_merge<RB, HD>(p, sq, si, kvh, n_rows, threadIdx.x, kConsumers, kBarConsumers, s_ticket);
+    }
+
+    __syncthreads();
+    // After an abort, copies may still be in flight: wait (bounded) for the
+    // last tile issued on every stage before the CTA's shared memory goes away.
+    if (threadIdx.x == 0 && *abort_flag) {
+        const int issued = *s_issued;
+        const uint64_t start = ptx::globaltimer();
+        for (int i = max(0, issued - kDecStages); i < issued; ++i)
+            while (!ptx::mbar_try_wait(full(i % kDecStages), (i / kDecStages) & 1) &&
+                   ptx::globaltimer() - start < 4000000ull) {
+            }
+    }
+}
+
+// ============================================================================
+// d = 128: tensor-core form.  With keys on the M side of the MMA the few query
+// rows become N = 16 (rows padded):
+//     S^T [128 keys x 16] = K [128 x d] . Q^T          (A = K tile, B = Q; K-major)
+//     O^T [d x 16]       += V^T [d x 128 keys] . P^T   (A = V tile, MN-major; B = P^T, K-major)
+// both accumulated in TMEM (lane = key for S^T, lane = d-column for O^T), so a
+// softmax thread owns one key and touches only its RB valid row values per
+// 128-key tile.  Roles (224 threads):
+//   warps 0-3  softmax: thread t = key t of the tile (TMEM lane t); masks,
+//              exp2 against a per-row reference, P^T (bf16) to shared memory,
+//              per-thread partial row sums; epilogue (thread t = d-column t).
+//   warp 4     K producer: TMA boxes of K into a 3-stage ring of 128-key tiles;
+//              a K stage is free again as soon as its S^T MMA completes.
+//   warp 6     V producer: the same for V; a V stage frees after O^T += V^T P^T.
+//              Separate rings give the loads a longer lead than one K+V stage
+//              held until the last MMA on it.
+//   warp 5     MMA: TMEM allocation; one thread issues S^T(j+1) before
+//              O^T += V^T P^T(j), so a tile's softmax overlaps the next scores.
+// The row reference m is the first tile's max (log2 units) and only moves
+// when a tile's weight would pass 2^64 (or a row saw no key yet); then the
+// tile max is taken and O^T and the partial sums are rescaled in place.
+constexpr int kTcKeys = 128;
+constexpr int kTcStages = 3;
+constexpr int kTcThreads = 224;
+constexpr int kBarSoftmax = 2;                     // named barrier of the softmax warps
+constexpr float kTcWeightLimit = 1.8446744e19f;    // 2^64
+
+template <int RB>
+struct TcCfg {
+    static constexpr int kRegionBytes = kTcKeys * 128;      // 128 keys x 64 columns (bf16), 128-byte swizzle
+    static constexpr int kTileBytes = 2 * kRegionBytes;     // one K or V tile
+    static constexpr int kOffV = kTcStages * kTileBytes;    // K ring, then V ring
+    static constexpr int kOffQ = 2 * kTcStages * kTileBytes;  // Q [16 rows][128] bf16: 2 regions x 2 KB
+    static constexpr int kOffP = kOffQ + 4096;              // P^T x2: [16 rows][128 keys] bf16, 2 regions x 2 KB each
+    static constexpr int kOffRed = kOffP + 2 * 4096;        // float [4 warps][16]
+    static constexpr int kOffBar = kOffRed + 4 * 16 * 4;
+    // k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_full[2], o_done[2], o_final, mma_drain
+    static constexpr int kNumBars = 4 * kTcStages + 8;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort, ticket, K / V tiles issued
+    static constexpr int kSmem = kOffMisc + 32;
+    static constexpr int kDynSmem = kSmem + 1024;
+    static constexpr uint32_t kTmemCols = 64;               // S^T buffers at 0 and 16, O^T at 32
+    static_assert(kDynSmem <= 232448, "shared memory budget");
+    static_assert(RB == 4 || RB == 8 || RB == 16, "row capacity");
+};
+
+template <int RB>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    decode_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                     const __grid_constant__ DecodeParams p)
+{
+    using C = TcCfg<RB>;
+    constexpr int HD = 128;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    int si = 0;
+    while (si + 1 < p.n_seqs && static_cast<int>(blockIdx.x) >= p.seqs[si + 1].cta0) ++si;
+    const DecodeSeq &sq = p.seqs[si];
+    const int local = static_cast<int>(blockIdx.x) - sq.cta0;
+    const int kvh = local / sq.n_splits;
+    const int split = local - kvh * sq.n_splits;
+    const int g = p.group;
+    const int n_rows = sq.n_q * g;
+    const int n_tiles_all = (sq.n_keys + kTcKeys - 1) / kTcKeys;
+    const int t0 = split * p.split_tiles;
+    const int nt = max(0, min(t0 + p.split_tiles, n_tiles_all) - t0);
+    const int qpos0 = sq.n_keys - sq.n_q;
+
+    const uint32_t sbase = ptx::smem_addr(smem);
+    const uint32_t q_smem = sbase + C::kOffQ;
+    const uint32_t p_smem = sbase + C::kOffP;
+    float *s_red = reinterpret_cast<float *>(smem + C::kOffRed);
+    const uint32_t bar0 = sbase + C::kOffBar;
+    auto k_full = [&](int s) { return bar0 + 8u * s; };
+    auto k_empty = [&](int s) { return bar0 + 8u * (kTcStages + s); };
+    auto v_full = [&](int s) { return bar0 + 8u * (2 * kTcStages + s); };
+    auto v_empty = [&](int s) { return bar0 + 8u * (3 * kTcStages + s); };
+    const uint32_t b_s_full = bar0 + 8u * (4 * kTcStages);      // [2]
+    const uint32_t b_p_full = b_s_full + 16;                     // [2]
+    const uint32_t b_o_done = b_p_full + 16;                     // [2]
+    const uint32_t b_o_final = b_o_done + 16;
+    const uint32_t b_drain = b_o_final + 8;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 4);
+    int *s_ticket = reinterpret_cast<int *>(smem + C::kOffMisc + 8);
+    volatile int *s_issued = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 12);  // [2]: K, V
+    const WaitCtx wctx{abort_flag, p.status};
+
+    if (threadIdx.x == 128) {  // K producer warp, lane 0
+        for (int s = 0; s < kTcStages; ++s) {
+            ptx::mbar_init(k_full(s), 1);
+            ptx::mbar_init(k_empty(s), 1);
+            ptx::mbar_init(v_full(s), 1);
+            ptx::mbar_init(v_empty(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(b_s_full + 8 * b, 1);
+            ptx::mbar_init(b_p_full + 8 * b, 128);
+            ptx::mbar_init(b_o_done + 8 * b, 1);
+        }
+        ptx::mbar_init(b_o_final, 1);
+        ptx::mbar_init(b_drain, 1);
+        *abort_flag = 0;
+        s_issued[0] = 0;
+        s_issued[1] = 0;
+        ptx::fence_barrier_init();
+        ptx::prefetch_tensormap(&tm_k);
+        ptx::prefetch_tensormap(&tm_v);
+    }
+    if (warp == 5) {
+        ptx::tmem_alloc(ptx::smem_addr(tmem_slot), C::kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp < 4) {
+        // Q rows of this kv-head into [16 rows][128] bf16, 128-byte swizzle; rows past n_q x g are zero
+        for (int e = threadIdx.x; e < 16 * 16; e += 128) {
+            const int r = e >> 4;
+            const int c = e & 15;  // 16-byte chunk along d
+            uint4 v = make_uint4(0u, 0u, 0u, 0u);
+            if (r < n_rows)
+                v = *reinterpret_cast<const uint4 *>(
+                    static_cast<const __nv_bfloat16 *>(p.q) +
+                    (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD + c * 8);
+            *reinterpret_cast<uint4 *>(smem + C::kOffQ + (c >> 3) * 2048 + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
+        }
+        // both P^T buffers start at zero (rows past RB stay zero)
+        for (int e = threadIdx.x; e < 2 * 4096 / 16; e += 128)
+            reinterpret_cast<uint4 *>(smem + C::kOffP)[e] = make_uint4(0u, 0u, 0u, 0u);
+        ptx::fence_proxy_async_smem();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const uint32_t t_s = tmem;         // S^T buffers: columns 0 and 16
+    const uint32_t t_o = tmem + 32;    // O^T: columns 32..47
+
+    if (warp == 4 || warp == 6) {
+        // ============================================================ producers (warp 4: K, warp 6: V)
+        const bool is_v = warp == 6;
+        const CUtensorMap *map = is_v ? &tm_v : &tm_k;
+        const int kpc = p.ps < kDecKeys ? p.ps : kDecKeys;  // keys per box (<= 64)
+        const int n_ops = (kTcKeys / kpc) * 2;              // boxes per tile, <= 32
+        const int op_slot = lane >> 1;
+        const int op_reg = lane & 1;
+        const bool op_on = lane < n_ops;
+        auto page_of = [&](int t) -> int {
+            const int key0 = t * kTcKeys + op_slot * kpc;
+            if (!op_on || key0 >= sq.n_keys) return -1;
+            const int pg = p.page_table[sq.table_row + key0 / p.ps];
+            if (pg < 0 || pg >= p.num_pages) {
+                atomicCAS(p.status, 0, kStatusBadPage);
+                return -1;
+            }
+            return pg;
+        };
+        int page_next = nt > 0 ? page_of(t0) : -1;
+        for (int i = 0; i < nt; ++i) {
+            const int t = t0 + i;
+            const int s = i % kTcStages;
+            const int page = page_next;
+            if (i + 1 < nt) page_next = page_of(t + 1);
+            const uint32_t b_empty = is_v ? v_empty(s) : k_empty(s);
+            const uint32_t b_full = is_v ? v_full(s) : k_full(s);
+            if (i >= kTcStages && !wait_bar_warp(b_empty, ((i / kTcStages) - 1) & 1, wctx)) break;
+            if (lane == 0) ptx::mbar_arrive_expect_tx(b_full, C::kTileBytes);
+            __syncwarp();
+            if (op_on) {
+                const int key0 = t * kTcKeys + op_slot * kpc;
+                const int y = page >= 0
+                                  ? ((p.layer * p.num_pages + page) * p.hkv + kvh) * p.ps + (key0 % p.ps)
+                                  : p.oob_row;
+                const uint32_t dst = sbase + (is_v ? C::kOffV : 0) + s * C::kTileBytes + op_reg * C::kRegionBytes +
+                                     op_slot * kpc * 128;
+                ptx::tma_load_2d(dst, map, op_reg * 64, y, b_full);
+            }
+            __syncwarp();
+            if (lane == 0) s_issued[is_v ? 1 : 0] = i + 1;
+        }
+    } else if (warp == 5) {
+        // ============================================================ MMA issuer
+        if (lane == 0 && nt > 0) {
+            constexpr uint32_t kIdS = ptx::idesc_bf16_f32(128, 16, false, false);
+            constexpr uint32_t kIdPV = ptx::idesc_bf16_f32(128, 16, false, true);
+            auto issue_s = [&](int j) -> bool {
+                const int s = j % kTcStages;
+                if (!wait_bar(k_full(s), (j / kTcStages) & 1, wctx)) return false;
+                ptx::tc_fence_after();
+                const uint32_t ka = sbase + s * C::kTileBytes;
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint32_t off = (kk >> 2) * C::kRegionBytes + (kk & 3) * 32;
+                    const uint32_t qoff = (kk >> 2) * 2048 + (kk & 3) * 32;
+                    ptx::mma_bf16(t_s + 16 * (j & 1), ptx::smem_desc_sw128(ka + off, 16, 1024),
+                                  ptx::smem_desc_sw128(q_smem + qoff, 16, 1024), kIdS, kk > 0 ? 1u : 0u);
+                }
+                ptx::mma_commit(b_s_full + 8 * (j & 1));
+                ptx::mma_commit(k_empty(s));  // the K stage is free once S^T(j) is done
+                return true;
+            };
+            bool ok = issue_s(0);
+            for (int j = 0; ok && j < nt; ++j) {
+                if (j + 1 < nt && !issue_s(j + 1)) break;
+                if (!wait_bar(v_full(j % kTcStages), (j / kTcStages) & 1, wctx)) break;
+                if (!wait_bar(b_p_full + 8 * (j & 1), (j >> 1) & 1, wctx)) break;
+                ptx::tc_fence_after();
+                const uint32_t vb = sbase + C::kOffV + (j % kTcStages) * C::kTileBytes;
+                const uint32_t pb = p_smem + (j & 1) * 4096;
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    ptx::mma_bf16(t_o, ptx::smem_desc_sw128(vb + kk * 16 * 128, C::kRegionBytes, 1024),
+                                  ptx::smem_desc_sw128(pb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024), kIdPV,
+                                  (j > 0 || kk > 0) ? 1u : 0u);
+                }
+                ptx::mma_commit(v_empty(j % kTcStages));
+                ptx::mma_commit(b_o_done + 8 * (j & 1));
+            }
+            ptx::mma_commit(b_o_final);
+        }
+        // every tcgen05 op of this CTA completes before TMEM is released
+        if (lane == 0) {
+            ptx::mma_commit(b_drain);
+            const uint64_t start = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(b_drain, 0) && ptx::globaltimer() - start < 4000000ull) {
+            }
+        }
+        __syncwarp();
+    } else {
+        // ============================================================ softmax (thread = key of the tile)
+        const int t = threadIdx.x;              // TMEM lane
+        const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+        float mref[RB], lpart[RB];
+#pragma unroll
+        for (int r = 0; r < RB; ++r) {
+            mref[r] = -INFINITY;
+            lpart[r] = 0.f;
+        }
+        // row maxima over the tile's 128 keys, for every row (all softmax threads take part)
+        auto tile_max = [&](const float (&x)[RB], float (&m)[RB]) {
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                float v = x[r];
+#pragma unroll
+                for (int off = 16; off >= 1; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+                if (lane == 0) s_red[warp * 16 + r] = v;
+            }
+            ptx::bar_sync(kBarSoftmax, 128);
+#pragma unroll
+            for (int r = 0; r < RB; ++r)
+                m[r] = fmaxf(fmaxf(s_red[r], s_red[16 + r]), fmaxf(s_red[32 + r], s_red[48 + r]));
+            ptx::bar_sync(kBarSoftmax, 128);  // s_red is reused
+        };
+        bool stopped = false;
+        for (int j = 0; j < nt; ++j) {
+            const bool ok = wait_bar_warp(b_s_full + 8 * (j & 1), (j >> 1) & 1, wctx);
+            if (ptx::bar_sync_or(kBarSoftmax, 128, !ok || *abort_flag)) {
+                stopped = true;
+                break;
+            }
+            ptx::tc_fence_after();
+            float x[RB];
+            ptx::tmem_ld_n<RB>(t_s + 16 * (j & 1) + lane_off, x);
+            ptx::tmem_wait_ld();
+            const int key = (t0 + j) * kTcKeys + t;
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                const int qpos = r < n_rows ? qpos0 + r / g : sq.n_keys - 1;
+                x[r] = (key < sq.n_keys && key <= qpos) ? x[r] * p.scale_log2 : -INFINITY;
+            }
+            if (j == 0) tile_max(x, mref);
+            float pr[RB];
+            bool big = false;
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                pr[r] = mref[r] == -INFINITY ? (x[r] == -INFINITY ? 0.f : INFINITY) : ex2(x[r] - mref[r]);
+                big = big || !(pr[r] <= kTcWeightLimit);
+            }
+            if (ptx::bar_sync_or(kBarSoftmax, 128, big)) {
+                // rare: move the reference to the running max, rescale O^T and the partial sums
+                float tm[RB], f[RB];
+                tile_max(x, tm);
+#pragma unroll
+                for (int r = 0; r < RB; ++r) {
+                    const float mn = fmaxf(mref[r], tm[r]);
+                    f[r] = mn == -INFINITY ? 1.f : ex2(mref[r] - mn);
+                    mref[r] = mn;
+                    lpart[r] *= f[r];
+                    pr[r] = mn == -INFINITY ? 0.f : ex2(x[r] - mn);
+                }
+                if (j > 0) {  // every earlier O^T update has landed
+                    const bool done = wait_bar_warp(b_o_done + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wctx);
+                    if (done) {
+                        ptx::tc_fence_after();
+                        float o[RB];
+                        ptx::tmem_ld_n<RB>(t_o + lane_off, o);
+                        ptx::tmem_wait_ld();
+#pragma unroll
+                        for (int r = 0; r < RB; ++r) o[r] *= f[r];
+                        ptx::tmem_st_n<RB>(t_o + lane_off, o);
+                        ptx::tmem_wait_st();
+                    }
+                }
+            }
+#pragma unroll
+            for (int r = 0; r < RB; ++r) lpart[r] += pr[r];
+            // P^T(j) into buffer j & 1 once O^T += V^T P^T(j - 2) has read it
+            if (j >= 2 && !wait_bar_warp(b_o_done + 8 * (j & 1), ((j - 2) >> 1) & 1, wctx)) {
+                stopped = true;  // the other softmax warps see the abort flag at the next tile
+            }
+            uint8_t *pt = smem + C::kOffP + (j & 1) * 4096 + (t >> 6) * 2048;
+            const int chunk = (t & 63) >> 3;
+#pragma unroll
+            for (int r = 0; r < RB; ++r)
+                *reinterpret_cast<__nv_bfloat16 *>(pt + r * 128 + ((chunk ^ (r & 7)) << 4) + (t & 7) * 2) =
+                    __float2bfloat16_rn(pr[r]);
+            ptx::fence_proxy_async_smem();
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(b_p_full + 8 * (j & 1));
+        }
+
+        // ---------------------------------------------------------- epilogue (thread t = d-column t)
+        float o[RB];
+#pragma unroll
+        for (int r = 0; r < RB; ++r) o[r] = 0.f;
+        if (!stopped && nt > 0) {
+            if (wait_bar_warp(b_o_final, 0, wctx)) {
+                ptx::tc_fence_after();
+                ptx::tmem_ld_n<RB>(t_o + lane_off, o);
+                ptx::tmem_wait_ld();
+            }
+        }
+        // row sums over the 128 key lanes
+        float lsum[RB];
+#pragma unroll
+        for (int r = 0; r < RB; ++r) {
+            float v = lpart[r];
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+            if (lane == 0) s_red[warp * 16 + r] = v;
+        }
+        ptx::bar_sync(kBarSoftmax, 128);
+#pragma unroll
+        for (int r = 0; r < RB; ++r) lsum[r] = (s_red[r] + s_red[16 + r]) + (s_red[32 + r] + s_red[48 + r]);
+        const bool single = sq.n_splits == 1;
+        if (single) {
+            if (!stopped) {
+#pragma unroll
+                for (int r = 0; r < RB; ++r) {
+                    if (r < n_rows) {
+                        const float inv = lsum[r] > 0.f ? 1.0f / lsum[r] : 0.f;
+                        static_cast<__nv_bfloat16 *>(p.out)[(static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g +
+                                                             r % g) * HD + t] = __float2bfloat16_rn(o[r] * inv);
+                    }
+                }
+            }
+        } else {
+            float *po = p.part + static_cast<int64_t>(blockIdx.x) * RB * HD;
+            float *pm = p.part + static_cast<int64_t>(p.total_ctas) * RB * HD;
+            float *pl = pm + static_cast<int64_t>(p.total_ctas) * RB;
+#pragma unroll
+            for (int r = 0; r < RB; ++r) po[r * HD + t] = o[r];
+            if (t < RB) {
+                float mv = -INFINITY, lv = 0.f;
+#pragma unroll
+                for (int r = 0; r < RB; ++r)
+                    if (r == t) {
+                        mv = mref[r];
+                        lv = lsum[r];
+                    }
+                pm[static_cast<int64_t>(blockIdx.x) * RB + t] = mv;
+                pl[static_cast<int64_t>(blockIdx.x) * RB + t] = lv;
+            }
+            split_merge<RB, HD>(p, sq, si, kvh, n_rows, t, 128, kBarSoftmax, s_ticket);
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (threadIdx.x == 0 && *abort_flag) {
+        // after an abort, copies may still be in flight: bounded wait for the last ones issued
+        const uint64_t start = ptx::globaltimer();
+        for (int ring = 0; ring < 2; ++ring) {
+            const int issued = s_issued[ring];
+            for (int i = max(0, issued - kTcStages); i < issued; ++i) {
+                const uint32_t b = ring ? v_full(i % kTcStages) : k_full(i % kTcStages);
+                while (!ptx::mbar_try_wait(b, (i / kTcStages) & 1) && ptx::globaltimer() - start < 4000000ull) {
+                }
+            }
+        }
+    }
+    if (warp == 5) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+template <int RB>
+cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st)
+{
+    using C = TcCfg<RB>;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e =
+            cudaFuncSetAttribute(decode_tc_kernel<RB>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kDynSmem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    decode_tc_kernel<RB><<<p.total_ctas, kTcThreads, C::kDynSmem, st>>>(tm_k, tm_v, p);
+    return cudaGetLastError();
+}
+
+template <int HD, int RB>
+cudaError_t launch_t(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st)
+{
+    using C = DecCfg<HD, RB>;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(decode_attn_kernel<HD, RB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             C::kDynSmem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    decode_attn_kernel<HD, RB><<<p.total_ctas, kDecThreads, C::kDynSmem, st>>>(tm_k, tm_v, p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_decode_attn(int head_dim, int rows_cap, bool tensor_core, const CUtensorMap &tm_k,
+                               const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st)
+{
+    if (p.total_ctas <= 0) return cudaSuccess;
+    if (tensor_core) {
+        if (head_dim != 128) return cudaErrorInvalidValue;
+        if (rows_cap == 4) return launch_tc<4>(tm_k, tm_v, p, st);
+        if (rows_cap == 8) return launch_tc<8>(tm_k, tm_v, p, st);
+        if (rows_cap == 16) return launch_tc<16>(tm_k, tm_v, p, st);
+        return cudaErrorInvalidValue;
+    }
+    if (head_dim == 128) {
+        if (rows_cap == 4) return launch_t<128, 4>(tm_k, tm_v, p, st);
+        if (rows_cap == 8) return launch_t<128, 8>(tm_k, tm_v, p, st);
+        if (rows_cap == 16) return launch_t<128, 16>(tm_k, tm_v, p, st);
+    } else if (head_dim == 64) {
+        if (rows_cap == 4) return launch_t<64, 4>(tm_k, tm_v, p, st);
+        if (rows_cap == 8) return launch_t<64, 8>(tm_k, tm_v, p, st);
+        if (rows_cap == 16) return launch_t<64, 16>(tm_k, tm_v, p, st);
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace pe

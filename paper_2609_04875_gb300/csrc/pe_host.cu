@@ -90,10 +90,12 @@ struct pe_cache {
     int32_t *d_status = nullptr;
     float *d_ws = nullptr;
     int64_t ws_bytes = 0;
+    int32_t *d_tickets = nullptr;  // decode split merge: one counter per (sequence, kv-head) of a launch
     int64_t pool_rows = 0;  // L * num_pages * Hkv * ps
-    CUtensorMap tm_k{}, tm_v{};
+    CUtensorMap tm_k{}, tm_v{};    // tensor-core kernel: 64 x ps boxes
+    CUtensorMap tm_kd{}, tm_vd{};  // decode kernel: 64 x min(ps, 64) boxes
     // options
-    int splitkv = -1, num_splits = 0, debug_poison = 0;
+    int splitkv = -1, num_splits = 0, debug_poison = 0, decode_kernel = 1;
     int64_t launches = 0;
     int32_t last_split = 0, last_splits = 0, last_ctas = 0;  // plan of the last attention launch
 };
@@ -150,7 +152,9 @@ void free_device(pe_cache *c)
     if (c->d_len) cudaFree(c->d_len);
     if (c->d_status) cudaFree(c->d_status);
     if (c->d_ws) cudaFree(c->d_ws);
+    if (c->d_tickets) cudaFree(c->d_tickets);
     c->k_pool = c->v_pool = nullptr;
+    c->d_tickets = nullptr;
     c->d_table = nullptr;
     c->d_len = nullptr;
     c->d_status = nullptr;
@@ -405,6 +409,94 @@ struct AttnItem {
     int32_t n_q;
 };
 
+// Decode kernel launches (groups of kMaxSegs sequences).  Key splits: about two
+// waves of the CTAs that fit on the GPU at once, at least 2 tiles per split;
+// "splitkv" = 0 keeps one split, "num_splits" fixes the count.
+pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t layer, const void *Q, void *out,
+                     int32_t hq, float scale, cudaStream_t st)
+{
+    const pe_cache_config &cf = c->cfg;
+    const int hkv = cf.num_kv_heads;
+    const int d = cf.head_dim;
+    const int g = hq / hkv;
+    // d = 128: tensor-core form (128-key tiles, one CTA per SM); otherwise CUDA cores (64-key tiles, two per SM)
+    const bool tc = d == 128 && c->decode_kernel == 1;
+    const int64_t tile_keys = tc ? 128 : kDecKeys;
+    std::vector<char> pbuf(sizeof(DecodeParams));
+    DecodeParams &p = *reinterpret_cast<DecodeParams *>(pbuf.data());
+    for (size_t lo = 0; lo < items.size(); lo += kMaxSegs) {
+        const size_t hi = std::min(items.size(), lo + kMaxSegs);
+        int64_t max_rows = 1, work = 0, max_tiles = 1;
+        for (size_t i = lo; i < hi; ++i) {
+            const int64_t tiles = ceil_div(c->len[items[i].seq], tile_keys);
+            max_rows = std::max<int64_t>(max_rows, static_cast<int64_t>(items[i].n_q) * g);
+            max_tiles = std::max(max_tiles, tiles);
+            work += tiles * hkv;
+        }
+        const int rb = max_rows <= 4 ? 4 : (max_rows <= 8 ? 8 : 16);
+        const int64_t resident = static_cast<int64_t>(c->num_sms) * (!tc && rb <= 8 ? 2 : 1);
+        auto ctas_for = [&](int64_t stile) {
+            int64_t n = 0;
+            for (size_t i = lo; i < hi; ++i) n += ceil_div(ceil_div(c->len[items[i].seq], tile_keys), stile) * hkv;
+            return n;
+        };
+        // about two waves of resident CTAs, never a third one started by a few stragglers
+        int64_t split_tiles = std::max<int64_t>(2, ceil_div(work, 2 * resident));
+        while (split_tiles < max_tiles && ctas_for(split_tiles) > 2 * resident) ++split_tiles;
+        if (c->splitkv == 0) split_tiles = max_tiles;
+        if (c->splitkv != 0 && c->num_splits > 0) split_tiles = std::max<int64_t>(1, ceil_div(max_tiles, c->num_splits));
+        if (c->splitkv == 1 && c->num_splits == 0 && split_tiles >= max_tiles && max_tiles > 1)
+            split_tiles = ceil_div(max_tiles, 2);
+        split_tiles = std::min(split_tiles, max_tiles);
+        for (;;) {
+            std::memset(&p, 0, sizeof p);
+            int32_t cta = 0;
+            bool any_split = false;
+            for (size_t i = lo; i < hi; ++i) {
+                const AttnItem &it = items[i];
+                DecodeSeq &q = p.seqs[p.n_seqs++];
+                q.table_row = it.seq * cf.max_pages_per_seq;
+                q.n_pages = static_cast<int32_t>(c->table[it.seq].size());
+                q.q_row0 = it.q_row0;
+                q.n_q = it.n_q;
+                q.n_keys = static_cast<int32_t>(c->len[it.seq]);
+                q.n_splits = static_cast<int32_t>(ceil_div(ceil_div(c->len[it.seq], tile_keys), split_tiles));
+                q.cta0 = cta;
+                cta += q.n_splits * hkv;
+                any_split = any_split || q.n_splits > 1;
+            }
+            p.total_ctas = cta;
+            const int64_t need = static_cast<int64_t>(cta) * rb * (d + 2) * 4;
+            if (!any_split || need <= c->ws_bytes) break;
+            split_tiles *= 2;  // partials do not fit the workspace: fewer splits
+        }
+        p.page_table = c->d_table;
+        p.q = Q;
+        p.out = out;
+        p.k_pool = c->k_pool;
+        p.v_pool = c->v_pool;
+        p.part = c->d_ws;
+        p.tickets = c->d_tickets;
+        p.status = c->d_status;
+        p.hq = hq;
+        p.hkv = hkv;
+        p.group = g;
+        p.layer = layer;
+        p.num_pages = cf.num_pages;
+        p.ps = cf.page_size;
+        p.oob_row = static_cast<int32_t>(c->pool_rows);
+        p.split_tiles = static_cast<int32_t>(split_tiles);
+        p.scale_log2 = scale * 1.4426950408889634f;
+        c->last_split = p.seqs[0].n_splits > 1 ? 1 : 0;
+        c->last_splits = p.seqs[0].n_splits;
+        c->last_ctas = p.total_ctas;
+        cudaError_t e = launch_decode_attn(d, rb, tc, c->tm_kd, c->tm_vd, p, st);
+        if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
+        c->launches++;
+    }
+    return PE_OK;
+}
+
 pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t layer, const void *Q,
                         int64_t q_rows, void *out, int32_t hq, float scale, cudaStream_t st)
 {
@@ -413,10 +505,20 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     const int d = cf.head_dim;
     const int g = hq / hkv;
     const int bmq = kBM / g;
-    // heaviest sequences first (more key tiles per q-tile)
-    std::vector<AttnItem> order;
-    for (const AttnItem &it : items)
-        if (it.n_q > 0) order.push_back(it);
+    // Items whose queries pack into at most kDecMaxRows rows per kv-head take
+    // the decode kernel; the rest the tensor-core kernel.
+    std::vector<AttnItem> order, dec;
+    for (const AttnItem &it : items) {
+        if (it.n_q <= 0) continue;
+        if (c->decode_kernel && static_cast<int64_t>(it.n_q) * g <= kDecMaxRows && (d == 64 || d == 128))
+            dec.push_back(it);
+        else
+            order.push_back(it);
+    }
+    if (!dec.empty()) {
+        pe_status s = run_decode(c, dec, layer, Q, out, hq, scale, st);
+        if (s != PE_OK) return s;
+    }
     std::stable_sort(order.begin(), order.end(), [&](const AttnItem &a, const AttnItem &b) {
         return c->len[a.seq] > c->len[b.seq];
     });
@@ -658,8 +760,14 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
         if ((e = cudaMalloc(&cc->d_status, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
         if ((e = cudaMemset(cc->d_status, 0, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
         if ((e = cudaMalloc(&cc->d_ws, cc->ws_bytes)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc workspace"); break; }
+        const size_t tickets = sizeof(int32_t) * kMaxSegs * c.num_kv_heads;
+        if ((e = cudaMalloc(&cc->d_tickets, tickets)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
+        if ((e = cudaMemset(cc->d_tickets, 0, tickets)) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
         if ((st = encode_2d(&cc->tm_k, cc->k_pool, c.head_dim, pool_rows, 64, ps)) != PE_OK) break;
         if ((st = encode_2d(&cc->tm_v, cc->v_pool, c.head_dim, pool_rows, 64, ps)) != PE_OK) break;
+        const uint32_t dec_rows = ps < kDecKeys ? ps : kDecKeys;
+        if ((st = encode_2d(&cc->tm_kd, cc->k_pool, c.head_dim, pool_rows, 64, dec_rows)) != PE_OK) break;
+        if ((st = encode_2d(&cc->tm_vd, cc->v_pool, c.head_dim, pool_rows, 64, dec_rows)) != PE_OK) break;
         if ((e = cudaDeviceSynchronize()) != cudaSuccess) { st = cuda_fail(e, "create sync"); break; }
     } while (false);
     if (st != PE_OK) {
@@ -1128,6 +1236,9 @@ pe_status pe_set_option(pe_cache *c, const char *key, int64_t value)
         c->num_splits = static_cast<int>(value);
     } else if (!std::strcmp(key, "debug_poison")) {
         c->debug_poison = value ? 1 : 0;
+    } else if (!std::strcmp(key, "decode_kernel")) {
+        if (value < 0 || value > 2) return fail(PE_ERR_INVALID, "decode_kernel must be 0, 1 or 2");
+        c->decode_kernel = static_cast<int>(value);
     } else {
         return fail(PE_ERR_INVALID, "unknown option '%s'", key);
     }

@@ -97,6 +97,41 @@ struct AttnParams {
     AttnSeq seqs[kMaxSegs];
 };
 
+// ---------------------------------------------------------------- decode attention
+// Sequences whose queries pack into at most kDecMaxRows rows per kv-head
+// (n_q x group) take the decode kernel (pe_decode.cu): CUDA cores, 64-key
+// tiles streamed by bulk copies, split-KV merged in-kernel by the last split.
+constexpr int kDecMaxRows = 16;
+constexpr int kDecKeys = 64;           // keys per decode tile
+
+struct DecodeSeq {
+    int32_t table_row;     // seq * max_pages_per_seq
+    int32_t n_pages;
+    int32_t q_row0;        // first row of this sequence in Q / out
+    int32_t n_q;
+    int32_t n_keys;        // len
+    int32_t cta0;          // first CTA of this sequence: hkv x n_splits CTAs, kv-head major
+    int32_t n_splits;
+    int32_t pad_;
+};
+
+struct DecodeParams {
+    const int32_t *page_table;
+    const void *q;         // bf16 [rows][Hq][d]
+    void *out;             // bf16 [rows][Hq][d]
+    const void *k_pool;    // bf16 [L][num_pages][Hkv][ps][d]
+    const void *v_pool;
+    float *part;           // split partials: O [ctas][RB][d], then m [ctas][RB], then l [ctas][RB]
+    int32_t *tickets;      // one counter per (sequence, kv-head) of the launch; zero between launches
+    int32_t *status;
+    int32_t n_seqs, hq, hkv, group, layer, num_pages, ps;
+    int32_t oob_row;       // a pool row past the end: boxes there read zeros
+    int32_t split_tiles;   // decode tiles per split
+    int32_t total_ctas;
+    float scale_log2;      // softmax_scale * log2(e)
+    DecodeSeq seqs[kMaxSegs];
+};
+
 // Records `msg` as this thread's last error (pe_last_error) and returns code.
 int32_t report_error(int32_t code, const char *msg);
 
@@ -115,6 +150,12 @@ cudaError_t launch_cow_copy(uint4 *k_pool, uint4 *v_pool, int32_t src, int32_t d
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
                                const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);
+// rows_cap: 4, 8 or 16 (every sequence's n_q x group fits).
+// tm_k / tm_v: the pools as 2-D maps {d, L*num_pages*Hkv*ps} with 64 x min(ps, 64) boxes, 128-byte swizzle.
+// tensor_core (d = 128 only): keys on the MMA's M side, 128-key tiles (split_tiles
+// counts 128-key tiles); otherwise CUDA cores, 64-key tiles.
+cudaError_t launch_decode_attn(int head_dim, int rows_cap, bool tensor_core, const CUtensorMap &tm_k,
+                               const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st);
 cudaError_t launch_bounded_wait_selftest(int32_t *status, uint64_t limit_ns, cudaStream_t st);
 
 // Fixed split-KV scratch compiled into the library (pe_attn.cu), used only by

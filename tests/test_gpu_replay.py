@@ -134,12 +134,16 @@ def test_splitkv_many_splits():
     assert_close(out, oracle.replay_attention(pair.orc, s, 0, q, 1 / math.sqrt(d)), "37 splits")
 
 
-def test_splice_theorem_bitwise():
+@pytest.mark.parametrize("decode_kernel", [0, 1])
+def test_splice_theorem_bitwise(decode_kernel):
     """Theorem 1 on the GPU: crop to tau-1 + replay of the sanitized suffix equals
     a from-scratch pass over the counterfactual sequence, bit for bit (key tiles
-    are keyed to logical positions, not to physical pages)."""
+    are keyed to logical positions, not to physical pages).  With the decode
+    kernel on, a one-position suffix takes it on both sides (the from-scratch
+    side attends that position alone); off, every call takes the tensor-core
+    kernel and the from-scratch side attends every position."""
     L, hq, hkv, d, ps = 1, 32, 8, 128, 16
-    for (T, tau) in [(700, 301), (1000, 1), (513, 513), (2049, 1000)]:
+    for (T, tau) in [(700, 301), (1000, 1), (513, 513), (2049, 1000), (4100, 4100)]:
         P, S = tau - 1, T - tau + 1
         g = synth.rng(tau, 5)
         k0 = synth.normal_bf16(g, (L, T, hkv, d))
@@ -152,6 +156,7 @@ def test_splice_theorem_bitwise():
         npg = -(-T // ps) + 2
         a = pe.PagedKVCache(L, hkv, d, ps, npg, 1, npg, init_free_order=synth.page_permutation(1, npg))
         a.set_option("splitkv", 0)
+        a.set_option("decode_kernel", decode_kernel)
         sa = a.seq_create()
         a.append_kv(sa, dev(k0), dev(v0))
         a.crop(sa, tau)
@@ -159,11 +164,17 @@ def test_splice_theorem_bitwise():
         rep = a.replay_attn(sa, 0, dev(qc[0]))
         b = pe.PagedKVCache(L, hkv, d, ps, npg, 1, npg, init_free_order=synth.page_permutation(2, npg))
         b.set_option("splitkv", 0)
+        b.set_option("decode_kernel", decode_kernel)
         sb = b.seq_create()
         b.append_kv(sb, dev(np.concatenate([k0[:, :P], kc], 1)), dev(np.concatenate([v0[:, :P], vc], 1)))
-        full = b.replay_attn(sb, 0, dev(np.concatenate([qp[0], qc[0]], 0)))
-        torch.cuda.synchronize()
-        assert torch.equal(rep, full[P:]), f"T={T} tau={tau}: splice differs"
+        if decode_kernel and S * (hq // hkv) <= 16:
+            full = b.replay_attn(sb, 0, dev(qc[0]))
+            torch.cuda.synchronize()
+            assert torch.equal(rep, full), f"T={T} tau={tau}: splice differs (decode kernel)"
+        else:
+            full = b.replay_attn(sb, 0, dev(np.concatenate([qp[0], qc[0]], 0)))
+            torch.cuda.synchronize()
+            assert torch.equal(rep, full[P:]), f"T={T} tau={tau}: splice differs"
         assert a.seq_info(sa) == (T, S)
 
 
