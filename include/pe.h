@@ -255,7 +255,9 @@ pe_status pe_set_option(pe_cache *cache, const char *key, int64_t value);
 /* Synchronises `stream` and reads the device status word.  *code = 0 when no
  * kernel reported a problem, else the first recorded code (1 = a bounded
  * wait ran out; 2 = the decode kernel met a page id outside the pool and
- * skipped it).  clear != 0 resets it.  Returns DEVICE_TIMEOUT if *code != 0. */
+ * skipped it).  clear != 0 resets it, and after a nonzero code also the decode
+ * kernel's split-merge and scheduling counters.  Returns DEVICE_TIMEOUT if
+ * *code != 0. */
 pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *stream);
 
 /* Failure-detection self-test: launches one kernel whose single wait (the same

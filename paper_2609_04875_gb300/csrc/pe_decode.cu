@@ -187,15 +187,11 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
         const int op_slot = lane / C::kRegions;             // this lane's page slot in the tile
         const int op_reg = lane % C::kRegions;              // and 64-column half
         const bool op_on = lane < n_ops;
-        auto page_of = [&](int t) -> int {  // this lane's page of tile t, -1 past the sequence
+        // this lane's raw page id of tile t (checked where it is used), -1 past the sequence
+        auto page_of = [&](int t) -> int {
             const int key0 = t * kDecKeys + op_slot * kpc;
             if (!op_on || key0 >= sq.n_keys) return -1;
-            const int pg = p.page_table[sq.table_row + key0 / p.ps];
-            if (pg < 0 || pg >= p.num_pages) {
-                atomicCAS(p.status, 0, kStatusBadPage);
-                return -1;
-            }
-            return pg;
+            return p.page_table[sq.table_row + key0 / p.ps];
         };
         int page_next = nt > 0 ? page_of(t0) : -1;
         for (int i = 0; i < nt; ++i) {
@@ -208,9 +204,10 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
             __syncwarp();
             if (op_on) {
                 const int key0 = t * kDecKeys + op_slot * kpc;
-                const int y = page >= 0
-                                  ? ((p.layer * p.num_pages + page) * p.hkv + kvh) * p.ps + (key0 % p.ps)
-                                  : p.oob_row;  // past the sequence: zeros
+                const bool ok_page = page >= 0 && page < p.num_pages;
+                if (!ok_page && key0 < sq.n_keys) atomicCAS(p.status, 0, kStatusBadPage);
+                const int y = ok_page ? ((p.layer * p.num_pages + page) * p.hkv + kvh) * p.ps + (key0 % p.ps)
+                                      : p.oob_row;  // past the sequence (or a bad id): zeros
                 const uint32_t dst =
                     ptx::smem_addr(smem + s * C::kStageBytes) + op_reg * C::kRegionBytes + op_slot * kpc * 128;
                 ptx::tma_load_2d(dst, &tm_k, op_reg * 64, y, full(s));
@@ -449,23 +446,44 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 //     O^T [d x 16]       += V^T [d x 128 keys] . P^T   (A = V tile, MN-major; B = P^T, K-major)
 // both accumulated in TMEM (lane = key for S^T, lane = d-column for O^T), so a
 // softmax thread owns one key and touches only its RB valid row values per
-// 128-key tile.  Roles (224 threads):
+// 128-key tile.
+//
+// Persistent, dynamically scheduled: every (sequence, kv-head) item's 128-key
+// tiles are cut into chunks of at most 8 tiles (the host picks about three
+// chunks per SM); one CTA per SM takes chunk after chunk from a global
+// counter, so a slower SM simply takes fewer.  A chunk that is a whole item is written directly; otherwise
+// each chunk writes a partial (O, m, l) and the last of an item's chunks to
+// finish merges them (ticket counter), in chunk order.  The last CTA to exit
+// resets the chunk counter for the next launch.
+//
+// Roles (352 threads):
 //   warps 0-3  softmax: thread t = key t of the tile (TMEM lane t); masks,
 //              exp2 against a per-row reference, P^T (bf16) to shared memory,
-//              per-thread partial row sums; epilogue (thread t = d-column t).
-//   warp 4     K producer: TMA boxes of K into a 3-stage ring of 128-key tiles;
-//              a K stage is free again as soon as its S^T MMA completes.
-//   warp 6     V producer: the same for V; a V stage frees after O^T += V^T P^T.
-//              Separate rings give the loads a longer lead than one K+V stage
-//              held until the last MMA on it.
-//   warp 5     MMA: TMEM allocation; one thread issues S^T(j+1) before
-//              O^T += V^T P^T(j), so a tile's softmax overlaps the next scores.
-// The row reference m is the first tile's max (log2 units) and only moves
+//              per-thread partial row sums; per chunk, the next chunk's Q rows
+//              and the row statistics (m, l) for the epilogue.
+//   warps 7-10 epilogue: thread = d-column (TMEM lane); per chunk, reads O^T
+//              (double-buffered in TMEM, so the next chunk accumulates into
+//              the other buffer meanwhile), writes the output or the chunk's
+//              partial, takes the item's ticket and merges when last.
+//   warp 4     scheduler + K producer: lane 0 takes chunk ids (one chunk
+//              ahead) into a ring that every role reads; the warp issues TMA
+//              boxes of K into a ring of 128-key tiles, a stage freeing as soon
+//              as its S^T MMA completes.  Page ids of the next chunk are
+//              loaded while the current one streams.
+//   warp 6     V producer: the same for V, with more stages (a V stage is held
+//              until O^T += V^T P^T, after the tile's softmax).
+//   warp 5     MMA: TMEM allocation; one thread issues each S^T and each
+//              O^T += V^T P^T as soon as its operands are in place (S^T up to
+//              two tiles ahead), so loads, softmax and MMAs overlap.
+// The row reference m is a chunk's first tile max (log2 units) and only moves
 // when a tile's weight would pass 2^64 (or a row saw no key yet); then the
 // tile max is taken and O^T and the partial sums are rescaled in place.
 constexpr int kTcKeys = 128;
-constexpr int kTcStages = 3;
-constexpr int kTcThreads = 224;
+constexpr int kTcKStages = 2;                      // K ring (32 KB stages)
+constexpr int kTcVStages = 4;                      // V ring
+constexpr int kTcThreads = 352;
+constexpr int kBarEpilogue = 3;                    // named barrier of the epilogue warps
+constexpr int kChunkRing = 4;                      // chunk ids in flight between the roles
 constexpr int kBarSoftmax = 2;                     // named barrier of the softmax warps
 constexpr float kTcWeightLimit = 1.8446744e19f;    // 2^64
 
@@ -473,20 +491,45 @@ template <int RB>
 struct TcCfg {
     static constexpr int kRegionBytes = kTcKeys * 128;      // 128 keys x 64 columns (bf16), 128-byte swizzle
     static constexpr int kTileBytes = 2 * kRegionBytes;     // one K or V tile
-    static constexpr int kOffV = kTcStages * kTileBytes;    // K ring, then V ring
-    static constexpr int kOffQ = 2 * kTcStages * kTileBytes;  // Q [16 rows][128] bf16: 2 regions x 2 KB
-    static constexpr int kOffP = kOffQ + 4096;              // P^T x2: [16 rows][128 keys] bf16, 2 regions x 2 KB each
+    static constexpr int kOffV = kTcKStages * kTileBytes;   // K ring, then V ring
+    static constexpr int kOffQ = (kTcKStages + kTcVStages) * kTileBytes;  // Q x2: [16 rows][128] bf16, 2 x 2 KB each
+    static constexpr int kOffP = kOffQ + 2 * 4096;          // P^T x2: [16 rows][128 keys] bf16, 2 regions x 2 KB each
     static constexpr int kOffRed = kOffP + 2 * 4096;        // float [4 warps][16]
     static constexpr int kOffBar = kOffRed + 4 * 16 * 4;
-    // k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_full[2], o_done[2], o_final, mma_drain
-    static constexpr int kNumBars = 4 * kTcStages + 8;
-    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort, ticket, K / V tiles issued
-    static constexpr int kSmem = kOffMisc + 32;
+    // k_full[KS], k_empty[KS], v_full[VS], v_empty[VS], s_full[2], p_full[2], o_done[2], q_ready[2], drain,
+    // ch_full[R], ch_empty[R], o_item[2], o_free[2], stats[2]
+    static constexpr int kNumBars = 2 * (kTcKStages + kTcVStages) + 9 + 2 * kChunkRing + 6;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort, ticket, K / V tiles issued, chunk ring
+    static constexpr int kOffStats = kOffMisc + 32 + 4 * kChunkRing;  // [2][id, m[RB], l[RB]] per chunk parity
+    static constexpr int kStatsFloats = 1 + 2 * RB;
+    static constexpr int kOffMerge = kOffStats + 2 * kStatsFloats * 4;  // merge staging: m[256], l[256]
+    static constexpr int kSmem = kOffMerge + 512 * 4;
     static constexpr int kDynSmem = kSmem + 1024;
-    static constexpr uint32_t kTmemCols = 64;               // S^T buffers at 0 and 16, O^T at 32
+    static constexpr uint32_t kTmemCols = 64;               // S^T buffers at 0 and 16, O^T buffers at 32 and 48
     static_assert(kDynSmem <= 232448, "shared memory budget");
     static_assert(RB == 4 || RB == 8 || RB == 16, "row capacity");
 };
+
+// A chunk: tiles [t0, t1) of item (sequence si, kv-head kvh), chunk m of the
+// item's cpi; first = the item's first chunk id.
+struct ChunkInfo {
+    int si, kvh, t0, t1, cpi, m, first;
+};
+
+__device__ __forceinline__ int tc_tiles(const DecodeSeq &sq) { return (sq.n_keys + kTcKeys - 1) / kTcKeys; }
+
+__device__ __forceinline__ ChunkInfo tc_chunk(const DecodeParams &p, int c)
+{
+    int si = 0;
+    while (si + 1 < p.n_seqs && p.seqs[si + 1].tile0 <= c) ++si;  // tile0: the sequence's first chunk id
+    const int nt = tc_tiles(p.seqs[si]);
+    const int ct = p.seqs[si].cta0;                                // this sequence's tiles per chunk
+    const int cpi = (nt + ct - 1) / ct;
+    const int off = c - p.seqs[si].tile0;
+    const int kvh = off / cpi;
+    const int m = off - kvh * cpi;
+    return ChunkInfo{si, kvh, m * ct, min((m + 1) * ct, nt), cpi, m, p.seqs[si].tile0 + kvh * cpi};
+}
 
 template <int RB>
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -495,23 +538,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 {
     using C = TcCfg<RB>;
     constexpr int HD = 128;
+    constexpr int R = kChunkRing;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-
-    int si = 0;
-    while (si + 1 < p.n_seqs && static_cast<int>(blockIdx.x) >= p.seqs[si + 1].cta0) ++si;
-    const DecodeSeq &sq = p.seqs[si];
-    const int local = static_cast<int>(blockIdx.x) - sq.cta0;
-    const int kvh = local / sq.n_splits;
-    const int split = local - kvh * sq.n_splits;
     const int g = p.group;
-    const int n_rows = sq.n_q * g;
-    const int n_tiles_all = (sq.n_keys + kTcKeys - 1) / kTcKeys;
-    const int t0 = split * p.split_tiles;
-    const int nt = max(0, min(t0 + p.split_tiles, n_tiles_all) - t0);
-    const int qpos0 = sq.n_keys - sq.n_q;
 
     const uint32_t sbase = ptx::smem_addr(smem);
     const uint32_t q_smem = sbase + C::kOffQ;
@@ -519,24 +551,68 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     float *s_red = reinterpret_cast<float *>(smem + C::kOffRed);
     const uint32_t bar0 = sbase + C::kOffBar;
     auto k_full = [&](int s) { return bar0 + 8u * s; };
-    auto k_empty = [&](int s) { return bar0 + 8u * (kTcStages + s); };
-    auto v_full = [&](int s) { return bar0 + 8u * (2 * kTcStages + s); };
-    auto v_empty = [&](int s) { return bar0 + 8u * (3 * kTcStages + s); };
-    const uint32_t b_s_full = bar0 + 8u * (4 * kTcStages);      // [2]
+    auto k_empty = [&](int s) { return bar0 + 8u * (kTcKStages + s); };
+    auto v_full = [&](int s) { return bar0 + 8u * (2 * kTcKStages + s); };
+    auto v_empty = [&](int s) { return bar0 + 8u * (2 * kTcKStages + kTcVStages + s); };
+    const uint32_t b_s_full = bar0 + 8u * (2 * (kTcKStages + kTcVStages));  // [2]
     const uint32_t b_p_full = b_s_full + 16;                     // [2]
     const uint32_t b_o_done = b_p_full + 16;                     // [2]
-    const uint32_t b_o_final = b_o_done + 16;
-    const uint32_t b_drain = b_o_final + 8;
+    const uint32_t b_q_ready = b_o_done + 16;                    // [2]
+    const uint32_t b_drain = b_q_ready + 16;
+    const uint32_t b_ch_full = b_drain + 8;                      // [R]
+    const uint32_t b_ch_empty = b_ch_full + 8 * R;               // [R]
+    const uint32_t b_o_item = b_ch_empty + 8 * R;                // [2] a chunk's O^T is complete
+    const uint32_t b_o_free = b_o_item + 16;                     // [2] the epilogue has read that O^T buffer
+    const uint32_t b_stats = b_o_free + 16;                      // [2] a chunk's id, m and l are in s_stats
+    float *s_stats = reinterpret_cast<float *>(smem + C::kOffStats);
+    float *s_merge = reinterpret_cast<float *>(smem + C::kOffMerge);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 4);
     int *s_ticket = reinterpret_cast<int *>(smem + C::kOffMisc + 8);
     volatile int *s_issued = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 12);  // [2]: K, V
+    volatile int *s_chunk = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 32);  // [R]
     const WaitCtx wctx{abort_flag, p.status};
 
+    // reads chunk ordinal n from the ring (every reader arrives once); -1 = no more chunks
+    auto read_chunk = [&](int n) -> int {
+        if (!wait_bar(b_ch_full + 8 * (n % R), (n / R) & 1, wctx)) return -1;
+        return s_chunk[n % R];
+    };
+    // Q rows of item (si, kvh): each softmax thread loads two 16-byte pieces (rows past n_q x g are zero),
+    // later stored into buffer qb as [16 rows][128] bf16 with the 128-byte swizzle
+    auto load_q = [&](int si, int kvh, uint4 (&v)[2]) {
+        const DecodeSeq &sq = p.seqs[si];
+        const int n_rows = sq.n_q * g;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int e = threadIdx.x + 128 * h;
+            const int r = e >> 4;
+            const int c = e & 15;  // 16-byte chunk along d
+            v[h] = make_uint4(0u, 0u, 0u, 0u);
+            if (r < n_rows)
+                v[h] = *reinterpret_cast<const uint4 *>(
+                    static_cast<const __nv_bfloat16 *>(p.q) +
+                    (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD + c * 8);
+        }
+    };
+    auto store_q = [&](const uint4 (&v)[2], int qb) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int e = threadIdx.x + 128 * h;
+            const int r = e >> 4;
+            const int c = e & 15;
+            *reinterpret_cast<uint4 *>(smem + C::kOffQ + qb * 4096 + (c >> 3) * 2048 + r * 128 +
+                                       (((c & 7) ^ (r & 7)) << 4)) = v[h];
+        }
+        ptx::fence_proxy_async_smem();
+    };
+
     if (threadIdx.x == 128) {  // K producer warp, lane 0
-        for (int s = 0; s < kTcStages; ++s) {
+        for (int s = 0; s < kTcKStages; ++s) {
             ptx::mbar_init(k_full(s), 1);
             ptx::mbar_init(k_empty(s), 1);
+        }
+        for (int s = 0; s < kTcVStages; ++s) {
             ptx::mbar_init(v_full(s), 1);
             ptx::mbar_init(v_empty(s), 1);
         }
@@ -544,9 +620,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             ptx::mbar_init(b_s_full + 8 * b, 1);
             ptx::mbar_init(b_p_full + 8 * b, 128);
             ptx::mbar_init(b_o_done + 8 * b, 1);
+            ptx::mbar_init(b_q_ready + 8 * b, 128);
         }
-        ptx::mbar_init(b_o_final, 1);
+        for (int b = 0; b < 2; ++b) {
+            ptx::mbar_init(b_o_item + 8 * b, 1);
+            ptx::mbar_init(b_o_free + 8 * b, 128);
+            ptx::mbar_init(b_stats + 8 * b, 1);
+        }
         ptx::mbar_init(b_drain, 1);
+        for (int r = 0; r < R; ++r) {
+            ptx::mbar_init(b_ch_full + 8 * r, 1);
+            ptx::mbar_init(b_ch_empty + 8 * r, 2 + 128);  // V producer, MMA, softmax threads
+        }
         *abort_flag = 0;
         s_issued[0] = 0;
         s_issued[1] = 0;
@@ -559,17 +644,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         ptx::tmem_relinquish();
     }
     if (warp < 4) {
-        // Q rows of this kv-head into [16 rows][128] bf16, 128-byte swizzle; rows past n_q x g are zero
-        for (int e = threadIdx.x; e < 16 * 16; e += 128) {
-            const int r = e >> 4;
-            const int c = e & 15;  // 16-byte chunk along d
-            uint4 v = make_uint4(0u, 0u, 0u, 0u);
-            if (r < n_rows)
-                v = *reinterpret_cast<const uint4 *>(
-                    static_cast<const __nv_bfloat16 *>(p.q) +
-                    (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD + c * 8);
-            *reinterpret_cast<uint4 *>(smem + C::kOffQ + (c >> 3) * 2048 + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = v;
-        }
         // both P^T buffers start at zero (rows past RB stay zero)
         for (int e = threadIdx.x; e < 2 * 4096 / 16; e += 128)
             reinterpret_cast<uint4 *>(smem + C::kOffP)[e] = make_uint4(0u, 0u, 0u, 0u);
@@ -580,89 +654,212 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     const uint32_t t_s = tmem;         // S^T buffers: columns 0 and 16
-    const uint32_t t_o = tmem + 32;    // O^T: columns 32..47
+    const uint32_t t_o = tmem + 32;    // O^T buffers: columns 32..47 (even chunks) and 48..63 (odd)
 
     if (warp == 4 || warp == 6) {
-        // ============================================================ producers (warp 4: K, warp 6: V)
+        // ============================================================ producers (warp 4: K + scheduler, warp 6: V)
         const bool is_v = warp == 6;
         const CUtensorMap *map = is_v ? &tm_v : &tm_k;
+        const int n_stages = is_v ? kTcVStages : kTcKStages;
         const int kpc = p.ps < kDecKeys ? p.ps : kDecKeys;  // keys per box (<= 64)
         const int n_ops = (kTcKeys / kpc) * 2;              // boxes per tile, <= 32
         const int op_slot = lane >> 1;
         const int op_reg = lane & 1;
         const bool op_on = lane < n_ops;
-        auto page_of = [&](int t) -> int {
-            const int key0 = t * kTcKeys + op_slot * kpc;
-            if (!op_on || key0 >= sq.n_keys) return -1;
-            const int pg = p.page_table[sq.table_row + key0 / p.ps];
-            if (pg < 0 || pg >= p.num_pages) {
-                atomicCAS(p.status, 0, kStatusBadPage);
-                return -1;
-            }
-            return pg;
+        // The scheduler (lane 0 of the K producer) takes chunk ids two ahead of the chunk it issues:
+        // the counter's reply is only needed when the id is published, after a whole chunk of loads.
+        // The first two chunks are fixed (CTA b takes b and N + b); later ones come from the counter.
+        auto take = [&](int n) -> int {  // lane 0: a chunk id for ordinal n (-1: none left), not yet published
+            if (lane != 0) return -1;
+            if (n < 2) return n * static_cast<int>(gridDim.x) + static_cast<int>(blockIdx.x);
+            if (n >= R && !wait_bar(b_ch_empty + 8 * (n % R), ((n / R) - 1) & 1, wctx)) return -1;
+            return 2 * static_cast<int>(gridDim.x) + atomicAdd(p.sched, 1);
         };
-        int page_next = nt > 0 ? page_of(t0) : -1;
-        for (int i = 0; i < nt; ++i) {
-            const int t = t0 + i;
-            const int s = i % kTcStages;
-            const int page = page_next;
-            if (i + 1 < nt) page_next = page_of(t + 1);
-            const uint32_t b_empty = is_v ? v_empty(s) : k_empty(s);
-            const uint32_t b_full = is_v ? v_full(s) : k_full(s);
-            if (i >= kTcStages && !wait_bar_warp(b_empty, ((i / kTcStages) - 1) & 1, wctx)) break;
-            if (lane == 0) ptx::mbar_arrive_expect_tx(b_full, C::kTileBytes);
-            __syncwarp();
-            if (op_on) {
-                const int key0 = t * kTcKeys + op_slot * kpc;
-                const int y = page >= 0
-                                  ? ((p.layer * p.num_pages + page) * p.hkv + kvh) * p.ps + (key0 % p.ps)
-                                  : p.oob_row;
-                const uint32_t dst = sbase + (is_v ? C::kOffV : 0) + s * C::kTileBytes + op_reg * C::kRegionBytes +
-                                     op_slot * kpc * 128;
-                ptx::tma_load_2d(dst, map, op_reg * 64, y, b_full);
+        auto publish = [&](int n, int c) -> int {  // lane 0 writes ordinal n's id; every lane gets it
+            if (lane == 0) {
+                if (c >= p.total_tiles) c = -1;  // total_tiles: the launch's chunk count
+                s_chunk[n % R] = c;
+                ptx::mbar_arrive(b_ch_full + 8 * (n % R));  // release: every role can read the id
             }
+            return __shfl_sync(0xffffffffu, c, 0);
+        };
+        // raw page ids of this lane's box in the chunk's tiles (checked where used), -1 past the sequence
+        constexpr int kMaxCT = 8;  // the host keeps chunks at most 8 tiles
+        auto load_pages = [&](int c, int (&pg)[kMaxCT]) {
+#pragma unroll
+            for (int k = 0; k < kMaxCT; ++k) pg[k] = -1;
+            if (c < 0) return;
+            const ChunkInfo ci = tc_chunk(p, c);
+            const DecodeSeq &sq = p.seqs[ci.si];
+#pragma unroll
+            for (int k = 0; k < kMaxCT; ++k) {
+                const int key0 = (ci.t0 + k) * kTcKeys + op_slot * kpc;
+                if (ci.t0 + k < ci.t1 && op_on && key0 < sq.n_keys) pg[k] = p.page_table[sq.table_row + key0 / p.ps];
+            }
+        };
+        int n = 0;
+        int c_cur = -1, c_next = -1;
+        if (!is_v) {
+            c_cur = publish(0, take(0));
+            c_next = c_cur >= 0 ? publish(1, take(1)) : publish(1, -1);
+        } else {
+            c_cur = read_chunk(0);
             __syncwarp();
-            if (lane == 0) s_issued[is_v ? 1 : 0] = i + 1;
+            if (lane == 0) ptx::mbar_arrive(b_ch_empty);
+            if (c_cur >= 0) {
+                c_next = read_chunk(1);
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(b_ch_empty + 8);
+            }
+        }
+        int pa[kMaxCT], pb[kMaxCT];
+        load_pages(c_cur, pa);
+        int i = 0;  // tile ordinal in this CTA
+        while (c_cur >= 0) {
+            // the next chunk's page ids now; (K) the chunk after it from the counter, published below
+            load_pages(c_next, pb);
+            const int c_after = (!is_v && c_next >= 0) ? take(n + 2) : -1;
+            const ChunkInfo ci = tc_chunk(p, c_cur);
+            bool ok = true;
+#pragma unroll
+            for (int k = 0; k < kMaxCT; ++k) {
+                if (ci.t0 + k >= ci.t1) break;
+                const int s = i % n_stages;
+                const uint32_t b_empty = is_v ? v_empty(s) : k_empty(s);
+                const uint32_t b_full = is_v ? v_full(s) : k_full(s);
+                if (i >= n_stages && !wait_bar_warp(b_empty, ((i / n_stages) - 1) & 1, wctx)) {
+                    ok = false;
+                    break;
+                }
+                if (lane == 0) ptx::mbar_arrive_expect_tx(b_full, C::kTileBytes);
+                __syncwarp();
+                if (op_on) {
+                    const int page = pa[k];
+                    const int key0 = (ci.t0 + k) * kTcKeys + op_slot * kpc;
+                    const bool ok_page = page >= 0 && page < p.num_pages;
+                    if (!ok_page && key0 < p.seqs[ci.si].n_keys) atomicCAS(p.status, 0, kStatusBadPage);
+                    const int y = ok_page
+                                      ? ((p.layer * p.num_pages + page) * p.hkv + ci.kvh) * p.ps + (key0 % p.ps)
+                                      : p.oob_row;  // past the sequence (or a bad id): zeros
+                    const uint32_t dst = sbase + (is_v ? C::kOffV : 0) + s * C::kTileBytes +
+                                         op_reg * C::kRegionBytes + op_slot * kpc * 128;
+                    ptx::tma_load_2d(dst, map, op_reg * 64, y, b_full);
+                }
+                __syncwarp();
+                ++i;
+                if (lane == 0) s_issued[is_v ? 1 : 0] = i;
+            }
+            if (!ok) break;
+            int c2 = -1;
+            if (!is_v) {
+                if (c_next >= 0) c2 = publish(n + 2, c_after);
+            } else if (c_next >= 0) {
+                c2 = read_chunk(n + 2);
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(b_ch_empty + 8 * ((n + 2) % R));
+            }
+#pragma unroll
+            for (int k = 0; k < kMaxCT; ++k) pa[k] = pb[k];
+            c_cur = c_next;
+            c_next = c2;
+            ++n;
         }
     } else if (warp == 5) {
         // ============================================================ MMA issuer
-        if (lane == 0 && nt > 0) {
+        if (lane == 0) {
             constexpr uint32_t kIdS = ptx::idesc_bf16_f32(128, 16, false, false);
             constexpr uint32_t kIdPV = ptx::idesc_bf16_f32(128, 16, false, true);
-            auto issue_s = [&](int j) -> bool {
-                const int s = j % kTcStages;
-                if (!wait_bar(k_full(s), (j / kTcStages) & 1, wctx)) return false;
-                ptx::tc_fence_after();
-                const uint32_t ka = sbase + s * C::kTileBytes;
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const uint32_t off = (kk >> 2) * C::kRegionBytes + (kk & 3) * 32;
-                    const uint32_t qoff = (kk >> 2) * 2048 + (kk & 3) * 32;
-                    ptx::mma_bf16(t_s + 16 * (j & 1), ptx::smem_desc_sw128(ka + off, 16, 1024),
-                                  ptx::smem_desc_sw128(q_smem + qoff, 16, 1024), kIdS, kk > 0 ? 1u : 0u);
-                }
-                ptx::mma_commit(b_s_full + 8 * (j & 1));
-                ptx::mma_commit(k_empty(s));  // the K stage is free once S^T(j) is done
-                return true;
-            };
-            bool ok = issue_s(0);
-            for (int j = 0; ok && j < nt; ++j) {
-                if (j + 1 < nt && !issue_s(j + 1)) break;
-                if (!wait_bar(v_full(j % kTcStages), (j / kTcStages) & 1, wctx)) break;
-                if (!wait_bar(b_p_full + 8 * (j & 1), (j >> 1) & 1, wctx)) break;
-                ptx::tc_fence_after();
-                const uint32_t vb = sbase + C::kOffV + (j % kTcStages) * C::kTileBytes;
-                const uint32_t pb = p_smem + (j & 1) * 4096;
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    ptx::mma_bf16(t_o, ptx::smem_desc_sw128(vb + kk * 16 * 128, C::kRegionBytes, 1024),
-                                  ptx::smem_desc_sw128(pb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024), kIdPV,
-                                  (j > 0 || kk > 0) ? 1u : 0u);
-                }
-                ptx::mma_commit(v_empty(j % kTcStages));
-                ptx::mma_commit(b_o_done + 8 * (j & 1));
+            // S^T cursor: chunk ordinal ns_chunk, tile k_s within it; P V cursor: tiles left in its chunk
+            int ns = 0, np = 0;                    // next S^T tile, next P V tile (ordinals in this CTA)
+            int ns_chunk = 0;                      // chunk ordinal of tile ns
+            int s_left = 0;                        // tiles of chunk ns_chunk not yet given an S^T
+            int pv_tiles[4] = {0, 0, 0, 0};        // tile counts of chunks the S^T cursor has read
+            int np_chunk = 0, p_done = 0;          // P V cursor: chunk ordinal, tiles done in it
+            bool more = true;                      // the S^T cursor may read another chunk
+            int c0 = read_chunk(0);
+            if (c0 >= 0) {
+                const ChunkInfo ci = tc_chunk(p, c0);
+                s_left = ci.t1 - ci.t0;
+                pv_tiles[0] = s_left;
+            } else {
+                more = false;
             }
-            ptx::mma_commit(b_o_final);
+            ptx::mbar_arrive(b_ch_empty);
+            uint64_t t_last = ptx::globaltimer();
+            while (s_left > 0 || np < ns) {
+                bool progress = false;
+                // S^T(ns): K landed, S buffer free (P V(ns - 2) issued), Q of its chunk ready
+                if (s_left > 0 && ns <= np + 1) {
+                    const int s = ns % kTcKStages;
+                    const int tile_in = pv_tiles[ns_chunk & 3] - s_left;
+                    if ((tile_in > 0 || ptx::mbar_test_wait(b_q_ready + 8 * (ns_chunk & 1), (ns_chunk >> 1) & 1)) &&
+                        ptx::mbar_test_wait(k_full(s), (ns / kTcKStages) & 1)) {
+                        ptx::tc_fence_after();
+                        const uint32_t ka = sbase + s * C::kTileBytes;
+                        const uint32_t qa = q_smem + (ns_chunk & 1) * 4096;
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t off = (kk >> 2) * C::kRegionBytes + (kk & 3) * 32;
+                            const uint32_t qoff = (kk >> 2) * 2048 + (kk & 3) * 32;
+                            ptx::mma_bf16(t_s + 16 * (ns & 1), ptx::smem_desc_sw128(ka + off, 16, 1024),
+                                          ptx::smem_desc_sw128(qa + qoff, 16, 1024), kIdS, kk > 0 ? 1u : 0u);
+                        }
+                        ptx::mma_commit(b_s_full + 8 * (ns & 1));
+                        ptx::mma_commit(k_empty(s));  // the K stage is free once S^T(ns) is done
+                        ++ns;
+                        if (--s_left == 0 && more) {
+                            // next chunk (the ring entry is read once, then released)
+                            const int c = read_chunk(ns_chunk + 1);
+                            ptx::mbar_arrive(b_ch_empty + 8 * ((ns_chunk + 1) % R));
+                            if (c >= 0) {
+                                ++ns_chunk;
+                                const ChunkInfo ci = tc_chunk(p, c);
+                                s_left = ci.t1 - ci.t0;
+                                pv_tiles[ns_chunk & 3] = s_left;
+                            } else {
+                                more = false;
+                            }
+                        }
+                        progress = true;
+                    }
+                }
+                // O^T += V^T P^T(np): V landed, P^T(np) written, and at a chunk's first tile the epilogue
+                // has read the O^T buffer's previous chunk
+                if (np < ns && ptx::mbar_test_wait(v_full(np % kTcVStages), (np / kTcVStages) & 1) &&
+                    ptx::mbar_test_wait(b_p_full + 8 * (np & 1), (np >> 1) & 1) &&
+                    (p_done > 0 || np_chunk < 2 ||
+                     ptx::mbar_test_wait(b_o_free + 8 * (np_chunk & 1), ((np_chunk - 2) >> 1) & 1))) {
+                    ptx::tc_fence_after();
+                    const uint32_t vb = sbase + C::kOffV + (np % kTcVStages) * C::kTileBytes;
+                    const uint32_t pb = p_smem + (np & 1) * 4096;
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        ptx::mma_bf16(t_o + 16 * (np_chunk & 1),
+                                      ptx::smem_desc_sw128(vb + kk * 16 * 128, C::kRegionBytes, 1024),
+                                      ptx::smem_desc_sw128(pb + (kk >> 2) * 2048 + (kk & 3) * 32, 16, 1024), kIdPV,
+                                      (p_done > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    ptx::mma_commit(v_empty(np % kTcVStages));
+                    ptx::mma_commit(b_o_done + 8 * (np & 1));
+                    ++np;
+                    if (++p_done == pv_tiles[np_chunk & 3]) {
+                        ptx::mma_commit(b_o_item + 8 * (np_chunk & 1));  // the chunk's O^T is complete
+                        ++np_chunk;
+                        p_done = 0;
+                    }
+                    progress = true;
+                }
+                if (progress) {
+                    t_last = ptx::globaltimer();
+                } else {
+                    if (*abort_flag) break;
+                    if (ptx::globaltimer() - t_last > kWaitNs) {  // bounded: give up, record, let every role leave
+                        *abort_flag = 1;
+                        atomicCAS(p.status, 0, kStatusWaitTimeout);
+                        break;
+                    }
+                }
+            }
         }
         // every tcgen05 op of this CTA completes before TMEM is released
         if (lane == 0) {
@@ -672,17 +869,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
         }
         __syncwarp();
-    } else {
+    } else if (warp < 4) {
         // ============================================================ softmax (thread = key of the tile)
         const int t = threadIdx.x;              // TMEM lane
         const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
         float mref[RB], lpart[RB];
-#pragma unroll
-        for (int r = 0; r < RB; ++r) {
-            mref[r] = -INFINITY;
-            lpart[r] = 0.f;
-        }
-        // row maxima over the tile's 128 keys, for every row (all softmax threads take part)
         auto tile_max = [&](const float (&x)[RB], float (&m)[RB]) {
 #pragma unroll
             for (int r = 0; r < RB; ++r) {
@@ -697,142 +888,302 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 m[r] = fmaxf(fmaxf(s_red[r], s_red[16 + r]), fmaxf(s_red[32 + r], s_red[48 + r]));
             ptx::bar_sync(kBarSoftmax, 128);  // s_red is reused
         };
+        // chunk 0: its id, its Q rows
+        int c_cur = read_chunk(0);
+        ptx::mbar_arrive(b_ch_empty);
+        if (c_cur >= 0) {
+            const ChunkInfo ci = tc_chunk(p, c_cur);
+            uint4 qv[2];
+            load_q(ci.si, ci.kvh, qv);
+            store_q(qv, 0);
+            ptx::mbar_arrive(b_q_ready);
+        }
+        int n = 0;   // chunk ordinal
+        int i = 0;   // tile ordinal in this CTA
         bool stopped = false;
-        for (int j = 0; j < nt; ++j) {
-            const bool ok = wait_bar_warp(b_s_full + 8 * (j & 1), (j >> 1) & 1, wctx);
-            if (ptx::bar_sync_or(kBarSoftmax, 128, !ok || *abort_flag)) {
-                stopped = true;
-                break;
+        while (c_cur >= 0 && !stopped) {
+            const ChunkInfo ci = tc_chunk(p, c_cur);
+            const DecodeSeq &sq = p.seqs[ci.si];
+            const int n_rows = sq.n_q * g;
+            const int qpos0 = sq.n_keys - sq.n_q;
+            // the next chunk's id, and its Q rows: loaded now, stored after this chunk's first tile (its
+            // buffer was last read by S^T of chunk n - 1, all done)
+            const int c_next = read_chunk(n + 1);
+            ptx::mbar_arrive(b_ch_empty + 8 * ((n + 1) % R));
+            uint4 qn[2];
+            bool q_pending = false;
+            if (c_next >= 0) {
+                const ChunkInfo cn = tc_chunk(p, c_next);
+                load_q(cn.si, cn.kvh, qn);
+                q_pending = true;
             }
-            ptx::tc_fence_after();
-            float x[RB];
-            ptx::tmem_ld_n<RB>(t_s + 16 * (j & 1) + lane_off, x);
-            ptx::tmem_wait_ld();
-            const int key = (t0 + j) * kTcKeys + t;
 #pragma unroll
             for (int r = 0; r < RB; ++r) {
-                const int qpos = r < n_rows ? qpos0 + r / g : sq.n_keys - 1;
-                x[r] = (key < sq.n_keys && key <= qpos) ? x[r] * p.scale_log2 : -INFINITY;
+                mref[r] = -INFINITY;
+                lpart[r] = 0.f;
             }
-            if (j == 0) tile_max(x, mref);
-            float pr[RB];
-            bool big = false;
-#pragma unroll
-            for (int r = 0; r < RB; ++r) {
-                pr[r] = mref[r] == -INFINITY ? (x[r] == -INFINITY ? 0.f : INFINITY) : ex2(x[r] - mref[r]);
-                big = big || !(pr[r] <= kTcWeightLimit);
-            }
-            if (ptx::bar_sync_or(kBarSoftmax, 128, big)) {
-                // rare: move the reference to the running max, rescale O^T and the partial sums
-                float tm[RB], f[RB];
-                tile_max(x, tm);
+            for (int lt = ci.t0; lt < ci.t1; ++lt, ++i) {
+                const int j = lt - ci.t0;
+                const bool ok = wait_bar_warp(b_s_full + 8 * (i & 1), (i >> 1) & 1, wctx);
+                if (ptx::bar_sync_or(kBarSoftmax, 128, !ok || *abort_flag)) {
+                    stopped = true;
+                    break;
+                }
+                ptx::tc_fence_after();
+                float x[RB];
+                ptx::tmem_ld_n<RB>(t_s + 16 * (i & 1) + lane_off, x);
+                ptx::tmem_wait_ld();
+                const int key = lt * kTcKeys + t;
 #pragma unroll
                 for (int r = 0; r < RB; ++r) {
-                    const float mn = fmaxf(mref[r], tm[r]);
-                    f[r] = mn == -INFINITY ? 1.f : ex2(mref[r] - mn);
-                    mref[r] = mn;
-                    lpart[r] *= f[r];
-                    pr[r] = mn == -INFINITY ? 0.f : ex2(x[r] - mn);
+                    const int qpos = r < n_rows ? qpos0 + r / g : sq.n_keys - 1;
+                    x[r] = (key < sq.n_keys && key <= qpos) ? x[r] * p.scale_log2 : -INFINITY;
                 }
-                if (j > 0) {  // every earlier O^T update has landed
-                    const bool done = wait_bar_warp(b_o_done + 8 * ((j - 1) & 1), ((j - 1) >> 1) & 1, wctx);
-                    if (done) {
-                        ptx::tc_fence_after();
-                        float o[RB];
-                        ptx::tmem_ld_n<RB>(t_o + lane_off, o);
-                        ptx::tmem_wait_ld();
+                if (j == 0) tile_max(x, mref);
+                float pr[RB];
+                bool big = false;
 #pragma unroll
-                        for (int r = 0; r < RB; ++r) o[r] *= f[r];
-                        ptx::tmem_st_n<RB>(t_o + lane_off, o);
-                        ptx::tmem_wait_st();
+                for (int r = 0; r < RB; ++r) {
+                    pr[r] = mref[r] == -INFINITY ? (x[r] == -INFINITY ? 0.f : INFINITY) : ex2(x[r] - mref[r]);
+                    big = big || !(pr[r] <= kTcWeightLimit);
+                }
+                if (ptx::bar_sync_or(kBarSoftmax, 128, big)) {
+                    // rare: move the reference to the running max, rescale O^T and the partial sums
+                    float tm[RB], f[RB];
+                    tile_max(x, tm);
+#pragma unroll
+                    for (int r = 0; r < RB; ++r) {
+                        const float mn = fmaxf(mref[r], tm[r]);
+                        f[r] = mn == -INFINITY ? 1.f : ex2(mref[r] - mn);
+                        mref[r] = mn;
+                        lpart[r] *= f[r];
+                        pr[r] = mn == -INFINITY ? 0.f : ex2(x[r] - mn);
+                    }
+                    if (j > 0) {  // every earlier O^T update of this chunk has landed
+                        const bool done = wait_bar_warp(b_o_done + 8 * ((i - 1) & 1), ((i - 1) >> 1) & 1, wctx);
+                        if (done) {
+                            ptx::tc_fence_after();
+                            float o[RB];
+                            ptx::tmem_ld_n<RB>(t_o + 16 * (n & 1) + lane_off, o);
+                            ptx::tmem_wait_ld();
+#pragma unroll
+                            for (int r = 0; r < RB; ++r) o[r] *= f[r];
+                            ptx::tmem_st_n<RB>(t_o + 16 * (n & 1) + lane_off, o);
+                            ptx::tmem_wait_st();
+                        }
                     }
                 }
-            }
 #pragma unroll
-            for (int r = 0; r < RB; ++r) lpart[r] += pr[r];
-            // P^T(j) into buffer j & 1 once O^T += V^T P^T(j - 2) has read it
-            if (j >= 2 && !wait_bar_warp(b_o_done + 8 * (j & 1), ((j - 2) >> 1) & 1, wctx)) {
-                stopped = true;  // the other softmax warps see the abort flag at the next tile
-            }
-            uint8_t *pt = smem + C::kOffP + (j & 1) * 4096 + (t >> 6) * 2048;
-            const int chunk = (t & 63) >> 3;
+                for (int r = 0; r < RB; ++r) lpart[r] += pr[r];
+                // P^T(i) into buffer i & 1 once O^T += V^T P^T(i - 2) has read it
+                if (i >= 2) (void)wait_bar_warp(b_o_done + 8 * (i & 1), ((i - 2) >> 1) & 1, wctx);
+                uint8_t *pt = smem + C::kOffP + (i & 1) * 4096 + (t >> 6) * 2048;
+                const int chunk = (t & 63) >> 3;
 #pragma unroll
-            for (int r = 0; r < RB; ++r)
-                *reinterpret_cast<__nv_bfloat16 *>(pt + r * 128 + ((chunk ^ (r & 7)) << 4) + (t & 7) * 2) =
-                    __float2bfloat16_rn(pr[r]);
-            ptx::fence_proxy_async_smem();
-            ptx::tc_fence_before();
-            ptx::mbar_arrive(b_p_full + 8 * (j & 1));
-        }
+                for (int r = 0; r < RB; ++r)
+                    *reinterpret_cast<__nv_bfloat16 *>(pt + r * 128 + ((chunk ^ (r & 7)) << 4) + (t & 7) * 2) =
+                        __float2bfloat16_rn(pr[r]);
+                ptx::fence_proxy_async_smem();
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(b_p_full + 8 * (i & 1));
+                if (q_pending) {
+                    store_q(qn, (n + 1) & 1);
+                    ptx::mbar_arrive(b_q_ready + 8 * ((n + 1) & 1));
+                    q_pending = false;
+                }
+            }
+            if (stopped) break;
 
-        // ---------------------------------------------------------- epilogue (thread t = d-column t)
-        float o[RB];
+            // ---------------------------------------------------- row statistics for the epilogue warps
+            float lsum[RB];
 #pragma unroll
-        for (int r = 0; r < RB; ++r) o[r] = 0.f;
-        if (!stopped && nt > 0) {
-            if (wait_bar_warp(b_o_final, 0, wctx)) {
+            for (int r = 0; r < RB; ++r) {
+                float v = lpart[r];
+#pragma unroll
+                for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+                if (lane == 0) s_red[warp * 16 + r] = v;
+            }
+            ptx::bar_sync(kBarSoftmax, 128);
+#pragma unroll
+            for (int r = 0; r < RB; ++r) lsum[r] = (s_red[r] + s_red[16 + r]) + (s_red[32 + r] + s_red[48 + r]);
+            ptx::bar_sync(kBarSoftmax, 128);  // s_red is reused
+            if (t == 0) {
+                // the stats slot of chunk n - 2 must have been read
+                if (n >= 2) (void)wait_bar(b_o_free + 8 * (n & 1), ((n - 2) >> 1) & 1, wctx);
+                float *st = s_stats + (n & 1) * C::kStatsFloats;
+                st[0] = __int_as_float(c_cur);
+#pragma unroll
+                for (int r = 0; r < RB; ++r) {
+                    st[1 + r] = mref[r];
+                    st[1 + RB + r] = lsum[r];
+                }
+                ptx::mbar_arrive(b_stats + 8 * (n & 1));  // release: the epilogue reads the slot
+            }
+            c_cur = c_next;
+            ++n;
+        }
+        if (t == 0) {  // no more chunks: the epilogue warps stop at ordinal n
+            if (n >= 2) (void)wait_bar(b_o_free + 8 * (n & 1), ((n - 2) >> 1) & 1, wctx);
+            s_stats[(n & 1) * C::kStatsFloats] = __int_as_float(-1);
+            ptx::mbar_arrive(b_stats + 8 * (n & 1));
+        }
+    } else if (warp >= 7) {
+        // ============================================================ epilogue (thread = d-column = TMEM lane)
+        const int q4 = warp & 3;                       // TMEM lane quarter this warp may access
+        const int t = q4 * 32 + lane;                  // d-column
+        const int et = (warp - 7) * 32 + lane;         // thread index within the epilogue group
+        const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+        int *e_ticket = reinterpret_cast<int *>(smem + C::kOffMisc + 20);
+        for (int n = 0;; ++n) {
+            if (!wait_bar_warp(b_stats + 8 * (n & 1), (n >> 1) & 1, wctx)) break;
+            const float *st = s_stats + (n & 1) * C::kStatsFloats;
+            const int c = __float_as_int(st[0]);
+            if (c < 0) break;
+            float o[RB], mref[RB], lsum[RB];
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                mref[r] = st[1 + r];
+                lsum[r] = st[1 + RB + r];
+                o[r] = 0.f;
+            }
+            if (wait_bar_warp(b_o_item + 8 * (n & 1), (n >> 1) & 1, wctx)) {
                 ptx::tc_fence_after();
-                ptx::tmem_ld_n<RB>(t_o + lane_off, o);
+                ptx::tmem_ld_n<RB>(t_o + 16 * (n & 1) + lane_off, o);
                 ptx::tmem_wait_ld();
             }
-        }
-        // row sums over the 128 key lanes
-        float lsum[RB];
-#pragma unroll
-        for (int r = 0; r < RB; ++r) {
-            float v = lpart[r];
-#pragma unroll
-            for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-            if (lane == 0) s_red[warp * 16 + r] = v;
-        }
-        ptx::bar_sync(kBarSoftmax, 128);
-#pragma unroll
-        for (int r = 0; r < RB; ++r) lsum[r] = (s_red[r] + s_red[16 + r]) + (s_red[32 + r] + s_red[48 + r]);
-        const bool single = sq.n_splits == 1;
-        if (single) {
-            if (!stopped) {
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(b_o_free + 8 * (n & 1));  // O^T buffer and stats slot may be reused
+            const ChunkInfo ci = tc_chunk(p, c);
+            const DecodeSeq &sq = p.seqs[ci.si];
+            const int n_rows = sq.n_q * g;
+            if (ci.cpi == 1) {
 #pragma unroll
                 for (int r = 0; r < RB; ++r) {
                     if (r < n_rows) {
                         const float inv = lsum[r] > 0.f ? 1.0f / lsum[r] : 0.f;
-                        static_cast<__nv_bfloat16 *>(p.out)[(static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g +
-                                                             r % g) * HD + t] = __float2bfloat16_rn(o[r] * inv);
+                        static_cast<__nv_bfloat16 *>(p.out)[(static_cast<int64_t>(sq.q_row0 + r / g) * p.hq +
+                                                             ci.kvh * g + r % g) * HD + t] = __float2bfloat16_rn(o[r] * inv);
                     }
                 }
+                continue;
             }
-        } else {
-            float *po = p.part + static_cast<int64_t>(blockIdx.x) * RB * HD;
-            float *pm = p.part + static_cast<int64_t>(p.total_ctas) * RB * HD;
-            float *pl = pm + static_cast<int64_t>(p.total_ctas) * RB;
+            // partial of chunk c; the last of the item's chunks to finish merges, in chunk order
+            float *po = p.part + static_cast<int64_t>(c) * RB * HD;
+            float *pm = p.part + static_cast<int64_t>(p.total_tiles) * RB * HD;
+            float *pl = pm + static_cast<int64_t>(p.total_tiles) * RB;
 #pragma unroll
             for (int r = 0; r < RB; ++r) po[r * HD + t] = o[r];
-            if (t < RB) {
+            if (et < RB) {
                 float mv = -INFINITY, lv = 0.f;
 #pragma unroll
                 for (int r = 0; r < RB; ++r)
-                    if (r == t) {
+                    if (r == et) {
                         mv = mref[r];
                         lv = lsum[r];
                     }
-                pm[static_cast<int64_t>(blockIdx.x) * RB + t] = mv;
-                pl[static_cast<int64_t>(blockIdx.x) * RB + t] = lv;
+                pm[static_cast<int64_t>(c) * RB + et] = mv;
+                pl[static_cast<int64_t>(c) * RB + et] = lv;
             }
-            split_merge<RB, HD>(p, sq, si, kvh, n_rows, t, 128, kBarSoftmax, s_ticket);
+            ptx::bar_sync(kBarEpilogue, 128);  // every thread's partial is written
+            int32_t *ticket = p.tickets + ci.si * p.hkv + ci.kvh;
+            if (et == 0) {
+                __threadfence();  // the CTA's partial before its ticket
+                *e_ticket = atomicAdd(ticket, 1);
+            }
+            ptx::bar_sync(kBarEpilogue, 128);
+            const bool merge = *e_ticket == ci.cpi - 1;
+            ptx::bar_sync(kBarEpilogue, 128);  // e_ticket is reused
+            if (!merge) continue;
+            __threadfence();
+            // merge in batches of kMB chunks: their m and l staged in shared memory (one load each), the
+            // O loads of a batch issued together; M = max_k m_k, O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k
+            constexpr int kMB = 256 / RB;  // chunks per batch (the staging area holds 256 (m, l) pairs)
+            float mx[RB], den[RB], acc[RB];
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                mx[r] = -INFINITY;
+                den[r] = 0.f;
+                acc[r] = 0.f;
+            }
+            float *s_m = s_merge;
+            float *s_l = s_merge + 256;
+            for (int k0 = 0; k0 < ci.cpi; k0 += kMB) {
+                const int nb = min(kMB, ci.cpi - k0);
+                for (int e = et; e < nb * RB; e += 128) {
+                    const int64_t sl = static_cast<int64_t>(ci.first + k0) * RB + e;
+                    s_m[e] = __ldcg(pm + sl);
+                    s_l[e] = __ldcg(pl + sl);
+                }
+                ptx::bar_sync(kBarEpilogue, 128);
+                float bmx[RB];
+#pragma unroll
+                for (int r = 0; r < RB; ++r) bmx[r] = -INFINITY;
+                for (int k = 0; k < nb; ++k)
+#pragma unroll
+                    for (int r = 0; r < RB; ++r) bmx[r] = fmaxf(bmx[r], s_m[k * RB + r]);
+#pragma unroll
+                for (int r = 0; r < RB; ++r) {  // rescale the running sums to the new max
+                    const float mn = fmaxf(mx[r], bmx[r]);
+                    const float f = (mx[r] == -INFINITY || mn == -INFINITY) ? 0.f : ex2(mx[r] - mn);
+                    den[r] *= f;
+                    acc[r] *= f;
+                    mx[r] = mn;
+                }
+                for (int k = 0; k < nb; k += 4) {
+                    float ov[4][RB];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+#pragma unroll
+                        for (int r = 0; r < RB; ++r)
+                            ov[u][r] = k + u < nb ? __ldcg(p.part + ((static_cast<int64_t>(ci.first + k0 + k + u)) * RB + r) *
+                                                                      HD + t)
+                                                  : 0.f;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+#pragma unroll
+                        for (int r = 0; r < RB; ++r) {
+                            if (k + u >= nb) continue;
+                            const float ms = s_m[(k + u) * RB + r];
+                            const float w = (ms == -INFINITY || mx[r] == -INFINITY) ? 0.f : ex2(ms - mx[r]);
+                            den[r] += w * s_l[(k + u) * RB + r];
+                            acc[r] += w * ov[u][r];
+                        }
+                }
+                ptx::bar_sync(kBarEpilogue, 128);  // the staging area is reused
+            }
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                if (r >= n_rows) continue;
+                const float inv = den[r] > 0.f ? 1.0f / den[r] : 0.f;
+                static_cast<__nv_bfloat16 *>(p.out)[(static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + ci.kvh * g +
+                                                     r % g) * HD + t] = __float2bfloat16_rn(acc[r] * inv);
+            }
+            if (et == 0) *ticket = 0;
         }
     }
 
     ptx::tc_fence_before();
     __syncthreads();
-    if (threadIdx.x == 0 && *abort_flag) {
-        // after an abort, copies may still be in flight: bounded wait for the last ones issued
-        const uint64_t start = ptx::globaltimer();
-        for (int ring = 0; ring < 2; ++ring) {
-            const int issued = s_issued[ring];
-            for (int i = max(0, issued - kTcStages); i < issued; ++i) {
-                const uint32_t b = ring ? v_full(i % kTcStages) : k_full(i % kTcStages);
-                while (!ptx::mbar_try_wait(b, (i / kTcStages) & 1) && ptx::globaltimer() - start < 4000000ull) {
+    if (threadIdx.x == 0) {
+        if (*abort_flag) {
+            // after an abort, copies may still be in flight: bounded wait for the last ones issued
+            const uint64_t start = ptx::globaltimer();
+            for (int ring = 0; ring < 2; ++ring) {
+                const int issued = s_issued[ring];
+                const int n_stages = ring ? kTcVStages : kTcKStages;
+                for (int i = max(0, issued - n_stages); i < issued; ++i) {
+                    const uint32_t b = ring ? v_full(i % n_stages) : k_full(i % n_stages);
+                    while (!ptx::mbar_try_wait(b, (i / n_stages) & 1) && ptx::globaltimer() - start < 4000000ull) {
+                    }
                 }
             }
+        }
+        // the last CTA to leave resets the chunk counter for the next launch
+        __threadfence();
+        if (atomicAdd(p.sched + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+            p.sched[0] = 0;
+            p.sched[1] = 0;
+            __threadfence();
         }
     }
     if (warp == 5) {

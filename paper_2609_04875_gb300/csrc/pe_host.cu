@@ -95,7 +95,7 @@ struct pe_cache {
     CUtensorMap tm_k{}, tm_v{};    // tensor-core kernel: 64 x ps boxes
     CUtensorMap tm_kd{}, tm_vd{};  // decode kernel: 64 x min(ps, 64) boxes
     // options
-    int splitkv = -1, num_splits = 0, debug_poison = 0, decode_kernel = 1;
+    int splitkv = -1, num_splits = 0, debug_poison = 0, decode_kernel = 1, dec_chunks_per_sm = 3;
     int64_t launches = 0;
     int32_t last_split = 0, last_splits = 0, last_ctas = 0;  // plan of the last attention launch
 };
@@ -426,6 +426,76 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
     DecodeParams &p = *reinterpret_cast<DecodeParams *>(pbuf.data());
     for (size_t lo = 0; lo < items.size(); lo += kMaxSegs) {
         const size_t hi = std::min(items.size(), lo + kMaxSegs);
+        if (tc) {
+            // chunks of at most 8 tiles; CTAs (one per SM) take them from a counter
+            std::memset(&p, 0, sizeof p);
+            int64_t tiles = 0, max_rows = 1, max_tiles = 1;
+            for (size_t i = lo; i < hi; ++i) {
+                const int64_t nt = ceil_div(c->len[items[i].seq], 128);
+                tiles += nt * hkv;
+                max_tiles = std::max(max_tiles, nt);
+                max_rows = std::max<int64_t>(max_rows, static_cast<int64_t>(items[i].n_q) * g);
+            }
+            const int rb = max_rows <= 4 ? 4 : (max_rows <= 8 ? 8 : 16);
+            // chunks of ceil(tiles / (k x SMs)) tiles, 1..8 (k = "decode_chunks_per_sm", 3 by default)
+            const int64_t k_per_sm = c->dec_chunks_per_sm;
+            int64_t force = std::min<int64_t>(8, std::max<int64_t>(1, ceil_div(tiles, k_per_sm * c->num_sms)));
+            if (c->splitkv == 1 && c->num_splits > 0) force = std::min<int64_t>(8, ceil_div(max_tiles, c->num_splits));
+            int64_t chunks = 0;
+            bool any_split = false;
+            for (int pass = 0;; ++pass) {
+                chunks = 0;
+                p.n_seqs = 0;
+                any_split = false;
+                for (size_t i = lo; i < hi; ++i) {
+                    const AttnItem &it = items[i];
+                    const int64_t nt = ceil_div(c->len[it.seq], 128);
+                    int64_t ct = pass > 0 ? 8 : force;  // on a second pass the partials must fit: longest chunks
+                    DecodeSeq &q = p.seqs[p.n_seqs++];
+                    q.table_row = it.seq * cf.max_pages_per_seq;
+                    q.n_pages = static_cast<int32_t>(c->table[it.seq].size());
+                    q.q_row0 = it.q_row0;
+                    q.n_q = it.n_q;
+                    q.n_keys = static_cast<int32_t>(c->len[it.seq]);
+                    q.tile0 = static_cast<int32_t>(chunks);
+                    q.cta0 = static_cast<int32_t>(ct);
+                    const int64_t cpi = ceil_div(nt, ct);
+                    q.n_splits = static_cast<int32_t>(cpi);
+                    any_split = any_split || cpi > 1;
+                    chunks += cpi * hkv;
+                }
+                if (chunks * rb * (d + 2) * 4 <= c->ws_bytes || pass > 0) break;
+            }
+            if (chunks * rb * (d + 2) * 4 > c->ws_bytes || chunks > INT32_MAX)
+                return fail(PE_ERR_RANGE, "decode partials exceed the workspace (%lld chunks)", static_cast<long long>(chunks));
+            p.split_tiles = 0;
+            p.total_tiles = static_cast<int32_t>(chunks);
+            p.total_ctas = static_cast<int32_t>(std::min<int64_t>(chunks, c->num_sms));
+            p.page_table = c->d_table;
+            p.q = Q;
+            p.out = out;
+            p.k_pool = c->k_pool;
+            p.v_pool = c->v_pool;
+            p.part = c->d_ws;
+            p.tickets = c->d_tickets;
+            p.sched = c->d_tickets + kMaxSegs * hkv;
+            p.status = c->d_status;
+            p.hq = hq;
+            p.hkv = hkv;
+            p.group = g;
+            p.layer = layer;
+            p.num_pages = cf.num_pages;
+            p.ps = cf.page_size;
+            p.oob_row = static_cast<int32_t>(c->pool_rows);
+            p.scale_log2 = scale * 1.4426950408889634f;
+            c->last_split = any_split ? 1 : 0;
+            c->last_splits = p.seqs[0].n_splits;
+            c->last_ctas = p.total_ctas;
+            cudaError_t e = launch_decode_attn(d, rb, true, c->tm_kd, c->tm_vd, p, st);
+            if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
+            c->launches++;
+            continue;
+        }
         int64_t max_rows = 1, work = 0, max_tiles = 1;
         for (size_t i = lo; i < hi; ++i) {
             const int64_t tiles = ceil_div(c->len[items[i].seq], tile_keys);
@@ -510,7 +580,9 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     std::vector<AttnItem> order, dec;
     for (const AttnItem &it : items) {
         if (it.n_q <= 0) continue;
-        if (c->decode_kernel && static_cast<int64_t>(it.n_q) * g <= kDecMaxRows && (d == 64 || d == 128))
+        // (the tcgen05 decode kernel always splits keys across CTAs: "splitkv" = 0 keeps the prefill kernel)
+        const bool tc_nosplit = d == 128 && c->decode_kernel == 1 && c->splitkv == 0;
+        if (c->decode_kernel && static_cast<int64_t>(it.n_q) * g <= kDecMaxRows && (d == 64 || d == 128) && !tc_nosplit)
             dec.push_back(it);
         else
             order.push_back(it);
@@ -760,7 +832,8 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
         if ((e = cudaMalloc(&cc->d_status, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
         if ((e = cudaMemset(cc->d_status, 0, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
         if ((e = cudaMalloc(&cc->d_ws, cc->ws_bytes)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc workspace"); break; }
-        const size_t tickets = sizeof(int32_t) * kMaxSegs * c.num_kv_heads;
+        // per-(sequence, kv-head) merge tickets, then the decode scheduler's chunk and done counters
+        const size_t tickets = sizeof(int32_t) * (kMaxSegs * c.num_kv_heads + 2);
         if ((e = cudaMalloc(&cc->d_tickets, tickets)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
         if ((e = cudaMemset(cc->d_tickets, 0, tickets)) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
         if ((st = encode_2d(&cc->tm_k, cc->k_pool, c.head_dim, pool_rows, 64, ps)) != PE_OK) break;
@@ -1236,6 +1309,9 @@ pe_status pe_set_option(pe_cache *c, const char *key, int64_t value)
         c->num_splits = static_cast<int>(value);
     } else if (!std::strcmp(key, "debug_poison")) {
         c->debug_poison = value ? 1 : 0;
+    } else if (!std::strcmp(key, "decode_chunks_per_sm")) {
+        if (value < 1 || value > 64) return fail(PE_ERR_INVALID, "decode_chunks_per_sm must be 1..64");
+        c->dec_chunks_per_sm = static_cast<int>(value);
     } else if (!std::strcmp(key, "decode_kernel")) {
         if (value < 0 || value > 2) return fail(PE_ERR_INVALID, "decode_kernel must be 0, 1 or 2");
         c->decode_kernel = static_cast<int>(value);
@@ -1282,6 +1358,9 @@ pe_status pe_device_status(pe_cache *c, int32_t *code, int32_t clear, void *stre
     cudaError_t e = cudaStreamSynchronize(st);
     if (e == cudaSuccess) e = cudaMemcpy(code, c->d_status, sizeof(int32_t), cudaMemcpyDeviceToHost);
     if (e == cudaSuccess && clear) e = cudaMemset(c->d_status, 0, sizeof(int32_t));
+    // after a kernel gave up, its merge tickets and scheduler counters may be mid-count: reset them
+    if (e == cudaSuccess && clear && *code != 0)
+        e = cudaMemset(c->d_tickets, 0, sizeof(int32_t) * (kMaxSegs * c->cfg.num_kv_heads + 2));
     if (e != cudaSuccess) return cuda_fail(e, "device status read");
     if (*code != 0) return fail(PE_ERR_DEVICE_TIMEOUT, "a kernel reported status %d", *code);
     return PE_OK;

@@ -110,9 +110,11 @@ struct DecodeSeq {
     int32_t q_row0;        // first row of this sequence in Q / out
     int32_t n_q;
     int32_t n_keys;        // len
-    int32_t cta0;          // first CTA of this sequence: hkv x n_splits CTAs, kv-head major
+    int32_t cta0;          // CUDA-core kernel: first CTA of this sequence (hkv x n_splits CTAs, kv-head major);
+                           // tensor-core kernel: tiles per chunk of this sequence's items
     int32_t n_splits;
-    int32_t pad_;
+    int32_t tile0;         // tensor-core kernel: the first chunk id of this sequence's items (chunks
+                           // numbered sequence-major, kv-head next)
 };
 
 struct DecodeParams {
@@ -123,11 +125,13 @@ struct DecodeParams {
     const void *v_pool;
     float *part;           // split partials: O [ctas][RB][d], then m [ctas][RB], then l [ctas][RB]
     int32_t *tickets;      // one counter per (sequence, kv-head) of the launch; zero between launches
+    int32_t *sched;        // tensor-core kernel: [0] next chunk, [1] CTAs done; zero between launches
     int32_t *status;
     int32_t n_seqs, hq, hkv, group, layer, num_pages, ps;
     int32_t oob_row;       // a pool row past the end: boxes there read zeros
-    int32_t split_tiles;   // decode tiles per split
+    int32_t split_tiles;   // decode tiles per split (CUDA-core kernel) / per chunk (tensor-core kernel, <= 8)
     int32_t total_ctas;
+    int32_t total_tiles;   // tensor-core kernel: chunks of all (sequence, kv-head) items
     float scale_log2;      // softmax_scale * log2(e)
     DecodeSeq seqs[kMaxSegs];
 };
