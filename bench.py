@@ -220,6 +220,9 @@ def roofline_for(w, flops_launch, bytes_launch, attn_s, peaks, peak_src, plan=(F
         r = {"bound": "hbm", "achieved": achieved, "peak": gbs, "unit": "GB/s",
              "peak_source": f"hbm_gbs of {peak_src}"}
     r["frac"] = r["achieved"] / r["peak"]
+    if r["bound"] == "tensor":  # the same against the cuBLAS loop measured under the power cap
+        sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+        r["frac_of_sustained"] = r["achieved"] / sus
     r["traffic"] = traffic
     r["traffic_profile"] = prof
     rows = max(a.S for a in w.agents) * (w.num_q_heads // w.num_kv_heads)

@@ -161,3 +161,25 @@ def test_debug_poison_never_read(d):
         out = pair.gpu.replay_attn(s, 0, dev(q))
         torch.cuda.synchronize()
         assert_close(out, oracle.replay_attention(pair.orc, s, 0, q, 1 / math.sqrt(d)), f"poison splits={ns}")
+
+
+def test_decode_batch_beyond_one_launch():
+    """70 sequences decoding one position each: two decode launches (64 + 6
+    sequences) back to back reuse the merge tickets and the chunk counter."""
+    d, hq, hkv, ps, n_seq = 128, 32, 8, 16, 70
+    g = synth.rng(70, 7)
+    lens = [int(x) for x in g.integers(1, 1500, size=n_seq)]
+    npg = sum(-(-n // ps) for n in lens) + 8
+    pair = Pair(1, hkv, d, ps, npg, n_seq, max(-(-n // ps) for n in lens), seed=70)
+    seqs = [pair.seq() for _ in lens]
+    for s, n in zip(seqs, lens):
+        _seq(pair, s, 1, hkv, d, n, g)
+    cu = list(range(n_seq + 1))
+    q = synth.normal_bf16(g, (n_seq, hq, d))
+    for rep in range(2):
+        out = pair.gpu.replay_attn_batch(seqs, 0, dev(q), cu)
+        torch.cuda.synchronize()
+        for i, s in enumerate(seqs):
+            assert_close(out[i:i + 1], oracle.replay_attention(pair.orc, s, 0, q[i:i + 1], 1 / math.sqrt(d)),
+                         f"rep {rep} seq {i}")
+    assert pair.gpu.device_status() == 0
