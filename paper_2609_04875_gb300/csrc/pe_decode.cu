@@ -456,7 +456,7 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 // finish merges them (ticket counter), in chunk order.  The last CTA to exit
 // resets the chunk counter for the next launch.
 //
-// Roles (352 threads):
+// Roles (384 threads):
 //   warps 0-3  softmax: thread t = key t of the tile (TMEM lane t); masks,
 //              exp2 against a per-row reference, P^T (bf16) to shared memory,
 //              per-thread partial row sums; per chunk, the next chunk's Q rows
@@ -465,13 +465,15 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 //              (double-buffered in TMEM, so the next chunk accumulates into
 //              the other buffer meanwhile), writes the output or the chunk's
 //              partial, takes the item's ticket and merges when last.
-//   warp 4     scheduler + K producer: lane 0 takes chunk ids (one chunk
-//              ahead) into a ring that every role reads; the warp issues TMA
-//              boxes of K into a ring of 128-key tiles, a stage freeing as soon
-//              as its S^T MMA completes.  Page ids of the next chunk are
-//              loaded while the current one streams.
-//   warp 6     V producer: the same for V, with more stages (a V stage is held
-//              until O^T += V^T P^T, after the tile's softmax).
+//   warp 11    scheduler + page-id loader: takes chunk ids (two chunks ahead of
+//              the producers) into a ring that the MMA issuer and the softmax
+//              warps read, and turns each chunk's page ids into TMA row
+//              coordinates in a descriptor ring for the producers, so that no
+//              producer ever waits on a global load.
+//   warp 4     K producer: issues TMA boxes of K into a ring of 128-key tiles,
+//              a stage freeing as soon as its S^T MMA completes.
+//   warp 6     V producer: the same for V (a V stage is held until
+//              O^T += V^T P^T, after the tile's softmax).
 //   warp 5     MMA: TMEM allocation; one thread issues each S^T and each
 //              O^T += V^T P^T as soon as its operands are in place (S^T up to
 //              two tiles ahead), so loads, softmax and MMAs overlap.
@@ -479,11 +481,13 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 // when a tile's weight would pass 2^64 (or a row saw no key yet); then the
 // tile max is taken and O^T and the partial sums are rescaled in place.
 constexpr int kTcKeys = 128;
-constexpr int kTcKStages = 2;                      // K ring (32 KB stages)
-constexpr int kTcVStages = 4;                      // V ring
-constexpr int kTcThreads = 352;
+constexpr int kTcKStages = 3;                      // K ring (32 KB stages)
+constexpr int kTcVStages = 3;                      // V ring
+constexpr int kTcThreads = 384;
 constexpr int kBarEpilogue = 3;                    // named barrier of the epilogue warps
 constexpr int kChunkRing = 4;                      // chunk ids in flight between the roles
+constexpr int kDescRing = 3;                       // chunk descriptors (TMA rows) for the producers
+constexpr int kDescInts = 8 + 8 * 16;              // header, then the row of box (tile k, slot j) at 8 + 16 k + j
 constexpr int kBarSoftmax = 2;                     // named barrier of the softmax warps
 constexpr float kTcWeightLimit = 1.8446744e19f;    // 2^64
 
@@ -497,13 +501,15 @@ struct TcCfg {
     static constexpr int kOffRed = kOffP + 2 * 4096;        // float [4 warps][16]
     static constexpr int kOffBar = kOffRed + 4 * 16 * 4;
     // k_full[KS], k_empty[KS], v_full[VS], v_empty[VS], s_full[2], p_full[2], o_done[2], q_ready[2], drain,
-    // ch_full[R], ch_empty[R], o_item[2], o_free[2], stats[2]
-    static constexpr int kNumBars = 2 * (kTcKStages + kTcVStages) + 9 + 2 * kChunkRing + 6;
+    // ch_full[R], ch_empty[R], o_item[2], o_free[2], stats[2], desc_full[D], desc_empty[D]
+    static constexpr int kNumBars = 2 * (kTcKStages + kTcVStages) + 9 + 2 * kChunkRing + 6 + 2 * kDescRing;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort, ticket, K / V tiles issued, chunk ring
     static constexpr int kOffStats = kOffMisc + 32 + 4 * kChunkRing;  // [2][id, m[RB], l[RB]] per chunk parity
     static constexpr int kStatsFloats = 1 + 2 * RB;
     static constexpr int kOffMerge = kOffStats + 2 * kStatsFloats * 4;  // merge staging: m[256], l[256]
-    static constexpr int kSmem = kOffMerge + 512 * 4;
+    static constexpr int kOffSeqs = kOffMerge + 512 * 4;    // the launch's sequence table
+    static constexpr int kOffDesc = kOffSeqs + kMaxSegs * static_cast<int>(sizeof(DecodeSeq));
+    static constexpr int kSmem = kOffDesc + kDescRing * kDescInts * 4;
     static constexpr int kDynSmem = kSmem + 1024;
     static constexpr uint32_t kTmemCols = 64;               // S^T buffers at 0 and 16, O^T buffers at 32 and 48
     static_assert(kDynSmem <= 232448, "shared memory budget");
@@ -518,17 +524,22 @@ struct ChunkInfo {
 
 __device__ __forceinline__ int tc_tiles(const DecodeSeq &sq) { return (sq.n_keys + kTcKeys - 1) / kTcKeys; }
 
-__device__ __forceinline__ ChunkInfo tc_chunk(const DecodeParams &p, int c)
+__device__ __forceinline__ ChunkInfo tc_chunk(const DecodeParams &p, const DecodeSeq *seqs, int c)
 {
-    int si = 0;
-    while (si + 1 < p.n_seqs && p.seqs[si + 1].tile0 <= c) ++si;  // tile0: the sequence's first chunk id
-    const int nt = tc_tiles(p.seqs[si]);
-    const int ct = p.seqs[si].cta0;                                // this sequence's tiles per chunk
+    // the last sequence whose first chunk id (tile0, increasing with the sequence) is at most c
+    int si = 0, hi = p.n_seqs;
+    while (hi - si > 1) {
+        const int mid = (si + hi) >> 1;
+        if (seqs[mid].tile0 <= c) si = mid;
+        else hi = mid;
+    }
+    const int nt = tc_tiles(seqs[si]);
+    const int ct = seqs[si].cta0;                                // this sequence's tiles per chunk
     const int cpi = (nt + ct - 1) / ct;
-    const int off = c - p.seqs[si].tile0;
+    const int off = c - seqs[si].tile0;
     const int kvh = off / cpi;
     const int m = off - kvh * cpi;
-    return ChunkInfo{si, kvh, m * ct, min((m + 1) * ct, nt), cpi, m, p.seqs[si].tile0 + kvh * cpi};
+    return ChunkInfo{si, kvh, m * ct, min((m + 1) * ct, nt), cpi, m, seqs[si].tile0 + kvh * cpi};
 }
 
 template <int RB>
@@ -564,6 +575,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t b_o_item = b_ch_empty + 8 * R;                // [2] a chunk's O^T is complete
     const uint32_t b_o_free = b_o_item + 16;                     // [2] the epilogue has read that O^T buffer
     const uint32_t b_stats = b_o_free + 16;                      // [2] a chunk's id, m and l are in s_stats
+    const uint32_t b_desc_full = b_stats + 16;                   // [D] a chunk's TMA rows are in s_desc
+    const uint32_t b_desc_empty = b_desc_full + 8 * kDescRing;   // [D] both producers have issued that chunk
     float *s_stats = reinterpret_cast<float *>(smem + C::kOffStats);
     float *s_merge = reinterpret_cast<float *>(smem + C::kOffMerge);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
@@ -571,6 +584,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     int *s_ticket = reinterpret_cast<int *>(smem + C::kOffMisc + 8);
     volatile int *s_issued = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 12);  // [2]: K, V
     volatile int *s_chunk = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 32);  // [R]
+    DecodeSeq *s_seqs = reinterpret_cast<DecodeSeq *>(smem + C::kOffSeqs);
+    int *s_desc = reinterpret_cast<int *>(smem + C::kOffDesc);  // [D][kDescInts]
     const WaitCtx wctx{abort_flag, p.status};
 
     // reads chunk ordinal n from the ring (every reader arrives once); -1 = no more chunks
@@ -581,7 +596,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // Q rows of item (si, kvh): each softmax thread loads two 16-byte pieces (rows past n_q x g are zero),
     // later stored into buffer qb as [16 rows][128] bf16 with the 128-byte swizzle
     auto load_q = [&](int si, int kvh, uint4 (&v)[2]) {
-        const DecodeSeq &sq = p.seqs[si];
+        const DecodeSeq &sq = s_seqs[si];
         const int n_rows = sq.n_q * g;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
@@ -630,7 +645,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         ptx::mbar_init(b_drain, 1);
         for (int r = 0; r < R; ++r) {
             ptx::mbar_init(b_ch_full + 8 * r, 1);
-            ptx::mbar_init(b_ch_empty + 8 * r, 2 + 128);  // V producer, MMA, softmax threads
+            ptx::mbar_init(b_ch_empty + 8 * r, 1 + 128);  // MMA, softmax threads
+        }
+        for (int d = 0; d < kDescRing; ++d) {
+            ptx::mbar_init(b_desc_full + 8 * d, 1);
+            ptx::mbar_init(b_desc_empty + 8 * d, 2);      // K and V producers
         }
         *abort_flag = 0;
         s_issued[0] = 0;
@@ -648,6 +667,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int e = threadIdx.x; e < 2 * 4096 / 16; e += 128)
             reinterpret_cast<uint4 *>(smem + C::kOffP)[e] = make_uint4(0u, 0u, 0u, 0u);
         ptx::fence_proxy_async_smem();
+    } else if (warp >= 7) {
+        // the sequence table, read at every chunk by every role (binary search on tile0)
+        constexpr int kWords = static_cast<int>(sizeof(DecodeSeq) / 4);
+        const int n_words = p.n_seqs * kWords;
+        const int32_t *src = reinterpret_cast<const int32_t *>(p.seqs);
+        for (int e = threadIdx.x - 224; e < n_words; e += kTcThreads - 224)
+            reinterpret_cast<int32_t *>(s_seqs)[e] = src[e];
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -657,7 +683,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t t_o = tmem + 32;    // O^T buffers: columns 32..47 (even chunks) and 48..63 (odd)
 
     if (warp == 4 || warp == 6) {
-        // ============================================================ producers (warp 4: K + scheduler, warp 6: V)
+        // ============================================================ producers (warp 4: K, warp 6: V)
+        // Each chunk's TMA rows come ready from the loader warp; lane 2 j + h issues box j (keys
+        // [j kpc, (j + 1) kpc) of the tile) of 64-column half h.
         const bool is_v = warp == 6;
         const CUtensorMap *map = is_v ? &tm_v : &tm_k;
         const int n_stages = is_v ? kTcVStages : kTcKStages;
@@ -666,64 +694,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int op_slot = lane >> 1;
         const int op_reg = lane & 1;
         const bool op_on = lane < n_ops;
-        // The scheduler (lane 0 of the K producer) takes chunk ids two ahead of the chunk it issues:
-        // the counter's reply is only needed when the id is published, after a whole chunk of loads.
-        // The first two chunks are fixed (CTA b takes b and N + b); later ones come from the counter.
-        auto take = [&](int n) -> int {  // lane 0: a chunk id for ordinal n (-1: none left), not yet published
-            if (lane != 0) return -1;
-            if (n < 2) return n * static_cast<int>(gridDim.x) + static_cast<int>(blockIdx.x);
-            if (n >= R && !wait_bar(b_ch_empty + 8 * (n % R), ((n / R) - 1) & 1, wctx)) return -1;
-            return 2 * static_cast<int>(gridDim.x) + atomicAdd(p.sched, 1);
-        };
-        auto publish = [&](int n, int c) -> int {  // lane 0 writes ordinal n's id; every lane gets it
-            if (lane == 0) {
-                if (c >= p.total_tiles) c = -1;  // total_tiles: the launch's chunk count
-                s_chunk[n % R] = c;
-                ptx::mbar_arrive(b_ch_full + 8 * (n % R));  // release: every role can read the id
-            }
-            return __shfl_sync(0xffffffffu, c, 0);
-        };
-        // raw page ids of this lane's box in the chunk's tiles (checked where used), -1 past the sequence
-        constexpr int kMaxCT = 8;  // the host keeps chunks at most 8 tiles
-        auto load_pages = [&](int c, int (&pg)[kMaxCT]) {
-#pragma unroll
-            for (int k = 0; k < kMaxCT; ++k) pg[k] = -1;
-            if (c < 0) return;
-            const ChunkInfo ci = tc_chunk(p, c);
-            const DecodeSeq &sq = p.seqs[ci.si];
-#pragma unroll
-            for (int k = 0; k < kMaxCT; ++k) {
-                const int key0 = (ci.t0 + k) * kTcKeys + op_slot * kpc;
-                if (ci.t0 + k < ci.t1 && op_on && key0 < sq.n_keys) pg[k] = p.page_table[sq.table_row + key0 / p.ps];
-            }
-        };
-        int n = 0;
-        int c_cur = -1, c_next = -1;
-        if (!is_v) {
-            c_cur = publish(0, take(0));
-            c_next = c_cur >= 0 ? publish(1, take(1)) : publish(1, -1);
-        } else {
-            c_cur = read_chunk(0);
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(b_ch_empty);
-            if (c_cur >= 0) {
-                c_next = read_chunk(1);
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(b_ch_empty + 8);
-            }
-        }
-        int pa[kMaxCT], pb[kMaxCT];
-        load_pages(c_cur, pa);
         int i = 0;  // tile ordinal in this CTA
-        while (c_cur >= 0) {
-            // the next chunk's page ids now; (K) the chunk after it from the counter, published below
-            load_pages(c_next, pb);
-            const int c_after = (!is_v && c_next >= 0) ? take(n + 2) : -1;
-            const ChunkInfo ci = tc_chunk(p, c_cur);
+        for (int n = 0;; ++n) {
+            const int d = n % kDescRing;
+            if (!wait_bar_warp(b_desc_full + 8 * d, (n / kDescRing) & 1, wctx)) break;
+            const int *desc = s_desc + d * kDescInts;
+            if (desc[0] < 0) break;  // no more chunks
+            const int nt = desc[1];
             bool ok = true;
-#pragma unroll
-            for (int k = 0; k < kMaxCT; ++k) {
-                if (ci.t0 + k >= ci.t1) break;
+            for (int k = 0; k < nt; ++k) {
                 const int s = i % n_stages;
                 const uint32_t b_empty = is_v ? v_empty(s) : k_empty(s);
                 const uint32_t b_full = is_v ? v_full(s) : k_full(s);
@@ -734,35 +713,75 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (lane == 0) ptx::mbar_arrive_expect_tx(b_full, C::kTileBytes);
                 __syncwarp();
                 if (op_on) {
-                    const int page = pa[k];
-                    const int key0 = (ci.t0 + k) * kTcKeys + op_slot * kpc;
-                    const bool ok_page = page >= 0 && page < p.num_pages;
-                    if (!ok_page && key0 < p.seqs[ci.si].n_keys) atomicCAS(p.status, 0, kStatusBadPage);
-                    const int y = ok_page
-                                      ? ((p.layer * p.num_pages + page) * p.hkv + ci.kvh) * p.ps + (key0 % p.ps)
-                                      : p.oob_row;  // past the sequence (or a bad id): zeros
                     const uint32_t dst = sbase + (is_v ? C::kOffV : 0) + s * C::kTileBytes +
                                          op_reg * C::kRegionBytes + op_slot * kpc * 128;
-                    ptx::tma_load_2d(dst, map, op_reg * 64, y, b_full);
+                    ptx::tma_load_2d(dst, map, op_reg * 64, desc[8 + 16 * k + op_slot], b_full);
                 }
                 __syncwarp();
                 ++i;
                 if (lane == 0) s_issued[is_v ? 1 : 0] = i;
             }
             if (!ok) break;
-            int c2 = -1;
-            if (!is_v) {
-                if (c_next >= 0) c2 = publish(n + 2, c_after);
-            } else if (c_next >= 0) {
-                c2 = read_chunk(n + 2);
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(b_ch_empty + 8 * ((n + 2) % R));
+            if (lane == 0) ptx::mbar_arrive(b_desc_empty + 8 * d);  // the descriptor slot may be refilled
+        }
+    } else if (warp == 11) {
+        // ============================================================ scheduler + page-id loader
+        // Takes the chunk ids (the first two fixed: CTA b takes b and N + b; later ones from the
+        // launch's counter), publishes them to the MMA issuer and the softmax warps, and turns each
+        // chunk's page ids into the producers' TMA rows.  Ordinal n is taken once the producers are
+        // done with ordinal n - 3, so a CTA holds at most two chunks it has not started; the page-id
+        // loads wait here, not in the producers.
+        const int kpc = p.ps < kDecKeys ? p.ps : kDecKeys;
+        const int n_slots = kTcKeys / kpc;  // boxes per 64-column half, <= 16
+        constexpr int kMaxCT = 8;           // the host keeps chunks at most 8 tiles
+        for (int n = 0;; ++n) {
+            const int d = n % kDescRing;
+            const bool ok = n < kDescRing || wait_bar_warp(b_desc_empty + 8 * d, ((n / kDescRing) - 1) & 1, wctx);
+            int c = -1;
+            if (ok && lane == 0) {
+                c = n < 2 ? n * static_cast<int>(gridDim.x) + static_cast<int>(blockIdx.x)
+                          : 2 * static_cast<int>(gridDim.x) + atomicAdd(p.sched, 1);
+                if (c >= p.total_tiles) c = -1;  // total_tiles: the launch's chunk count
             }
+            c = __shfl_sync(0xffffffffu, c, 0);
+            if (lane == 0) {
+                if (n >= R) (void)wait_bar(b_ch_empty + 8 * (n % R), ((n / R) - 1) & 1, wctx);
+                s_chunk[n % R] = c;
+                ptx::mbar_arrive(b_ch_full + 8 * (n % R));  // release: the MMA issuer and softmax read the id
+            }
+            int *desc = s_desc + d * kDescInts;
+            if (c >= 0) {
+                const ChunkInfo ci = tc_chunk(p, s_seqs, c);
+                const DecodeSeq &sq = s_seqs[ci.si];
+                constexpr int kPer = kMaxCT * 16 / 32;
+                int pg[kPer];
+                bool in[kPer];
 #pragma unroll
-            for (int k = 0; k < kMaxCT; ++k) pa[k] = pb[k];
-            c_cur = c_next;
-            c_next = c2;
-            ++n;
+                for (int u = 0; u < kPer; ++u) {  // entry e = 32 u + lane: tile e / 16, box e % 16
+                    const int e = 32 * u + lane;
+                    const int key0 = (ci.t0 + (e >> 4)) * kTcKeys + (e & 15) * kpc;
+                    in[u] = ci.t0 + (e >> 4) < ci.t1 && (e & 15) < n_slots && key0 < sq.n_keys;
+                    pg[u] = in[u] ? p.page_table[sq.table_row + key0 / p.ps] : -1;
+                }
+#pragma unroll
+                for (int u = 0; u < kPer; ++u) {
+                    const int e = 32 * u + lane;
+                    const int key0 = (ci.t0 + (e >> 4)) * kTcKeys + (e & 15) * kpc;
+                    const bool ok_page = pg[u] >= 0 && pg[u] < p.num_pages;
+                    if (!ok_page && in[u]) atomicCAS(p.status, 0, kStatusBadPage);
+                    desc[8 + e] = ok_page ? ((p.layer * p.num_pages + pg[u]) * p.hkv + ci.kvh) * p.ps + key0 % p.ps
+                                          : p.oob_row;  // past the sequence (or a bad id): zeros
+                }
+                if (lane == 0) {
+                    desc[0] = c;
+                    desc[1] = ci.t1 - ci.t0;
+                }
+            } else if (lane == 0) {
+                desc[0] = -1;
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(b_desc_full + 8 * d);  // release: the producers read the rows
+            if (c < 0) break;
         }
     } else if (warp == 5) {
         // ============================================================ MMA issuer
@@ -778,7 +797,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             bool more = true;                      // the S^T cursor may read another chunk
             int c0 = read_chunk(0);
             if (c0 >= 0) {
-                const ChunkInfo ci = tc_chunk(p, c0);
+                const ChunkInfo ci = tc_chunk(p, s_seqs, c0);
                 s_left = ci.t1 - ci.t0;
                 pv_tiles[0] = s_left;
             } else {
@@ -813,7 +832,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             ptx::mbar_arrive(b_ch_empty + 8 * ((ns_chunk + 1) % R));
                             if (c >= 0) {
                                 ++ns_chunk;
-                                const ChunkInfo ci = tc_chunk(p, c);
+                                const ChunkInfo ci = tc_chunk(p, s_seqs, c);
                                 s_left = ci.t1 - ci.t0;
                                 pv_tiles[ns_chunk & 3] = s_left;
                             } else {
@@ -891,8 +910,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // chunk 0: its id, its Q rows
         int c_cur = read_chunk(0);
         ptx::mbar_arrive(b_ch_empty);
+        ChunkInfo ci{};
         if (c_cur >= 0) {
-            const ChunkInfo ci = tc_chunk(p, c_cur);
+            ci = tc_chunk(p, s_seqs, c_cur);
             uint4 qv[2];
             load_q(ci.si, ci.kvh, qv);
             store_q(qv, 0);
@@ -902,8 +922,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         int i = 0;   // tile ordinal in this CTA
         bool stopped = false;
         while (c_cur >= 0 && !stopped) {
-            const ChunkInfo ci = tc_chunk(p, c_cur);
-            const DecodeSeq &sq = p.seqs[ci.si];
+            const DecodeSeq &sq = s_seqs[ci.si];
             const int n_rows = sq.n_q * g;
             const int qpos0 = sq.n_keys - sq.n_q;
             // the next chunk's id, and its Q rows: loaded now, stored after this chunk's first tile (its
@@ -912,8 +931,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             ptx::mbar_arrive(b_ch_empty + 8 * ((n + 1) % R));
             uint4 qn[2];
             bool q_pending = false;
+            ChunkInfo cn{};
             if (c_next >= 0) {
-                const ChunkInfo cn = tc_chunk(p, c_next);
+                cn = tc_chunk(p, s_seqs, c_next);
                 load_q(cn.si, cn.kvh, qn);
                 q_pending = true;
             }
@@ -1019,6 +1039,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
                 ptx::mbar_arrive(b_stats + 8 * (n & 1));  // release: the epilogue reads the slot
             }
+            ci = cn;
             c_cur = c_next;
             ++n;
         }
@@ -1027,7 +1048,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             s_stats[(n & 1) * C::kStatsFloats] = __int_as_float(-1);
             ptx::mbar_arrive(b_stats + 8 * (n & 1));
         }
-    } else if (warp >= 7) {
+    } else if (warp >= 7 && warp < 11) {
         // ============================================================ epilogue (thread = d-column = TMEM lane)
         const int q4 = warp & 3;                       // TMEM lane quarter this warp may access
         const int t = q4 * 32 + lane;                  // d-column
@@ -1053,8 +1074,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             ptx::tc_fence_before();
             ptx::mbar_arrive(b_o_free + 8 * (n & 1));  // O^T buffer and stats slot may be reused
-            const ChunkInfo ci = tc_chunk(p, c);
-            const DecodeSeq &sq = p.seqs[ci.si];
+            const ChunkInfo ci = tc_chunk(p, s_seqs, c);
+            const DecodeSeq &sq = s_seqs[ci.si];
             const int n_rows = sq.n_q * g;
             if (ci.cpi == 1) {
 #pragma unroll
