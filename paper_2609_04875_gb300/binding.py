@@ -122,14 +122,24 @@ def _check(rc: int):
         raise PEError(rc, _lib.pe_last_error().decode())
 
 
-def _i32_array(vals):
+def i32_array(vals):
+    """A ctypes int32 array of ``vals``; the batch calls take it as is, so a
+    caller repeating a call with the same ids can convert them once."""
+    if isinstance(vals, ctypes.Array) and vals._type_ is ctypes.c_int32:
+        return vals
     vals = [int(v) for v in vals]
     return (ctypes.c_int32 * max(1, len(vals)))(*vals)
 
 
-def _i64_array(vals):
+def i64_array(vals):
+    """A ctypes int64 array of ``vals`` (taken as is by the batch calls)."""
+    if isinstance(vals, ctypes.Array) and vals._type_ is ctypes.c_int64:
+        return vals
     vals = [int(v) for v in vals]
     return (ctypes.c_int64 * max(1, len(vals)))(*vals)
+
+
+_i32_array, _i64_array = i32_array, i64_array
 
 
 def replay_schedule(agents_turns, policy):
@@ -158,6 +168,10 @@ def replay_schedule(agents_turns, policy):
 def _stream(stream):
     import torch
     if stream is None:
+        raw = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+        dev = getattr(torch._C, "_cuda_getDevice", None)
+        if raw is not None and dev is not None and torch.cuda.is_initialized():
+            return ctypes.c_void_p(raw(dev()))  # the current stream's handle, without a Stream object
         stream = torch.cuda.current_stream()
     return ctypes.c_void_p(int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream))
 

@@ -451,10 +451,13 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 // Persistent, dynamically scheduled: every (sequence, kv-head) item's 128-key
 // tiles are cut into chunks of at most 8 tiles (the host picks about three
 // chunks per SM); one CTA per SM takes chunk after chunk from a global
-// counter, so a slower SM simply takes fewer.  A chunk that is a whole item is written directly; otherwise
+// counter, so a slower SM simply takes fewer.  Chunks are numbered longest
+// first (every full chunk, then the items' shorter remainders by decreasing
+// length), so the chunks taken last are the short ones and the CTAs finish
+// close together.  A chunk that is a whole item is written directly; otherwise
 // each chunk writes a partial (O, m, l) and the last of an item's chunks to
-// finish merges them (ticket counter), in chunk order.  The last CTA to exit
-// resets the chunk counter for the next launch.
+// finish merges them (ticket counter), in the item's chunk order.  The last
+// CTA to exit resets the chunk counter for the next launch.
 //
 // Roles (384 threads):
 //   warps 0-3  softmax: thread t = key t of the tile (TMEM lane t); masks,
@@ -465,7 +468,7 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 //              (double-buffered in TMEM, so the next chunk accumulates into
 //              the other buffer meanwhile), writes the output or the chunk's
 //              partial, takes the item's ticket and merges when last.
-//   warp 11    scheduler + page-id loader: takes chunk ids (two chunks ahead of
+//   warp 11    scheduler + page-id loader: takes chunk ids (one chunk ahead of
 //              the producers) into a ring that the MMA issuer and the softmax
 //              warps read, and turns each chunk's page ids into TMA row
 //              coordinates in a descriptor ring for the producers, so that no
@@ -486,7 +489,7 @@ constexpr int kTcVStages = 3;                      // V ring
 constexpr int kTcThreads = 384;
 constexpr int kBarEpilogue = 3;                    // named barrier of the epilogue warps
 constexpr int kChunkRing = 4;                      // chunk ids in flight between the roles
-constexpr int kDescRing = 3;                       // chunk descriptors (TMA rows) for the producers
+constexpr int kDescRing = 2;                       // chunk descriptors (TMA rows) for the producers
 constexpr int kDescInts = 8 + 8 * 16;              // header, then the row of box (tile k, slot j) at 8 + 16 k + j
 constexpr int kBarSoftmax = 2;                     // named barrier of the softmax warps
 constexpr float kTcWeightLimit = 1.8446744e19f;    // 2^64
@@ -508,7 +511,7 @@ struct TcCfg {
     static constexpr int kStatsFloats = 1 + 2 * RB;
     static constexpr int kOffMerge = kOffStats + 2 * kStatsFloats * 4;  // merge staging: m[256], l[256]
     static constexpr int kOffSeqs = kOffMerge + 512 * 4;    // the launch's sequence table
-    static constexpr int kOffDesc = kOffSeqs + kMaxSegs * static_cast<int>(sizeof(DecodeSeq));
+    static constexpr int kOffDesc = kOffSeqs + kMaxSegs * static_cast<int>(sizeof(DecodeSeq) + 4);  // + rem_seq
     static constexpr int kSmem = kOffDesc + kDescRing * kDescInts * 4;
     static constexpr int kDynSmem = kSmem + 1024;
     static constexpr uint32_t kTmemCols = 64;               // S^T buffers at 0 and 16, O^T buffers at 32 and 48
@@ -516,30 +519,54 @@ struct TcCfg {
     static_assert(RB == 4 || RB == 8 || RB == 16, "row capacity");
 };
 
-// A chunk: tiles [t0, t1) of item (sequence si, kv-head kvh), chunk m of the
-// item's cpi; first = the item's first chunk id.
+// A chunk: tiles [t0, t1) of item (sequence si, kv-head kvh).  An item has
+// nfull full chunks (ids first .. first + nfull - 1) and, when its tile count
+// is not a multiple of the chunk size, one shorter remainder chunk (id rem);
+// id(k) is the item's k-th chunk, k < cpi.
 struct ChunkInfo {
-    int si, kvh, t0, t1, cpi, m, first;
+    int si, kvh, t0, t1, cpi, first, nfull, rem;
+    __device__ __forceinline__ int id(int k) const { return k < nfull ? first + k : rem; }
 };
 
 __device__ __forceinline__ int tc_tiles(const DecodeSeq &sq) { return (sq.n_keys + kTcKeys - 1) / kTcKeys; }
 
-__device__ __forceinline__ ChunkInfo tc_chunk(const DecodeParams &p, const DecodeSeq *seqs, int c)
+// seqs, rem_seq: shared-memory copies of the launch's sequence table and remainder order
+__device__ __forceinline__ ChunkInfo tc_chunk(const DecodeParams &p, const DecodeSeq *seqs, const int32_t *rem_seq,
+                                              int c)
 {
-    // the last sequence whose first chunk id (tile0, increasing with the sequence) is at most c
-    int si = 0, hi = p.n_seqs;
-    while (hi - si > 1) {
-        const int mid = (si + hi) >> 1;
-        if (seqs[mid].tile0 <= c) si = mid;
-        else hi = mid;
+    int si = 0;
+    if (c < p.full_chunks) {
+        // the last sequence whose first full chunk id (tile0, non-decreasing) is at most c: a sequence
+        // without full chunks shares tile0 with the next one, which then wins
+        int hi = p.n_seqs;
+        while (hi - si > 1) {
+            const int mid = (si + hi) >> 1;
+            if (seqs[mid].tile0 <= c) si = mid;
+            else hi = mid;
+        }
+    } else {
+        si = rem_seq[(c - p.full_chunks) / p.hkv];
     }
-    const int nt = tc_tiles(seqs[si]);
-    const int ct = seqs[si].cta0;                                // this sequence's tiles per chunk
-    const int cpi = (nt + ct - 1) / ct;
-    const int off = c - seqs[si].tile0;
-    const int kvh = off / cpi;
-    const int m = off - kvh * cpi;
-    return ChunkInfo{si, kvh, m * ct, min((m + 1) * ct, nt), cpi, m, seqs[si].tile0 + kvh * cpi};
+    const DecodeSeq &sq = seqs[si];
+    const int nt = tc_tiles(sq);
+    const int ct = sq.cta0;  // tiles per full chunk
+    ChunkInfo ci;
+    ci.si = si;
+    ci.nfull = nt / ct;
+    if (c < p.full_chunks) {
+        const int off = c - sq.tile0;
+        ci.kvh = off / ci.nfull;
+        ci.t0 = (off - ci.kvh * ci.nfull) * ct;
+        ci.t1 = ci.t0 + ct;
+    } else {
+        ci.kvh = c - sq.rem0;
+        ci.t0 = ci.nfull * ct;
+        ci.t1 = nt;
+    }
+    ci.first = sq.tile0 + ci.kvh * ci.nfull;
+    ci.rem = sq.rem0 >= 0 ? sq.rem0 + ci.kvh : -1;
+    ci.cpi = ci.nfull + (sq.rem0 >= 0 ? 1 : 0);
+    return ci;
 }
 
 template <int RB>
@@ -585,6 +612,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     volatile int *s_issued = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 12);  // [2]: K, V
     volatile int *s_chunk = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 32);  // [R]
     DecodeSeq *s_seqs = reinterpret_cast<DecodeSeq *>(smem + C::kOffSeqs);
+    int32_t *s_rem_seq = reinterpret_cast<int32_t *>(smem + C::kOffSeqs + kMaxSegs * sizeof(DecodeSeq));
     int *s_desc = reinterpret_cast<int *>(smem + C::kOffDesc);  // [D][kDescInts]
     const WaitCtx wctx{abort_flag, p.status};
 
@@ -668,12 +696,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             reinterpret_cast<uint4 *>(smem + C::kOffP)[e] = make_uint4(0u, 0u, 0u, 0u);
         ptx::fence_proxy_async_smem();
     } else if (warp >= 7) {
-        // the sequence table, read at every chunk by every role (binary search on tile0)
+        // the sequence table and the remainder order, read at every chunk by every role
         constexpr int kWords = static_cast<int>(sizeof(DecodeSeq) / 4);
         const int n_words = p.n_seqs * kWords;
         const int32_t *src = reinterpret_cast<const int32_t *>(p.seqs);
-        for (int e = threadIdx.x - 224; e < n_words; e += kTcThreads - 224)
-            reinterpret_cast<int32_t *>(s_seqs)[e] = src[e];
+        for (int e = threadIdx.x - 224; e < n_words + p.n_seqs; e += kTcThreads - 224) {
+            if (e < n_words) reinterpret_cast<int32_t *>(s_seqs)[e] = src[e];
+            else s_rem_seq[e - n_words] = p.rem_seq[e - n_words];
+        }
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -729,8 +759,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // Takes the chunk ids (the first two fixed: CTA b takes b and N + b; later ones from the
         // launch's counter), publishes them to the MMA issuer and the softmax warps, and turns each
         // chunk's page ids into the producers' TMA rows.  Ordinal n is taken once the producers are
-        // done with ordinal n - 3, so a CTA holds at most two chunks it has not started; the page-id
-        // loads wait here, not in the producers.
+        // done with ordinal n - kDescRing, so a CTA holds at most kDescRing - 1 chunks it has not
+        // started; the page-id loads wait here, not in the producers.
         const int kpc = p.ps < kDecKeys ? p.ps : kDecKeys;
         const int n_slots = kTcKeys / kpc;  // boxes per 64-column half, <= 16
         constexpr int kMaxCT = 8;           // the host keeps chunks at most 8 tiles
@@ -751,7 +781,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             int *desc = s_desc + d * kDescInts;
             if (c >= 0) {
-                const ChunkInfo ci = tc_chunk(p, s_seqs, c);
+                const ChunkInfo ci = tc_chunk(p, s_seqs, s_rem_seq, c);
                 const DecodeSeq &sq = s_seqs[ci.si];
                 constexpr int kPer = kMaxCT * 16 / 32;
                 int pg[kPer];
@@ -797,7 +827,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             bool more = true;                      // the S^T cursor may read another chunk
             int c0 = read_chunk(0);
             if (c0 >= 0) {
-                const ChunkInfo ci = tc_chunk(p, s_seqs, c0);
+                const ChunkInfo ci = tc_chunk(p, s_seqs, s_rem_seq, c0);
                 s_left = ci.t1 - ci.t0;
                 pv_tiles[0] = s_left;
             } else {
@@ -832,7 +862,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                             ptx::mbar_arrive(b_ch_empty + 8 * ((ns_chunk + 1) % R));
                             if (c >= 0) {
                                 ++ns_chunk;
-                                const ChunkInfo ci = tc_chunk(p, s_seqs, c);
+                                const ChunkInfo ci = tc_chunk(p, s_seqs, s_rem_seq, c);
                                 s_left = ci.t1 - ci.t0;
                                 pv_tiles[ns_chunk & 3] = s_left;
                             } else {
@@ -912,7 +942,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         ptx::mbar_arrive(b_ch_empty);
         ChunkInfo ci{};
         if (c_cur >= 0) {
-            ci = tc_chunk(p, s_seqs, c_cur);
+            ci = tc_chunk(p, s_seqs, s_rem_seq, c_cur);
             uint4 qv[2];
             load_q(ci.si, ci.kvh, qv);
             store_q(qv, 0);
@@ -933,7 +963,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             bool q_pending = false;
             ChunkInfo cn{};
             if (c_next >= 0) {
-                cn = tc_chunk(p, s_seqs, c_next);
+                cn = tc_chunk(p, s_seqs, s_rem_seq, c_next);
                 load_q(cn.si, cn.kvh, qn);
                 q_pending = true;
             }
@@ -1074,7 +1104,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             ptx::tc_fence_before();
             ptx::mbar_arrive(b_o_free + 8 * (n & 1));  // O^T buffer and stats slot may be reused
-            const ChunkInfo ci = tc_chunk(p, s_seqs, c);
+            const ChunkInfo ci = tc_chunk(p, s_seqs, s_rem_seq, c);
             const DecodeSeq &sq = s_seqs[ci.si];
             const int n_rows = sq.n_q * g;
             if (ci.cpi == 1) {
@@ -1088,7 +1118,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
                 continue;
             }
-            // partial of chunk c; the last of the item's chunks to finish merges, in chunk order
+            // partial of chunk c; the last of the item's chunks to finish merges, in the item's chunk order
             float *po = p.part + static_cast<int64_t>(c) * RB * HD;
             float *pm = p.part + static_cast<int64_t>(p.total_tiles) * RB * HD;
             float *pl = pm + static_cast<int64_t>(p.total_tiles) * RB;
@@ -1131,7 +1161,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int k0 = 0; k0 < ci.cpi; k0 += kMB) {
                 const int nb = min(kMB, ci.cpi - k0);
                 for (int e = et; e < nb * RB; e += 128) {
-                    const int64_t sl = static_cast<int64_t>(ci.first + k0) * RB + e;
+                    const int kb = e / RB;
+                    const int64_t sl = static_cast<int64_t>(ci.id(k0 + kb)) * RB + (e - kb * RB);
                     s_m[e] = __ldcg(pm + sl);
                     s_l[e] = __ldcg(pl + sl);
                 }
@@ -1156,7 +1187,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     for (int u = 0; u < 4; ++u)
 #pragma unroll
                         for (int r = 0; r < RB; ++r)
-                            ov[u][r] = k + u < nb ? __ldcg(p.part + ((static_cast<int64_t>(ci.first + k0 + k + u)) * RB + r) *
+                            ov[u][r] = k + u < nb ? __ldcg(p.part + (static_cast<int64_t>(ci.id(k0 + k + u)) * RB + r) *
                                                                       HD + t)
                                                   : 0.f;
 #pragma unroll

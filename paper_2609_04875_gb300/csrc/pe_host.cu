@@ -441,17 +441,23 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
             const int64_t k_per_sm = c->dec_chunks_per_sm;
             int64_t force = std::min<int64_t>(8, std::max<int64_t>(1, ceil_div(tiles, k_per_sm * c->num_sms)));
             if (c->splitkv == 1 && c->num_splits > 0) force = std::min<int64_t>(8, ceil_div(max_tiles, c->num_splits));
+            // Chunk ids, longest first: every item's full chunks (sequence-major, kv-head next), then the
+            // items' shorter remainder chunks, sequences by decreasing remainder length (ties: batch
+            // order), so that the chunks the CTAs take last are the shortest.
             int64_t chunks = 0;
             bool any_split = false;
             for (int pass = 0;; ++pass) {
                 chunks = 0;
                 p.n_seqs = 0;
                 any_split = false;
+                int32_t rems[kMaxSegs];  // sequences with a remainder chunk
+                int32_t rem_tiles[kMaxSegs];
+                int n_rem = 0;
                 for (size_t i = lo; i < hi; ++i) {
                     const AttnItem &it = items[i];
                     const int64_t nt = ceil_div(c->len[it.seq], 128);
                     int64_t ct = pass > 0 ? 8 : force;  // on a second pass the partials must fit: longest chunks
-                    DecodeSeq &q = p.seqs[p.n_seqs++];
+                    DecodeSeq &q = p.seqs[p.n_seqs];
                     q.table_row = it.seq * cf.max_pages_per_seq;
                     q.n_pages = static_cast<int32_t>(c->table[it.seq].size());
                     q.q_row0 = it.q_row0;
@@ -459,10 +465,27 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
                     q.n_keys = static_cast<int32_t>(c->len[it.seq]);
                     q.tile0 = static_cast<int32_t>(chunks);
                     q.cta0 = static_cast<int32_t>(ct);
+                    q.rem0 = -1;
                     const int64_t cpi = ceil_div(nt, ct);
                     q.n_splits = static_cast<int32_t>(cpi);
                     any_split = any_split || cpi > 1;
-                    chunks += cpi * hkv;
+                    chunks += (nt / ct) * hkv;
+                    if (nt % ct) {  // insertion by decreasing remainder length, stable
+                        int j = n_rem++;
+                        for (; j > 0 && rem_tiles[j - 1] < nt % ct; --j) {
+                            rems[j] = rems[j - 1];
+                            rem_tiles[j] = rem_tiles[j - 1];
+                        }
+                        rems[j] = p.n_seqs;
+                        rem_tiles[j] = static_cast<int32_t>(nt % ct);
+                    }
+                    p.n_seqs++;
+                }
+                p.full_chunks = static_cast<int32_t>(std::min<int64_t>(chunks, INT32_MAX));
+                for (int j = 0; j < n_rem; ++j) {
+                    p.seqs[rems[j]].rem0 = static_cast<int32_t>(std::min<int64_t>(chunks, INT32_MAX));
+                    p.rem_seq[j] = rems[j];
+                    chunks += hkv;
                 }
                 if (chunks * rb * (d + 2) * 4 <= c->ws_bytes || pass > 0) break;
             }

@@ -113,8 +113,10 @@ struct DecodeSeq {
     int32_t cta0;          // CUDA-core kernel: first CTA of this sequence (hkv x n_splits CTAs, kv-head major);
                            // tensor-core kernel: tiles per chunk of this sequence's items
     int32_t n_splits;
-    int32_t tile0;         // tensor-core kernel: the first chunk id of this sequence's items (chunks
-                           // numbered sequence-major, kv-head next)
+    int32_t tile0;         // tensor-core kernel: the first full chunk id of this sequence's items (full
+                           // chunks numbered sequence-major, kv-head next)
+    int32_t rem0;          // tensor-core kernel: the id of kv-head 0's remainder chunk (kv-head h: rem0 + h),
+                           // -1 when the tile count is a multiple of the chunk size
 };
 
 struct DecodeParams {
@@ -132,8 +134,11 @@ struct DecodeParams {
     int32_t split_tiles;   // decode tiles per split (CUDA-core kernel) / per chunk (tensor-core kernel, <= 8)
     int32_t total_ctas;
     int32_t total_tiles;   // tensor-core kernel: chunks of all (sequence, kv-head) items
+    int32_t full_chunks;   // tensor-core kernel: ids below this are full chunks, the rest remainder chunks
     float scale_log2;      // softmax_scale * log2(e)
     DecodeSeq seqs[kMaxSegs];
+    int32_t rem_seq[kMaxSegs];  // tensor-core kernel: the sequence of remainder block j (ids
+                                // full_chunks + j hkv .., one per kv-head), blocks longest first
 };
 
 // Records `msg` as this thread's last error (pe_last_error) and returns code.

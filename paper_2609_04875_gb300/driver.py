@@ -19,7 +19,7 @@ from __future__ import annotations
 import numpy as np
 import torch
 
-from .binding import PagedKVCache
+from .binding import PagedKVCache, i32_array, i64_array
 
 
 def _dev(bits: np.ndarray, device) -> torch.Tensor:
@@ -44,6 +44,8 @@ class ReplayDriver:
         self.taus = [a.tau for a in w.agents]
         S = [a.S for a in w.agents]
         self.cu = [0] + list(np.cumsum(S).astype(int))
+        # the ids of every step's calls, converted once
+        self._seqs_c, self._taus_c, self._cu_c = i32_array(self.seqs), i64_array(self.taus), i32_array(self.cu)
         n = self.cu[-1]
         # sanitized suffix inputs, packed over agents: K'/V' [L][sum S][Hkv][d], Q' [L][sum S][Hq][d]
         self.Kc = torch.empty((L, n, hkv, d), dtype=torch.bfloat16, device=self.device)
@@ -78,15 +80,15 @@ class ReplayDriver:
         return self.Kc, self.Vc, self.Qc, self.out
 
     def crop(self, stream=None):
-        self.cache.crop_batch(self.seqs, self.taus, stream=stream)
+        self.cache.crop_batch(self._seqs_c, self._taus_c, stream=stream)
 
     def append(self, stream=None, bufs=None):
         K, V = (bufs or self.buffers())[:2]
-        self.cache.append_kv_batch(self.seqs, K, V, self.cu, stream=stream)
+        self.cache.append_kv_batch(self._seqs_c, K, V, self._cu_c, stream=stream)
 
     def attend(self, layer, stream=None, bufs=None):
         Q, out = (bufs or self.buffers())[2:]
-        self.cache.replay_attn_batch(self.seqs, layer, Q[layer], self.cu, out=out[layer],
+        self.cache.replay_attn_batch(self._seqs_c, layer, Q[layer], self._cu_c, out=out[layer],
                                      softmax_scale=self.w.softmax_scale, stream=stream)
 
     def step(self, stream=None, attn_events=None, bufs=None):
@@ -151,7 +153,7 @@ class RoundsDriver(ReplayDriver):
     def step(self, stream=None, attn_events=None, bufs=None):
         K, V, Q, out = bufs or self.buffers()
         self.crop(stream)
-        self.cache.replay_rounds(self.seqs, self.take, self.cu, K, V, Q, out, softmax_scale=self.w.softmax_scale,
+        self.cache.replay_rounds(self._seqs_c, self.take, self._cu_c, K, V, Q, out, softmax_scale=self.w.softmax_scale,
                                  stream=stream)
         return out
 
