@@ -457,22 +457,23 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 // close together.  A chunk that is a whole item is written directly; otherwise
 // each chunk writes a partial (O, m, l) and the last of an item's chunks to
 // finish merges them (ticket counter), in the item's chunk order.  The last
-// CTA to exit resets the chunk counter for the next launch.
+// CTA to stop taking chunks resets the chunk counter for the next launch.
 //
 // Roles (384 threads):
 //   warps 0-3  softmax: thread t = key t of the tile (TMEM lane t); masks,
 //              exp2 against a per-row reference, P^T (bf16) to shared memory,
-//              per-thread partial row sums; per chunk, the next chunk's Q rows
-//              and the row statistics (m, l) for the epilogue.
+//              per-thread partial row sums; per chunk, the row statistics
+//              (m, l) for the epilogue.
 //   warps 7-10 epilogue: thread = d-column (TMEM lane); per chunk, reads O^T
 //              (double-buffered in TMEM, so the next chunk accumulates into
 //              the other buffer meanwhile), writes the output or the chunk's
 //              partial, takes the item's ticket and merges when last.
 //   warp 11    scheduler + page-id loader: takes chunk ids (one chunk ahead of
 //              the producers) into a ring that the MMA issuer and the softmax
-//              warps read, and turns each chunk's page ids into TMA row
-//              coordinates in a descriptor ring for the producers, so that no
-//              producer ever waits on a global load.
+//              warps read, turns each chunk's page ids into TMA row
+//              coordinates in a descriptor ring for the producers, and stages
+//              each chunk's Q rows (double-buffered), so that no role on the
+//              streaming path ever waits on a global load.
 //   warp 4     K producer: issues TMA boxes of K into a ring of 128-key tiles,
 //              a stage freeing as soon as its S^T MMA completes.
 //   warp 6     V producer: the same for V (a V stage is held until
@@ -504,13 +505,13 @@ struct TcCfg {
     static constexpr int kOffRed = kOffP + 2 * 4096;        // float [4 warps][16]
     static constexpr int kOffBar = kOffRed + 4 * 16 * 4;
     // k_full[KS], k_empty[KS], v_full[VS], v_empty[VS], s_full[2], p_full[2], o_done[2], q_ready[2], drain,
-    // ch_full[R], ch_empty[R], o_item[2], o_free[2], stats[2], desc_full[D], desc_empty[D]
-    static constexpr int kNumBars = 2 * (kTcKStages + kTcVStages) + 9 + 2 * kChunkRing + 6 + 2 * kDescRing;
+    // ch_full[R], ch_empty[R], o_item[2], o_free[2], stats[2], desc_full[D], desc_empty[D], q_free[2]
+    static constexpr int kNumBars = 2 * (kTcKStages + kTcVStages) + 9 + 2 * kChunkRing + 8 + 2 * kDescRing;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort, ticket, K / V tiles issued, chunk ring
     static constexpr int kOffStats = kOffMisc + 32 + 4 * kChunkRing;  // [2][id, m[RB], l[RB]] per chunk parity
     static constexpr int kStatsFloats = 1 + 2 * RB;
-    static constexpr int kOffMerge = kOffStats + 2 * kStatsFloats * 4;  // merge staging: m[256], l[256]
-    static constexpr int kOffSeqs = kOffMerge + 512 * 4;    // the launch's sequence table
+    static constexpr int kOffMerge = kOffStats + 2 * kStatsFloats * 4;  // merge staging: m[32], l[32]
+    static constexpr int kOffSeqs = kOffMerge + 64 * 4;     // the launch's sequence table
     static constexpr int kOffDesc = kOffSeqs + kMaxSegs * static_cast<int>(sizeof(DecodeSeq) + 4);  // + rem_seq
     static constexpr int kSmem = kOffDesc + kDescRing * kDescInts * 4;
     static constexpr int kDynSmem = kSmem + 1024;
@@ -604,6 +605,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t b_stats = b_o_free + 16;                      // [2] a chunk's id, m and l are in s_stats
     const uint32_t b_desc_full = b_stats + 16;                   // [D] a chunk's TMA rows are in s_desc
     const uint32_t b_desc_empty = b_desc_full + 8 * kDescRing;   // [D] both producers have issued that chunk
+    const uint32_t b_q_free = b_desc_empty + 8 * kDescRing;      // [2] every S^T reading that Q buffer is done
     float *s_stats = reinterpret_cast<float *>(smem + C::kOffStats);
     float *s_merge = reinterpret_cast<float *>(smem + C::kOffMerge);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
@@ -621,35 +623,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (!wait_bar(b_ch_full + 8 * (n % R), (n / R) & 1, wctx)) return -1;
         return s_chunk[n % R];
     };
-    // Q rows of item (si, kvh): each softmax thread loads two 16-byte pieces (rows past n_q x g are zero),
-    // later stored into buffer qb as [16 rows][128] bf16 with the 128-byte swizzle
-    auto load_q = [&](int si, int kvh, uint4 (&v)[2]) {
-        const DecodeSeq &sq = s_seqs[si];
-        const int n_rows = sq.n_q * g;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int e = threadIdx.x + 128 * h;
-            const int r = e >> 4;
-            const int c = e & 15;  // 16-byte chunk along d
-            v[h] = make_uint4(0u, 0u, 0u, 0u);
-            if (r < n_rows)
-                v[h] = *reinterpret_cast<const uint4 *>(
-                    static_cast<const __nv_bfloat16 *>(p.q) +
-                    (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD + c * 8);
-        }
-    };
-    auto store_q = [&](const uint4 (&v)[2], int qb) {
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int e = threadIdx.x + 128 * h;
-            const int r = e >> 4;
-            const int c = e & 15;
-            *reinterpret_cast<uint4 *>(smem + C::kOffQ + qb * 4096 + (c >> 3) * 2048 + r * 128 +
-                                       (((c & 7) ^ (r & 7)) << 4)) = v[h];
-        }
-        ptx::fence_proxy_async_smem();
-    };
-
     if (threadIdx.x == 128) {  // K producer warp, lane 0
         for (int s = 0; s < kTcKStages; ++s) {
             ptx::mbar_init(k_full(s), 1);
@@ -663,7 +636,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             ptx::mbar_init(b_s_full + 8 * b, 1);
             ptx::mbar_init(b_p_full + 8 * b, 128);
             ptx::mbar_init(b_o_done + 8 * b, 1);
-            ptx::mbar_init(b_q_ready + 8 * b, 128);
+            ptx::mbar_init(b_q_ready + 8 * b, 1);
+            ptx::mbar_init(b_q_free + 8 * b, 1);
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(b_o_item + 8 * b, 1);
@@ -812,6 +786,46 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(b_desc_full + 8 * d);  // release: the producers read the rows
             if (c < 0) break;
+            // the chunk's Q rows into buffer n & 1 as [16 rows][128] bf16 (128-byte swizzle), rows past
+            // n_q x g zero; the buffer's previous chunk (n - 2) must be done with it
+            {
+                const ChunkInfo ci = tc_chunk(p, s_seqs, s_rem_seq, c);
+                const DecodeSeq &sq = s_seqs[ci.si];
+                const int n_rows = sq.n_q * g;
+                uint4 qv[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {  // piece e = 32 j + lane: row e / 16, 16-byte column e % 16
+                    const int e = 32 * j + lane;
+                    const int r = e >> 4;
+                    qv[j] = make_uint4(0u, 0u, 0u, 0u);
+                    if (r < n_rows)
+                        qv[j] = *reinterpret_cast<const uint4 *>(
+                            static_cast<const __nv_bfloat16 *>(p.q) +
+                            (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + ci.kvh * g + r % g) * HD + (e & 15) * 8);
+                }
+                if (n >= 2 && !wait_bar_warp(b_q_free + 8 * (n & 1), ((n - 2) >> 1) & 1, wctx)) break;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const int e = 32 * j + lane;
+                    const int r = e >> 4;
+                    const int cc = e & 15;
+                    *reinterpret_cast<uint4 *>(smem + C::kOffQ + (n & 1) * 4096 + (cc >> 3) * 2048 + r * 128 +
+                                               (((cc & 7) ^ (r & 7)) << 4)) = qv[j];
+                }
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(b_q_ready + 8 * (n & 1));  // release: S^T of chunk n may read it
+            }
+        }
+        // this CTA takes no more ids: the last loader to stop resets the counter for the next launch
+        // (every other CTA has made its last atomicAdd on it by then)
+        if (lane == 0) {
+            __threadfence();
+            if (atomicAdd(p.sched + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+                p.sched[0] = 0;
+                p.sched[1] = 0;
+                __threadfence();
+            }
         }
     } else if (warp == 5) {
         // ============================================================ MMA issuer
@@ -855,6 +869,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         }
                         ptx::mma_commit(b_s_full + 8 * (ns & 1));
                         ptx::mma_commit(k_empty(s));  // the K stage is free once S^T(ns) is done
+                        if (s_left == 1) ptx::mma_commit(b_q_free + 8 * (ns_chunk & 1));  // the chunk's last S^T
                         ++ns;
                         if (--s_left == 0 && more) {
                             // next chunk (the ring entry is read once, then released)
@@ -937,17 +952,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 m[r] = fmaxf(fmaxf(s_red[r], s_red[16 + r]), fmaxf(s_red[32 + r], s_red[48 + r]));
             ptx::bar_sync(kBarSoftmax, 128);  // s_red is reused
         };
-        // chunk 0: its id, its Q rows
         int c_cur = read_chunk(0);
         ptx::mbar_arrive(b_ch_empty);
         ChunkInfo ci{};
-        if (c_cur >= 0) {
-            ci = tc_chunk(p, s_seqs, s_rem_seq, c_cur);
-            uint4 qv[2];
-            load_q(ci.si, ci.kvh, qv);
-            store_q(qv, 0);
-            ptx::mbar_arrive(b_q_ready);
-        }
+        if (c_cur >= 0) ci = tc_chunk(p, s_seqs, s_rem_seq, c_cur);
         int n = 0;   // chunk ordinal
         int i = 0;   // tile ordinal in this CTA
         bool stopped = false;
@@ -955,18 +963,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const DecodeSeq &sq = s_seqs[ci.si];
             const int n_rows = sq.n_q * g;
             const int qpos0 = sq.n_keys - sq.n_q;
-            // the next chunk's id, and its Q rows: loaded now, stored after this chunk's first tile (its
-            // buffer was last read by S^T of chunk n - 1, all done)
+            // the next chunk's id
             const int c_next = read_chunk(n + 1);
             ptx::mbar_arrive(b_ch_empty + 8 * ((n + 1) % R));
-            uint4 qn[2];
-            bool q_pending = false;
             ChunkInfo cn{};
-            if (c_next >= 0) {
-                cn = tc_chunk(p, s_seqs, s_rem_seq, c_next);
-                load_q(cn.si, cn.kvh, qn);
-                q_pending = true;
-            }
+            if (c_next >= 0) cn = tc_chunk(p, s_seqs, s_rem_seq, c_next);
 #pragma unroll
             for (int r = 0; r < RB; ++r) {
                 mref[r] = -INFINITY;
@@ -1036,11 +1037,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 ptx::fence_proxy_async_smem();
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(b_p_full + 8 * (i & 1));
-                if (q_pending) {
-                    store_q(qn, (n + 1) & 1);
-                    ptx::mbar_arrive(b_q_ready + 8 * ((n + 1) & 1));
-                    q_pending = false;
-                }
             }
             if (stopped) break;
 
@@ -1146,9 +1142,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             ptx::bar_sync(kBarEpilogue, 128);  // e_ticket is reused
             if (!merge) continue;
             __threadfence();
-            // merge in batches of kMB chunks: their m and l staged in shared memory (one load each), the
-            // O loads of a batch issued together; M = max_k m_k, O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k
-            constexpr int kMB = 256 / RB;  // chunks per batch (the staging area holds 256 (m, l) pairs)
+            // merge in batches of kOB chunks, one round of loads each: thread et < nb RB loads one (m, l)
+            // pair (staged in shared memory for every thread), and every thread its d-column of each
+            // chunk's O, all issued together; M = max_k m_k, O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k
+            constexpr int kOB = 32 / RB;  // chunks per batch (32 O values per thread in registers)
             float mx[RB], den[RB], acc[RB];
 #pragma unroll
             for (int r = 0; r < RB; ++r) {
@@ -1157,22 +1154,36 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 acc[r] = 0.f;
             }
             float *s_m = s_merge;
-            float *s_l = s_merge + 256;
-            for (int k0 = 0; k0 < ci.cpi; k0 += kMB) {
-                const int nb = min(kMB, ci.cpi - k0);
-                for (int e = et; e < nb * RB; e += 128) {
-                    const int kb = e / RB;
-                    const int64_t sl = static_cast<int64_t>(ci.id(k0 + kb)) * RB + (e - kb * RB);
-                    s_m[e] = __ldcg(pm + sl);
-                    s_l[e] = __ldcg(pl + sl);
+            float *s_l = s_merge + 32;
+            for (int k0 = 0; k0 < ci.cpi; k0 += kOB) {
+                const int nb = min(kOB, ci.cpi - k0);
+                float mv = -INFINITY, lv = 0.f;
+                if (et < nb * RB) {
+                    const int kb = et / RB;
+                    const int64_t sl = static_cast<int64_t>(ci.id(k0 + kb)) * RB + (et - kb * RB);
+                    mv = __ldcg(pm + sl);
+                    lv = __ldcg(pl + sl);
+                }
+                float ov[kOB][RB];
+#pragma unroll
+                for (int u = 0; u < kOB; ++u)
+#pragma unroll
+                    for (int r = 0; r < RB; ++r)
+                        ov[u][r] = u < nb ? __ldcg(p.part + (static_cast<int64_t>(ci.id(k0 + u)) * RB + r) * HD + t)
+                                          : 0.f;
+                if (et < nb * RB) {
+                    s_m[et] = mv;
+                    s_l[et] = lv;
                 }
                 ptx::bar_sync(kBarEpilogue, 128);
                 float bmx[RB];
 #pragma unroll
                 for (int r = 0; r < RB; ++r) bmx[r] = -INFINITY;
-                for (int k = 0; k < nb; ++k)
 #pragma unroll
-                    for (int r = 0; r < RB; ++r) bmx[r] = fmaxf(bmx[r], s_m[k * RB + r]);
+                for (int u = 0; u < kOB; ++u)
+#pragma unroll
+                    for (int r = 0; r < RB; ++r)
+                        if (u < nb) bmx[r] = fmaxf(bmx[r], s_m[u * RB + r]);
 #pragma unroll
                 for (int r = 0; r < RB; ++r) {  // rescale the running sums to the new max
                     const float mn = fmaxf(mx[r], bmx[r]);
@@ -1181,26 +1192,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     acc[r] *= f;
                     mx[r] = mn;
                 }
-                for (int k = 0; k < nb; k += 4) {
-                    float ov[4][RB];
 #pragma unroll
-                    for (int u = 0; u < 4; ++u)
+                for (int u = 0; u < kOB; ++u)
 #pragma unroll
-                        for (int r = 0; r < RB; ++r)
-                            ov[u][r] = k + u < nb ? __ldcg(p.part + (static_cast<int64_t>(ci.id(k0 + k + u)) * RB + r) *
-                                                                      HD + t)
-                                                  : 0.f;
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-#pragma unroll
-                        for (int r = 0; r < RB; ++r) {
-                            if (k + u >= nb) continue;
-                            const float ms = s_m[(k + u) * RB + r];
-                            const float w = (ms == -INFINITY || mx[r] == -INFINITY) ? 0.f : ex2(ms - mx[r]);
-                            den[r] += w * s_l[(k + u) * RB + r];
-                            acc[r] += w * ov[u][r];
-                        }
-                }
+                    for (int r = 0; r < RB; ++r) {
+                        if (u >= nb) continue;
+                        const float ms = s_m[u * RB + r];
+                        const float w = (ms == -INFINITY || mx[r] == -INFINITY) ? 0.f : ex2(ms - mx[r]);
+                        den[r] += w * s_l[u * RB + r];
+                        acc[r] += w * ov[u][r];
+                    }
                 ptx::bar_sync(kBarEpilogue, 128);  // the staging area is reused
             }
 #pragma unroll
@@ -1229,13 +1230,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     }
                 }
             }
-        }
-        // the last CTA to leave resets the chunk counter for the next launch
-        __threadfence();
-        if (atomicAdd(p.sched + 1, 1) == static_cast<int>(gridDim.x) - 1) {
-            p.sched[0] = 0;
-            p.sched[1] = 0;
-            __threadfence();
         }
     }
     if (warp == 5) {

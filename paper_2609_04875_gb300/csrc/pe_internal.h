@@ -127,7 +127,7 @@ struct DecodeParams {
     const void *v_pool;
     float *part;           // split partials: O [ctas][RB][d], then m [ctas][RB], then l [ctas][RB]
     int32_t *tickets;      // one counter per (sequence, kv-head) of the launch; zero between launches
-    int32_t *sched;        // tensor-core kernel: [0] next chunk, [1] CTAs done; zero between launches
+    int32_t *sched;        // tensor-core kernel: [0] next chunk, [1] CTAs that stopped taking; zero between launches
     int32_t *status;
     int32_t n_seqs, hq, hkv, group, layer, num_pages, ps;
     int32_t oob_row;       // a pool row past the end: boxes there read zeros
