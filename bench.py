@@ -20,6 +20,8 @@ Multi-GPU (torchrun): every rank runs its own replica of the workload
 from __future__ import annotations
 
 import argparse
+import contextlib
+import gc
 import json
 import math
 import os
@@ -83,6 +85,18 @@ def workload_flops(w):
 
 
 # ------------------------------------------------------------------ clocks
+@contextlib.contextmanager
+def no_gc():
+    """A timed region without Python's cyclic garbage collector (a collection pass would land
+    inside the region).  No collection is forced before it either: after one, the host loop of
+    a small step ran markedly slower."""
+    gc.disable()
+    try:
+        yield
+    finally:
+        gc.enable()
+
+
 class ClockSampler:
     """nvidia-smi sampling of SM clocks and throttle reasons during a region."""
 
@@ -283,11 +297,12 @@ def run_pe(args, rank, world, local_rank):
     torch.cuda.synchronize(dev)
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    t_start.record(stream)
-    for k in range(args.steps):
-        drv.step(attn_events=attn_ev[k * L:(k + 1) * L])
-    t_end.record(stream)
-    torch.cuda.synchronize(dev)
+    with no_gc():
+        t_start.record(stream)
+        for k in range(args.steps):
+            drv.step(attn_events=attn_ev[k * L:(k + 1) * L])
+        t_end.record(stream)
+        torch.cuda.synchronize(dev)
     barrier()
     launches = drv.cache.kernel_launches() - launches0
     clk = clocks.stop() if clocks else None
@@ -296,6 +311,11 @@ def run_pe(args, rank, world, local_rank):
     elapsed_ms = reduce_max(elapsed_ms, dist)
     ms_per_step = elapsed_ms / args.steps
     value = world * tokens_per_step * args.steps / (elapsed_ms / 1e3)
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(drv, dev, min(args.steps, args.e2e_steps), world, dist)
 
     # ---- crop latency: host call time and device time of the crop kernel;
     #      append time of the same steps
@@ -344,11 +364,9 @@ def run_pe(args, rank, world, local_rank):
     tau_q = pg.first_entry(src)
     prov_us = (time.perf_counter() - h0) * 1e6
     pg.close()
+    n_arts = len(arts)
+    del arts, pg
 
-    # ---- end to end through the public API with host buffers
-    e2e = None
-    if not args.no_e2e:
-        e2e = run_e2e(drv, dev, min(args.steps, args.e2e_steps), world, dist)
 
     peaks, peak_src = load_peaks()
     flops = workload_flops(w) / L  # per attention launch (one per layer)
@@ -382,7 +400,7 @@ def run_pe(args, rank, world, local_rank):
                     "device_median": statistics.median(crop_dev_us), "agents": len(w.agents)},
         "fork_us": {"host_per_fork_median": statistics.median(fork_us),
                     "host_per_release_median": statistics.median(rel_us)},
-        "provenance_query_us": {"artifacts": len(arts), "closure": len(closure), "tau": tau_q,
+        "provenance_query_us": {"artifacts": n_arts, "closure": len(closure), "tau": tau_q,
                                 "locate_closure_first_entry": prov_us},
         "recomputed_tokens": tokens_per_step,
         "session_tokens": sum(a.T for a in w.agents),
@@ -408,10 +426,16 @@ def run_e2e(drv, dev, steps, world, dist):
     output copy."""
     import torch
     K, V, Q, O = drv.buffers()
-    hK, hV, hQ = K.cpu().pin_memory(), V.cpu().pin_memory(), Q.cpu().pin_memory()
+    # the step's inputs packed into one pinned host buffer (one host->device copy per step)
+    sizes = [K.numel(), V.numel(), Q.numel()]
+    h_in = torch.cat([x.reshape(-1).cpu() for x in (K, V, Q)]).pin_memory()
     hO = [torch.empty(O.shape, dtype=O.dtype).pin_memory() for _ in range(2)]
-    sets = [(K, V, Q, O), tuple(torch.empty_like(x) for x in (K, V, Q, O))]
-    h2d_bytes = (hK.numel() + hV.numel() + hQ.numel()) * 2
+
+    def views(flat, o):
+        k, v, q = torch.split(flat, sizes)
+        return flat, (k.view(K.shape), v.view(V.shape), q.view(Q.shape), o)
+    sets = [views(torch.empty_like(h_in, device=dev), torch.empty_like(O)) for _ in range(2)]
+    h2d_bytes = h_in.numel() * 2
     d2h_bytes = O.numel() * 2
     comp = torch.cuda.current_stream(dev)
     s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
@@ -423,15 +447,14 @@ def run_e2e(drv, dev, steps, world, dist):
 
     def one(k):
         b = k % 2
-        bk, bv, bq, bo = sets[b]
+        flat, bufs = sets[b]
+        bo = bufs[3]
         s_in.wait_event(free[b])
         with torch.cuda.stream(s_in):
-            bk.copy_(hK, non_blocking=True)
-            bv.copy_(hV, non_blocking=True)
-            bq.copy_(hQ, non_blocking=True)
+            flat.copy_(h_in, non_blocking=True)
             ready[b].record(s_in)
         comp.wait_event(ready[b])
-        drv.step(bufs=sets[b])
+        drv.step(bufs=bufs)
         done[b].record(comp)
         s_out.wait_event(done[b])
         with torch.cuda.stream(s_out):
@@ -442,13 +465,14 @@ def run_e2e(drv, dev, steps, world, dist):
         one(k)
     torch.cuda.synchronize(dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(comp)
-    s_in.wait_stream(comp)
-    for k in range(steps):
-        one(k)
-    comp.wait_stream(s_out)
-    e1.record(comp)
-    torch.cuda.synchronize(dev)
+    with no_gc():
+        e0.record(comp)
+        s_in.wait_stream(comp)
+        for k in range(steps):
+            one(k)
+        comp.wait_stream(s_out)
+        e1.record(comp)
+        torch.cuda.synchronize(dev)
     ms = reduce_max(e0.elapsed_time(e1), dist)
     tokens = world * drv.w.total_suffix * steps
     return {"value": tokens / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
@@ -491,11 +515,12 @@ def run_rounds(args, rank, world, local_rank):
         barrier()
         torch.cuda.synchronize(dev)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(steps):
-            drv.step()
-        e1.record(stream)
-        torch.cuda.synchronize(dev)
+        with no_gc():
+            e0.record(stream)
+            for _ in range(steps):
+                drv.step()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
         barrier()
         clk = clocks.stop() if clocks else None
         return reduce_max(e0.elapsed_time(e1), dist) / steps, drv.cache.kernel_launches() - l0, clk
@@ -542,7 +567,8 @@ def run_rounds(args, rank, world, local_rank):
                 "peak_source": f"bf16_tflops (burst) of {peak_src}"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     roof["traffic"] = None
-    roof["kernel"] = f"replay_attn_kernel<{w.head_dim},*> (+ splitkv_combine), one launch group per round"
+    roof["kernel"] = (f"replay_attn_kernel<{w.head_dim},*> (+ splitkv_combine) for prefill rounds, "
+                      "decode_tc_kernel for decode rounds; one launch group per round")
     roof["rounds_counted"] = len(rs)
     roof["frac_all_rounds"] = sum(roof_t) / sum(t_round)
     roof["attn_ms_all_rounds"] = sum(t_round) * 1e3
