@@ -682,6 +682,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
+    // Launched with programmatic serialization: the set-up above overlapped the previous kernel (the
+    // append of the new positions); nothing written by earlier kernels is read before this point.
+    ptx::griddep_wait();
     const uint32_t tmem = *tmem_slot;
     const uint32_t t_s = tmem;         // S^T buffers: columns 0 and 16
     const uint32_t t_o = tmem + 32;    // O^T buffers: columns 32..47 (even chunks) and 48..63 (odd)
@@ -1249,8 +1252,18 @@ cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const De
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    decode_tc_kernel<RB><<<p.total_ctas, kTcThreads, C::kDynSmem, st>>>(tm_k, tm_v, p);
-    return cudaGetLastError();
+    // programmatic serialization: the CTAs' set-up may overlap the tail of the previous kernel
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(p.total_ctas));
+    cfg.blockDim = dim3(kTcThreads);
+    cfg.dynamicSmemBytes = C::kDynSmem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<RB>, tm_k, tm_v, p);
 }
 
 template <int HD, int RB>

@@ -6,6 +6,7 @@
 // chunks of one d-row, so a warp reads 512 contiguous bytes of the caller's
 // K/V and writes whole 256-byte rows (d = 128) of a page slot.
 #include "pe_internal.h"
+#include "ptx.cuh"
 
 namespace pe {
 
@@ -23,6 +24,8 @@ __device__ __forceinline__ uint4 ld_stream(const uint4 *p)
 
 __global__ void __launch_bounds__(256) append_kv_kernel(const __grid_constant__ AppendParams p, int64_t chunks)
 {
+    // the attention launch that follows may start its set-up now; it waits for this grid's writes
+    ptx::griddep_launch_dependents();
     // 1) mirror the new page ids and lengths into the device tables
     if (blockIdx.x == 0) {
         for (int s = 0; s < p.n_segs; ++s) {

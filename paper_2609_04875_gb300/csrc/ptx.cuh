@@ -13,6 +13,19 @@ __device__ __forceinline__ uint32_t smem_addr(const void *p)
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// Programmatic dependent launch: launch_dependents lets the next kernel in the
+// stream (launched with programmatic serialization) start its blocks; wait
+// blocks the calling thread until every grid this one depends on has completed
+// and its memory writes are visible (a no-op when launched without it).
+__device__ __forceinline__ void griddep_launch_dependents()
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_wait()
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 __device__ __forceinline__ uint64_t globaltimer()
 {
     uint64_t t;
