@@ -128,8 +128,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     // ---- work item -> (sequence, kv-head, split, q-tile pair); heaviest pairs first
     const int item = blockIdx.x;
-    int si = 0;
-    while (si + 1 < p.n_seqs && item >= p.seqs[si + 1].item0) ++si;
+    int si = 0, si_hi = p.n_seqs;  // the last sequence whose first item is at most `item` (binary search)
+    while (si_hi - si > 1) {
+        const int mid = (si + si_hi) >> 1;
+        if (p.seqs[mid].item0 <= item) si = mid;
+        else si_hi = mid;
+    }
     const AttnSeq &sq = p.seqs[si];
     const int n_pairs = (sq.n_qtiles + 1) >> 1;
     int local = item - sq.item0;
