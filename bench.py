@@ -187,10 +187,10 @@ def oracle_tokens_per_s(w, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "agent_batch": {"bytes": 695.853056e6 + 328.461824e6, "profile": "profiles/replay_attn_agent_batch.md",
-                    "src_sha256": "41d26fc6835fb329162de834ec0cfa144301682912a9d2651026e677a1f7a4e1"},
-    "short_suffix": {"bytes": 1.076216e9 + 21.185280e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
-                     "src_sha256": "41d26fc6835fb329162de834ec0cfa144301682912a9d2651026e677a1f7a4e1"},
+    "agent_batch": {"bytes": 696.263168e6 + 328.400896e6, "profile": "profiles/replay_attn_agent_batch.md",
+                    "src_sha256": "f24199d153228f547845e9ee5201ad6f0b528bee5df3e682544ec0496351f98b"},
+    "short_suffix": {"bytes": 1.076231e9 + 21.225984e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
+                     "src_sha256": "f24199d153228f547845e9ee5201ad6f0b528bee5df3e682544ec0496351f98b"},
 }
 ATTN_SRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc", "pe_attn.cu")
 
