@@ -191,19 +191,29 @@ NCU_TRAFFIC = {
                     "src_sha256": "f24199d153228f547845e9ee5201ad6f0b528bee5df3e682544ec0496351f98b"},
     "short_suffix": {"bytes": 1.076231e9 + 21.225984e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
                      "src_sha256": "f24199d153228f547845e9ee5201ad6f0b528bee5df3e682544ec0496351f98b"},
+    "decode_batch": {"bytes": 342.246144e6 + 4.516864e6, "profile": "profiles/decode_tc_decode_batch.md",
+                     "kernel": "decode",
+                     "src_sha256": "f1ad7fd4cc5e0b150afbdab37a0c8c662e01f9f53786b5c5fd49539b343492ed"},
 }
-ATTN_SRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc", "pe_attn.cu")
+CSRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc")
+# (file, first line of the kernel's source, the text that follows it): the span that is hashed
+KERNEL_SRC = {
+    "prefill": ("pe_attn.cu", "template <int HD, bool SPLIT>\n__global__", "// Exercises the bounded wait on its own"),
+    "decode": ("pe_decode.cu", "template <int RB>\n__global__ void __launch_bounds__(kTcThreads, 1)",
+               "template <int RB>\ncudaError_t launch_tc("),
+}
 
 
-def _src_sha():
-    """sha256 of the attention kernel function's source, so that recorded
-    counters lapse when the kernel changes."""
+def _src_sha(kernel="prefill"):
+    """sha256 of a kernel function's source, so that recorded counters lapse
+    when the kernel changes."""
     import hashlib
-    with open(ATTN_SRC) as f:
+    name, start, end = KERNEL_SRC[kernel]
+    with open(os.path.join(CSRC, name)) as f:
         txt = f.read()
     try:
-        a = txt.index("template <int HD, bool SPLIT>\n__global__")
-        b = txt.index("// Exercises the bounded wait on its own")
+        a = txt.index(start)
+        b = txt.index(end, a)
     except ValueError:
         return None
     return hashlib.sha256(txt[a:b].encode()).hexdigest()
@@ -211,7 +221,7 @@ def _src_sha():
 
 def traffic_for(workload):
     t = NCU_TRAFFIC.get(workload)
-    if not t or t["src_sha256"] != _src_sha():
+    if not t or t["src_sha256"] != _src_sha(t.get("kernel", "prefill")):
         return None, None
     return t["bytes"], t["profile"]
 
