@@ -431,8 +431,8 @@ def run_e2e(drv, dev, steps, world, dist):
     """The same step through the public API with the step's inputs (K', V', Q')
     in pinned host memory: every step copies its inputs host->device, runs
     crop + append + replay and copies its output device->host.  Copies run on
-    their own streams and overlap other steps' compute; with three device
-    buffer sets, step k's input copy only waits for step k-3's output copy, so
+    their own streams and overlap other steps' compute; with four device
+    buffer sets, step k's input copy only waits for step k-4's output copy, so
     the loop runs at the copy engines' pace rather than at the sum of a copy
     in, a step and a copy out.  The timed region spans the first input copy to
     the last output copy."""
@@ -441,7 +441,7 @@ def run_e2e(drv, dev, steps, world, dist):
     # the step's inputs packed into one pinned host buffer (one host->device copy per step)
     sizes = [K.numel(), V.numel(), Q.numel()]
     h_in = torch.cat([x.reshape(-1).cpu() for x in (K, V, Q)]).pin_memory()
-    nb = 3  # buffer sets in flight
+    nb = 4  # buffer sets in flight
 
     def views(flat, o):
         k, v, q = torch.split(flat, sizes)
@@ -490,7 +490,7 @@ def run_e2e(drv, dev, steps, world, dist):
     tokens = world * drv.w.total_suffix * steps
     return {"value": tokens / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
             "d2h_bytes_per_step": d2h_bytes, "steps": steps, "ms_per_step": ms / steps,
-            "overlap": "three buffer sets: copies of other steps overlap the compute of step k"}
+            "overlap": "four buffer sets: copies of other steps overlap the compute of step k"}
 
 
 def run_rounds(args, rank, world, local_rank):
