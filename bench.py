@@ -325,7 +325,7 @@ def run_pe(args, rank, world, local_rank):
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(drv, dev, min(args.steps, args.e2e_steps), world, dist)
+        e2e = run_e2e(drv, dev, min(args.steps, args.e2e_steps), world, dist, ms_per_step)
 
     # ---- crop latency: host call time and device time of the crop kernel;
     #      append time of the same steps
@@ -427,21 +427,27 @@ def run_pe(args, rank, world, local_rank):
         print(json.dumps(result), flush=True)
 
 
-def run_e2e(drv, dev, steps, world, dist):
+PINNED_COPY_GBS = 330.0  # measured pinned host<->device rate, both directions at once (GB300 machine)
+
+
+def run_e2e(drv, dev, steps, world, dist, step_ms):
     """The same step through the public API with the step's inputs (K', V', Q')
     in pinned host memory: every step copies its inputs host->device, runs
     crop + append + replay and copies its output device->host.  Copies run on
-    their own streams and overlap other steps' compute; with four device
-    buffer sets, step k's input copy only waits for step k-4's output copy, so
-    the loop runs at the copy engines' pace rather than at the sum of a copy
-    in, a step and a copy out.  The timed region spans the first input copy to
-    the last output copy."""
+    their own streams and overlap other steps' compute.  When the copies take
+    at least half as long as a step (step_ms, measured device-resident), four
+    device buffer sets keep them running back to back: step k's input copy
+    only waits for step k-4's output copy, so the loop runs at the copy
+    engines' pace rather than at the sum of a copy in, a step and a copy out.
+    Otherwise two sets suffice: the copies hide behind the step.  The timed
+    region spans the first input copy to the last output copy."""
     import torch
     K, V, Q, O = drv.buffers()
     # the step's inputs packed into one pinned host buffer (one host->device copy per step)
     sizes = [K.numel(), V.numel(), Q.numel()]
     h_in = torch.cat([x.reshape(-1).cpu() for x in (K, V, Q)]).pin_memory()
-    nb = 4  # buffer sets in flight
+    copy_ms = (h_in.numel() + O.numel()) * 2 / (PINNED_COPY_GBS * 1e9) * 1e3
+    nb = 4 if copy_ms >= 0.5 * step_ms else 2  # buffer sets in flight
 
     def views(flat, o):
         k, v, q = torch.split(flat, sizes)
@@ -490,7 +496,7 @@ def run_e2e(drv, dev, steps, world, dist):
     tokens = world * drv.w.total_suffix * steps
     return {"value": tokens / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
             "d2h_bytes_per_step": d2h_bytes, "steps": steps, "ms_per_step": ms / steps,
-            "overlap": "four buffer sets: copies of other steps overlap the compute of step k"}
+            "overlap": f"{nb} buffer sets: copies of other steps overlap the compute of step k"}
 
 
 def run_rounds(args, rank, world, local_rank):
@@ -590,7 +596,7 @@ def run_rounds(args, rank, world, local_rank):
     e2e = None
     if not args.no_e2e:
         drv.set_policy(POLICY_SELECTIVE)
-        e2e = run_e2e(drv, dev, min(args.steps, args.e2e_steps), world, dist)
+        e2e = run_e2e(drv, dev, min(args.steps, args.e2e_steps), world, dist, ms_sel)
     value = world * tokens_per_step / (ms_sel / 1e3)
     result = {
         "metric": METRIC,
