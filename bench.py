@@ -427,7 +427,7 @@ def run_pe(args, rank, world, local_rank):
         print(json.dumps(result), flush=True)
 
 
-PINNED_COPY_GBS = 330.0  # measured pinned host<->device rate, both directions at once (GB300 machine)
+PINNED_COPY_GBS = 330.0  # pinned host<->device copy rate, both directions at once, measured on a GB300
 
 
 def run_e2e(drv, dev, steps, world, dist, step_ms):
