@@ -135,13 +135,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         else si_hi = mid;
     }
     const AttnSeq &sq = p.seqs[si];
-    const int n_pairs = (sq.n_qtiles + 1) >> 1;
     int local = item - sq.item0;
     const int kvh = local % p.hkv;
     local /= p.hkv;
     const int split = local % sq.n_splits;
     local /= sq.n_splits;
-    const int pair = n_pairs - 1 - local;
+    const int pair = sq.pair_top - 1 - local;
     const int g = p.group;
     const int bmq = kBM / g;
     const int kt0 = SPLIT ? split * p.split_tiles : 0;

@@ -623,7 +623,8 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     pe_status s = encode_q(&tm_q, Q, q_rows, hq, d, g);
     if (s != PE_OK) return s;
 
-    // split-KV decision over the whole launch group
+    // split-KV decision over the whole launch group; plan_est: the cost model's time of the plan
+    double plan_est = 0.0;
     auto plan_group = [&](size_t lo, size_t hi, AttnParams &p, bool &split) -> pe_status {
         // C CTAs (pairs of q-tiles x kv-heads), W key tiles per CTA on average.
         int64_t C = 0, tiles = 0, rows = 0, valid_rows = 0, max_tiles = 0;
@@ -664,6 +665,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             if (c->splitkv == -1 && best > 1 && best_t > 0.95 * cost(1)) best = 1;  // keep the single pass unless clearly faster
         }
         if (c->splitkv != 0 && c->num_splits > 0) best = c->num_splits;
+        plan_est = cost(best);
         int split_tiles = static_cast<int>(max_tiles);
         split = best > 1 || c->splitkv == 1;
         if (split) split_tiles = static_cast<int>(std::max<int64_t>(1, ceil_div(max_tiles, std::max<int64_t>(best, 1))));
@@ -692,6 +694,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
                 q.n_q = it.n_q;
                 q.n_keys = static_cast<int32_t>(c->len[it.seq]);
                 q.n_qtiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(it.n_q) * g, kBM));
+                q.pair_top = (q.n_qtiles + 1) / 2;
                 const int64_t ktiles = ceil_div(c->len[it.seq], kBN);
                 q.n_splits = split ? static_cast<int32_t>(ceil_div(ktiles, split_tiles)) : 1;
                 q.item0 = item;
@@ -723,6 +726,51 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         return PE_OK;
     };
 
+    // Tail launch for a launch group of one sequence (one long agent): when its CTAs leave the last
+    // wave mostly empty, the lightest q-tile pairs (the last CTAs in the heaviest-first order) move
+    // to a second launch that splits their keys over every SM; the first launch then fills whole
+    // waves.  Chosen by the same cost model, when it beats the group's plan by 5 %.
+    struct TailPlan {
+        int64_t pairs = 0, splits = 0, split_tiles = 0, qtiles = 0;
+    };
+    auto plan_tail = [&](const AttnItem &it, TailPlan &tp) -> bool {
+        const int64_t len = c->len[it.seq];
+        const int64_t nqt = ceil_div(static_cast<int64_t>(it.n_q) * g, kBM);
+        const int64_t n_pairs = ceil_div(nqt, 2);
+        const int64_t C = n_pairs * hkv, N = c->num_sms;
+        if (C <= N || C % N == 0) return false;
+        const int64_t cut = ceil_div(C % N, hkv);  // lightest pairs moved to the tail launch
+        if (cut >= n_pairs) return false;
+        const int64_t ktiles = ceil_div(len, kBN);
+        double wa = 0.0, wb = 0.0;  // mean key tiles of a pair in the first / tail launch
+        for (int64_t pp = 0; pp < n_pairs; ++pp) {
+            const int64_t q_last = std::min<int64_t>((std::min(2 * pp + 1, nqt - 1) + 1) * bmq, it.n_q) - 1;
+            const double t = static_cast<double>(ceil_div(len - it.n_q + q_last + 1, kBN));
+            (pp < cut ? wb : wa) += t;
+        }
+        wa /= static_cast<double>(n_pairs - cut);
+        wb /= static_cast<double>(cut);
+        const int64_t qt_b = std::min<int64_t>(nqt, 2 * cut);
+        const int64_t row_bytes = static_cast<int64_t>(d) * 4 + 4;
+        const double t_a = std::ceil(static_cast<double>(C - cut * hkv) / N) * (wa + 2.0) * 1.5e-6;
+        double best_t = 1e30;
+        for (int64_t sp = 2; sp <= std::min<int64_t>(128, std::max<int64_t>(2, ktiles / 4)); ++sp) {
+            if (qt_b * hkv * sp * kBM * row_bytes > c->ws_bytes) break;
+            const double waves = std::ceil(static_cast<double>(cut * hkv * sp) / N);
+            const double t = t_a + waves * (wb / sp + 2.0) * 1.5e-6 +
+                             static_cast<double>(qt_b * hkv * kBM * sp * row_bytes * 2) / 6.0e12 + 10e-6;
+            if (t < best_t) {
+                best_t = t;
+                tp.splits = sp;
+            }
+        }
+        if (tp.splits == 0 || best_t > 0.95 * plan_est) return false;
+        tp.pairs = cut;
+        tp.qtiles = qt_b;
+        tp.split_tiles = ceil_div(ktiles, tp.splits);
+        return true;
+    };
+
     std::vector<char> pbuf(sizeof(AttnParams));
     AttnParams &p = *reinterpret_cast<AttnParams *>(pbuf.data());
     for (size_t lo = 0; lo < order.size(); lo += kMaxSegs) {
@@ -730,13 +778,43 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         bool split = false;
         s = plan_group(lo, hi, p, split);
         if (s != PE_OK) return s;
-        c->last_split = split ? 1 : 0;
-        c->last_splits = split ? p.seqs[0].n_splits : 1;
-        c->last_ctas = p.total_items;
+        TailPlan tp;
+        const bool tail = hi - lo == 1 && c->splitkv == -1 && c->num_splits == 0 && plan_tail(order[lo], tp);
+        if (tail && split) {  // the first launch runs unsplit: re-plan the group without splits
+            const int saved = c->splitkv;
+            c->splitkv = 0;
+            s = plan_group(lo, hi, p, split);
+            c->splitkv = saved;
+            if (s != PE_OK) return s;
+        }
+        if (tail) p.total_items -= static_cast<int32_t>(tp.pairs * hkv);  // pairs [cut, n_pairs), heaviest first
+        c->last_split = split || tail ? 1 : 0;
+        c->last_splits = tail ? static_cast<int32_t>(tp.splits) : (split ? p.seqs[0].n_splits : 1);
+        c->last_ctas = p.total_items + (tail ? static_cast<int32_t>(tp.pairs * hkv * tp.splits) : 0);
         cudaError_t e = launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, p, st);
         if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
         c->launches++;
         if (split) {
+            e = launch_splitkv_combine(d, p, st);
+            if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
+            c->launches++;
+        }
+        if (tail) {
+            // the lightest pairs [0, cut), keys split over the SMs, merged by the combine kernel
+            AttnSeq &q = p.seqs[0];
+            q.pair_top = static_cast<int32_t>(tp.pairs);
+            q.n_splits = static_cast<int32_t>(tp.splits);
+            q.item0 = 0;
+            q.part_row0 = 0;
+            q.comb0 = 0;
+            p.split_tiles = static_cast<int32_t>(tp.split_tiles);
+            p.total_items = static_cast<int32_t>(tp.pairs * hkv * tp.splits);
+            p.total_comb = static_cast<int32_t>(tp.qtiles * hkv * kBM);  // q-tiles [0, 2 cut)
+            p.part_o = c->d_ws;
+            p.part_lse = c->d_ws + tp.qtiles * hkv * tp.splits * kBM * d;
+            e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, p, st);
+            if (e != cudaSuccess) return cuda_fail(e, "replay attention tail launch");
+            c->launches++;
             e = launch_splitkv_combine(d, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
             c->launches++;
@@ -1249,6 +1327,7 @@ pe_status pe_replay_attn_static_scratch(pe_cache *c, int32_t seq, int32_t layer,
     q.n_keys = static_cast<int32_t>(c->len[seq]);
     q.n_qtiles = static_cast<int32_t>(n_qtiles);
     q.n_splits = static_cast<int32_t>(n_splits);
+    q.pair_top = static_cast<int32_t>(ceil_div(n_qtiles, 2));
     const int64_t prow = n_qtiles * hkv * n_splits * kBM;
     p.total_items = static_cast<int32_t>(ceil_div(n_qtiles, 2) * hkv * n_splits);
     p.total_comb = static_cast<int32_t>(n_qtiles * hkv * kBM);

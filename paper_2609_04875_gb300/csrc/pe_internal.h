@@ -80,7 +80,8 @@ struct AttnSeq {
     int32_t n_splits;      // key splits per q-tile (1 without split-KV)
     int64_t part_row0;     // first partial row in the workspace (split-KV)
     int32_t comb0;         // first combine row item (split-KV)
-    int32_t pad_;
+    int32_t pair_top;      // the launch covers q-tile pairs [pair_top - items / (Hkv x splits), pair_top),
+                           // heaviest first (pair_top = all pairs, unless a tail launch takes the lightest)
 };
 
 struct AttnParams {

@@ -136,7 +136,7 @@ def test_long_suffix():
     _check_attention(drv, inputs, range(len(w.agents)), [0], n_random=32)
 
 
-@pytest.mark.parametrize("ratio", [0.1, 0.9])
+@pytest.mark.parametrize("ratio", [0.1, 0.7, 0.9])
 def test_tau_sweep(ratio):
     w = synth.tau_sweep(ratio)
     drv, inputs = _run(w)
