@@ -187,10 +187,10 @@ def oracle_tokens_per_s(w, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "agent_batch": {"bytes": 696.263168e6 + 328.400896e6, "profile": "profiles/replay_attn_agent_batch.md",
-                    "src_sha256": "f24199d153228f547845e9ee5201ad6f0b528bee5df3e682544ec0496351f98b"},
-    "short_suffix": {"bytes": 1.076231e9 + 21.225984e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
-                     "src_sha256": "f24199d153228f547845e9ee5201ad6f0b528bee5df3e682544ec0496351f98b"},
+    "agent_batch": {"bytes": 696.787712e6 + 328.413184e6, "profile": "profiles/replay_attn_agent_batch.md",
+                    "src_sha256": "7189e778c5f940b1c537cf93b422f5087750bc5f64e748a579bd47bb8bdff10d"},
+    "short_suffix": {"bytes": 1.076235e9 + 21.172736e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
+                     "src_sha256": "7189e778c5f940b1c537cf93b422f5087750bc5f64e748a579bd47bb8bdff10d"},
     "decode_batch": {"bytes": 342.246144e6 + 4.516864e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernel": "decode",
                      "src_sha256": "f1ad7fd4cc5e0b150afbdab37a0c8c662e01f9f53786b5c5fd49539b343492ed"},
