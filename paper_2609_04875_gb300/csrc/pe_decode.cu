@@ -455,9 +455,10 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 // first (every full chunk, then the items' shorter remainders by decreasing
 // length), so the chunks taken last are the short ones and the CTAs finish
 // close together.  A chunk that is a whole item is written directly; otherwise
-// each chunk writes a partial (O, m, l) and the last of an item's chunks to
-// finish merges them (ticket counter), in the item's chunk order.  The last
-// CTA to stop taking chunks resets the chunk counter for the next launch.
+// each chunk writes a partial (O, m, l) and a combine launch that follows
+// (programmatic serialization, so its launch overlaps this grid's end) merges
+// an item's partials in the item's chunk order.  The last CTA to stop taking chunks resets the
+// chunk counter for the next launch.
 //
 // Roles (384 threads):
 //   warps 0-3  softmax: thread t = key t of the tile (TMEM lane t); masks,
@@ -467,7 +468,7 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 //   warps 7-10 epilogue: thread = d-column (TMEM lane); per chunk, reads O^T
 //              (double-buffered in TMEM, so the next chunk accumulates into
 //              the other buffer meanwhile), writes the output or the chunk's
-//              partial, takes the item's ticket and merges when last.
+//              partial.
 //   warp 11    scheduler + page-id loader: takes chunk ids (one chunk ahead of
 //              the producers) into a ring that the MMA issuer and the softmax
 //              warps read, turns each chunk's page ids into TMA row
@@ -488,7 +489,6 @@ constexpr int kTcKeys = 128;
 constexpr int kTcKStages = 3;                      // K ring (32 KB stages)
 constexpr int kTcVStages = 3;                      // V ring
 constexpr int kTcThreads = 384;
-constexpr int kBarEpilogue = 3;                    // named barrier of the epilogue warps
 constexpr int kChunkRing = 4;                      // chunk ids in flight between the roles
 constexpr int kDescRing = 2;                       // chunk descriptors (TMA rows) for the producers
 constexpr int kDescInts = 8 + 8 * 16;              // header, then the row of box (tile k, slot j) at 8 + 16 k + j
@@ -507,11 +507,10 @@ struct TcCfg {
     // k_full[KS], k_empty[KS], v_full[VS], v_empty[VS], s_full[2], p_full[2], o_done[2], q_ready[2], drain,
     // ch_full[R], ch_empty[R], o_item[2], o_free[2], stats[2], desc_full[D], desc_empty[D], q_free[2]
     static constexpr int kNumBars = 2 * (kTcKStages + kTcVStages) + 9 + 2 * kChunkRing + 8 + 2 * kDescRing;
-    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort, ticket, K / V tiles issued, chunk ring
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort, K / V tiles issued, chunk ring
     static constexpr int kOffStats = kOffMisc + 32 + 4 * kChunkRing;  // [2][id, m[RB], l[RB]] per chunk parity
     static constexpr int kStatsFloats = 1 + 2 * RB;
-    static constexpr int kOffMerge = kOffStats + 2 * kStatsFloats * 4;  // merge staging: m[32], l[32]
-    static constexpr int kOffSeqs = kOffMerge + 64 * 4;     // the launch's sequence table
+    static constexpr int kOffSeqs = kOffStats + 2 * kStatsFloats * 4;  // the launch's sequence table
     static constexpr int kOffDesc = kOffSeqs + kMaxSegs * static_cast<int>(sizeof(DecodeSeq) + 4);  // + rem_seq
     static constexpr int kSmem = kOffDesc + kDescRing * kDescInts * 4;
     static constexpr int kDynSmem = kSmem + 1024;
@@ -523,10 +522,9 @@ struct TcCfg {
 // A chunk: tiles [t0, t1) of item (sequence si, kv-head kvh).  An item has
 // nfull full chunks (ids first .. first + nfull - 1) and, when its tile count
 // is not a multiple of the chunk size, one shorter remainder chunk (id rem);
-// id(k) is the item's k-th chunk, k < cpi.
+// cpi chunks in all.
 struct ChunkInfo {
     int si, kvh, t0, t1, cpi, first, nfull, rem;
-    __device__ __forceinline__ int id(int k) const { return k < nfull ? first + k : rem; }
 };
 
 __device__ __forceinline__ int tc_tiles(const DecodeSeq &sq) { return (sq.n_keys + kTcKeys - 1) / kTcKeys; }
@@ -607,10 +605,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const uint32_t b_desc_empty = b_desc_full + 8 * kDescRing;   // [D] both producers have issued that chunk
     const uint32_t b_q_free = b_desc_empty + 8 * kDescRing;      // [2] every S^T reading that Q buffer is done
     float *s_stats = reinterpret_cast<float *>(smem + C::kOffStats);
-    float *s_merge = reinterpret_cast<float *>(smem + C::kOffMerge);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 4);
-    int *s_ticket = reinterpret_cast<int *>(smem + C::kOffMisc + 8);
     volatile int *s_issued = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 12);  // [2]: K, V
     volatile int *s_chunk = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 32);  // [R]
     DecodeSeq *s_seqs = reinterpret_cast<DecodeSeq *>(smem + C::kOffSeqs);
@@ -1083,7 +1079,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int t = q4 * 32 + lane;                  // d-column
         const int et = (warp - 7) * 32 + lane;         // thread index within the epilogue group
         const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-        int *e_ticket = reinterpret_cast<int *>(smem + C::kOffMisc + 20);
         for (int n = 0;; ++n) {
             if (!wait_bar_warp(b_stats + 8 * (n & 1), (n >> 1) & 1, wctx)) break;
             const float *st = s_stats + (n & 1) * C::kStatsFloats;
@@ -1117,7 +1112,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
                 continue;
             }
-            // partial of chunk c; the last of the item's chunks to finish merges, in the item's chunk order
+            // partial of chunk c (O / l unnormalised, with its reference m and sum l); the combine
+            // launch that follows merges an item's partials
             float *po = p.part + static_cast<int64_t>(c) * RB * HD;
             float *pm = p.part + static_cast<int64_t>(p.total_tiles) * RB * HD;
             float *pl = pm + static_cast<int64_t>(p.total_tiles) * RB;
@@ -1134,87 +1130,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 pm[static_cast<int64_t>(c) * RB + et] = mv;
                 pl[static_cast<int64_t>(c) * RB + et] = lv;
             }
-            ptx::bar_sync(kBarEpilogue, 128);  // every thread's partial is written
-            int32_t *ticket = p.tickets + ci.si * p.hkv + ci.kvh;
-            if (et == 0) {
-                __threadfence();  // the CTA's partial before its ticket
-                *e_ticket = atomicAdd(ticket, 1);
-            }
-            ptx::bar_sync(kBarEpilogue, 128);
-            const bool merge = *e_ticket == ci.cpi - 1;
-            ptx::bar_sync(kBarEpilogue, 128);  // e_ticket is reused
-            if (!merge) continue;
-            __threadfence();
-            // merge in batches of kOB chunks, one round of loads each: thread et < nb RB loads one (m, l)
-            // pair (staged in shared memory for every thread), and every thread its d-column of each
-            // chunk's O, all issued together; M = max_k m_k, O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k
-            constexpr int kOB = 32 / RB;  // chunks per batch (32 O values per thread in registers)
-            float mx[RB], den[RB], acc[RB];
-#pragma unroll
-            for (int r = 0; r < RB; ++r) {
-                mx[r] = -INFINITY;
-                den[r] = 0.f;
-                acc[r] = 0.f;
-            }
-            float *s_m = s_merge;
-            float *s_l = s_merge + 32;
-            for (int k0 = 0; k0 < ci.cpi; k0 += kOB) {
-                const int nb = min(kOB, ci.cpi - k0);
-                float mv = -INFINITY, lv = 0.f;
-                if (et < nb * RB) {
-                    const int kb = et / RB;
-                    const int64_t sl = static_cast<int64_t>(ci.id(k0 + kb)) * RB + (et - kb * RB);
-                    mv = __ldcg(pm + sl);
-                    lv = __ldcg(pl + sl);
-                }
-                float ov[kOB][RB];
-#pragma unroll
-                for (int u = 0; u < kOB; ++u)
-#pragma unroll
-                    for (int r = 0; r < RB; ++r)
-                        ov[u][r] = u < nb ? __ldcg(p.part + (static_cast<int64_t>(ci.id(k0 + u)) * RB + r) * HD + t)
-                                          : 0.f;
-                if (et < nb * RB) {
-                    s_m[et] = mv;
-                    s_l[et] = lv;
-                }
-                ptx::bar_sync(kBarEpilogue, 128);
-                float bmx[RB];
-#pragma unroll
-                for (int r = 0; r < RB; ++r) bmx[r] = -INFINITY;
-#pragma unroll
-                for (int u = 0; u < kOB; ++u)
-#pragma unroll
-                    for (int r = 0; r < RB; ++r)
-                        if (u < nb) bmx[r] = fmaxf(bmx[r], s_m[u * RB + r]);
-#pragma unroll
-                for (int r = 0; r < RB; ++r) {  // rescale the running sums to the new max
-                    const float mn = fmaxf(mx[r], bmx[r]);
-                    const float f = (mx[r] == -INFINITY || mn == -INFINITY) ? 0.f : ex2(mx[r] - mn);
-                    den[r] *= f;
-                    acc[r] *= f;
-                    mx[r] = mn;
-                }
-#pragma unroll
-                for (int u = 0; u < kOB; ++u)
-#pragma unroll
-                    for (int r = 0; r < RB; ++r) {
-                        if (u >= nb) continue;
-                        const float ms = s_m[u * RB + r];
-                        const float w = (ms == -INFINITY || mx[r] == -INFINITY) ? 0.f : ex2(ms - mx[r]);
-                        den[r] += w * s_l[u * RB + r];
-                        acc[r] += w * ov[u][r];
-                    }
-                ptx::bar_sync(kBarEpilogue, 128);  // the staging area is reused
-            }
-#pragma unroll
-            for (int r = 0; r < RB; ++r) {
-                if (r >= n_rows) continue;
-                const float inv = den[r] > 0.f ? 1.0f / den[r] : 0.f;
-                static_cast<__nv_bfloat16 *>(p.out)[(static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + ci.kvh * g +
-                                                     r % g) * HD + t] = __float2bfloat16_rn(acc[r] * inv);
-            }
-            if (et == 0) *ticket = 0;
         }
     }
 
@@ -1241,6 +1156,79 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
 }
 
+// Merge of an item's chunk partials (one block per (sequence, kv-head), thread = d-column), after
+// the decode kernel: M = max_k m_k, O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k over the item's
+// chunks in its chunk order.  Items held in one chunk were written by the decode kernel itself.
+template <int RB>
+__global__ void __launch_bounds__(128) decode_tc_combine_kernel(const __grid_constant__ DecodeParams p)
+{
+    constexpr int HD = 128;
+    ptx::griddep_wait();  // launched with programmatic serialization: the decode kernel's partials
+    const int si = static_cast<int>(blockIdx.x) / p.hkv;
+    const int kvh = static_cast<int>(blockIdx.x) - si * p.hkv;
+    if (si >= p.n_seqs) return;
+    const DecodeSeq &sq = p.seqs[si];
+    const int nt = tc_tiles(sq);
+    const int nfull = nt / sq.cta0;
+    const int first = sq.tile0 + kvh * nfull;
+    const int rem = sq.rem0 >= 0 ? sq.rem0 + kvh : -1;
+    const int cpi = nfull + (rem >= 0 ? 1 : 0);
+    if (cpi <= 1) return;
+    const int g = p.group;
+    const int n_rows = sq.n_q * g;
+    const int t = static_cast<int>(threadIdx.x);
+    const float *pm = p.part + static_cast<int64_t>(p.total_tiles) * RB * HD;
+    const float *pl = pm + static_cast<int64_t>(p.total_tiles) * RB;
+    // batches of kOB chunks, every load of a batch issued together (m and l are the same for
+    // every thread: broadcast reads)
+    constexpr int kOB = 32 / RB;
+    float mx[RB], den[RB], acc[RB];
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+        mx[r] = -INFINITY;
+        den[r] = 0.f;
+        acc[r] = 0.f;
+    }
+    for (int k0 = 0; k0 < cpi; k0 += kOB) {
+        float mv[kOB][RB], lv[kOB][RB], ov[kOB][RB];
+#pragma unroll
+        for (int u = 0; u < kOB; ++u) {
+            const int k = k0 + u;
+            const int64_t c = k < nfull ? first + k : rem;
+#pragma unroll
+            for (int r = 0; r < RB; ++r) {
+                const bool in = k < cpi && r < n_rows;
+                mv[u][r] = in ? __ldcg(pm + c * RB + r) : -INFINITY;
+                lv[u][r] = in ? __ldcg(pl + c * RB + r) : 0.f;
+                ov[u][r] = in ? __ldcg(p.part + (c * RB + r) * HD + t) : 0.f;
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < RB; ++r) {
+            float bmx = mx[r];
+#pragma unroll
+            for (int u = 0; u < kOB; ++u) bmx = fmaxf(bmx, mv[u][r]);
+            const float f = (mx[r] == -INFINITY || bmx == -INFINITY) ? 0.f : ex2(mx[r] - bmx);
+            den[r] *= f;
+            acc[r] *= f;
+            mx[r] = bmx;
+#pragma unroll
+            for (int u = 0; u < kOB; ++u) {
+                const float w = (mv[u][r] == -INFINITY || bmx == -INFINITY) ? 0.f : ex2(mv[u][r] - bmx);
+                den[r] += w * lv[u][r];
+                acc[r] += w * ov[u][r];
+            }
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+        if (r >= n_rows) continue;
+        const float inv = den[r] > 0.f ? 1.0f / den[r] : 0.f;
+        static_cast<__nv_bfloat16 *>(p.out)[(static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + kvh * g + r % g) * HD +
+                                            t] = __float2bfloat16_rn(acc[r] * inv);
+    }
+}
+
 template <int RB>
 cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st)
 {
@@ -1263,7 +1251,17 @@ cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const De
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<RB>, tm_k, tm_v, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<RB>, tm_k, tm_v, p);
+    if (e != cudaSuccess) return e;
+    // the merges, also with programmatic serialization (its launch overlaps the decode grid's end)
+    cudaLaunchConfig_t ccfg = {};
+    ccfg.gridDim = dim3(static_cast<unsigned>(p.n_seqs * p.hkv));
+    ccfg.blockDim = dim3(128);
+    ccfg.dynamicSmemBytes = 0;
+    ccfg.stream = st;
+    ccfg.attrs = attr;
+    ccfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&ccfg, decode_tc_combine_kernel<RB>, p);
 }
 
 template <int HD, int RB>
