@@ -252,10 +252,12 @@ def roofline_for(w, flops_launch, bytes_launch, attn_s, peaks, peak_src, plan=(F
     rows = max(a.S for a in w.agents) * (w.num_q_heads // w.num_kv_heads)
     if rows <= 16:  # every sequence's query rows fit the decode kernel
         rb = 4 if rows <= 4 else (8 if rows <= 8 else 16)
-        name = f"decode_tc_kernel<{rb}>" if w.head_dim == 128 else f"decode_attn_kernel<{w.head_dim},{rb}>"
-        r["kernel"] = f"{name} (split-KV merged in-kernel)"
+        if w.head_dim == 128:
+            r["kernel"] = f"decode_tc_kernel<{rb}> (+ decode_tc_combine_kernel<{rb}> for split items)"
+        else:
+            r["kernel"] = f"decode_attn_kernel<{w.head_dim},{rb}> (split-KV merged in-kernel)"
     else:
-        r["kernel"] = f"replay_attn_kernel<{w.head_dim},{'split' if plan[0] else 'single'}>"
+        r["kernel"] = f"replay_attn_kernel<{w.head_dim},{'split' if plan[0] else 'single'}> (+ splitkv_combine when split)"
     r["plan"] = {"split_kv": plan[0], "key_splits": plan[1], "ctas": plan[2]}
     r["attn_ms_per_launch"] = attn_s * 1e3
     r["algorithmic_flop_per_launch"] = flops_launch
