@@ -625,7 +625,8 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
 
     // split-KV decision over the whole launch group; plan_est: the cost model's time of the plan
     double plan_est = 0.0;
-    auto plan_group = [&](size_t lo, size_t hi, AttnParams &p, bool &split) -> pe_status {
+    // splitkv: the "splitkv" option's value for this plan (-1 auto, 0 never, 1 always)
+    auto plan_group = [&](size_t lo, size_t hi, AttnParams &p, bool &split, int splitkv) -> pe_status {
         // C CTAs (pairs of q-tiles x kv-heads), W key tiles per CTA on average.
         int64_t C = 0, tiles = 0, rows = 0, valid_rows = 0, max_tiles = 0;
         for (size_t i = lo; i < hi; ++i) {
@@ -654,20 +655,20 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             return t;
         };
         int64_t best = 1;
-        if (c->splitkv != 0) {
+        if (splitkv != 0) {
             const int64_t s_max = std::min<int64_t>(128, std::max<int64_t>(1, max_tiles / 4));
-            double best_t = c->splitkv == 1 ? 1e30 : cost(1);
+            double best_t = splitkv == 1 ? 1e30 : cost(1);
             for (int64_t sp = 2; sp <= s_max; ++sp) {
                 if (rows * sp * row_bytes > c->ws_bytes) break;
                 const double t = cost(sp);
                 if (t < best_t) { best_t = t; best = sp; }
             }
-            if (c->splitkv == -1 && best > 1 && best_t > 0.95 * cost(1)) best = 1;  // keep the single pass unless clearly faster
+            if (splitkv == -1 && best > 1 && best_t > 0.95 * cost(1)) best = 1;  // keep the single pass unless clearly faster
         }
-        if (c->splitkv != 0 && c->num_splits > 0) best = c->num_splits;
+        if (splitkv != 0 && c->num_splits > 0) best = c->num_splits;
         plan_est = cost(best);
         int split_tiles = static_cast<int>(max_tiles);
-        split = best > 1 || c->splitkv == 1;
+        split = best > 1 || splitkv == 1;
         if (split) split_tiles = static_cast<int>(std::max<int64_t>(1, ceil_div(max_tiles, std::max<int64_t>(best, 1))));
         std::memset(&p, 0, sizeof p);
         p.page_table = c->d_table;
@@ -776,15 +777,12 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     for (size_t lo = 0; lo < order.size(); lo += kMaxSegs) {
         const size_t hi = std::min(order.size(), lo + kMaxSegs);
         bool split = false;
-        s = plan_group(lo, hi, p, split);
+        s = plan_group(lo, hi, p, split, c->splitkv);
         if (s != PE_OK) return s;
         TailPlan tp;
         const bool tail = hi - lo == 1 && c->splitkv == -1 && c->num_splits == 0 && plan_tail(order[lo], tp);
         if (tail && split) {  // the first launch runs unsplit: re-plan the group without splits
-            const int saved = c->splitkv;
-            c->splitkv = 0;
-            s = plan_group(lo, hi, p, split);
-            c->splitkv = saved;
+            s = plan_group(lo, hi, p, split, 0);
             if (s != PE_OK) return s;
         }
         if (tail) p.total_items -= static_cast<int32_t>(tp.pairs * hkv);  // pairs [cut, n_pairs), heaviest first
