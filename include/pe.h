@@ -269,9 +269,11 @@ pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *
 pe_status pe_selftest_bounded_wait(pe_cache *cache, int64_t limit_ns, void *stream);
 
 /* Plan of the most recent replay-attention launch group on this cache: split
- * = 1 when the split-KV path ran (the tensor-core kernel's combine launch, or
- * the decode kernel's in-kernel merge), n_splits = key splits of its first
- * sequence, ctas = attention CTAs launched. */
+ * = 1 when the split-KV path ran (a combine launch followed the attention, or
+ * the CUDA-core decode kernel merged in-kernel), n_splits = key splits of its
+ * first sequence (of the tail launch, when one ran: a group of one sequence
+ * whose last wave of CTAs would be mostly empty runs its lightest q-tile pairs
+ * in a second, split-KV launch), ctas = attention CTAs launched in all. */
 pe_status pe_last_attn_plan(const pe_cache *cache, int32_t *split, int32_t *n_splits, int32_t *ctas);
 
 /* Number of kernel launches this cache has made so far (crop, append,
