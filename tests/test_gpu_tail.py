@@ -16,8 +16,7 @@ from gpu_common import Pair, assert_close, dev, requires_cuda
 pytestmark = [pytest.mark.gpu, requires_cuda]
 
 
-def _case(n_q, prefix, seed):
-    d, hq, hkv, ps = 128, 32, 8, 16
+def _case(n_q, prefix, seed, d=128, hq=32, hkv=8, ps=16):
     n = prefix + n_q
     npg = -(-n // ps) + 4
     pair = Pair(1, hkv, d, ps, npg, 1, npg, seed=seed)
@@ -28,15 +27,16 @@ def _case(n_q, prefix, seed):
     return pair, s, q
 
 
-@pytest.mark.parametrize("n_q,prefix", [(1280, 4096), (1344, 3000)])
-def test_tail_launch_matches_oracle(n_q, prefix):
+@pytest.mark.parametrize("n_q,prefix,d,hq", [(1280, 4096, 128, 32), (1344, 3000, 128, 32), (5120, 2048, 64, 8)])
+def test_tail_launch_matches_oracle(n_q, prefix, d, hq):
     """20 (or 21) q-tile pairs x 8 kv-heads = 160 (168) CTAs on 152 SMs: the lightest pair(s) move
-    to the split-KV tail launch."""
-    pair, s, q = _case(n_q, prefix, seed=n_q)
-    scale = 1 / math.sqrt(128)
-    g4 = 4                                      # q-heads per kv-head: 32 queries per 128-row q-tile
-    tail_rows = np.arange(0, 64 * 2)            # the two lightest pairs' queries: every row
-    rest = np.unique(np.concatenate([np.arange(128, n_q, 31), [n_q - 1]]))
+    to the split-KV tail launch (d = 128 with 4 q-heads per kv-head; d = 64 with one)."""
+    pair, s, q = _case(n_q, prefix, seed=n_q, d=d, hq=hq)
+    scale = 1 / math.sqrt(d)
+    g4 = hq // 8                                # q-heads per kv-head
+    bmq = 128 // g4                             # queries per 128-row q-tile
+    tail_rows = np.arange(0, 4 * bmq)           # the two lightest pairs' queries: every row
+    rest = np.unique(np.concatenate([np.arange(4 * bmq, n_q, 31), [n_q - 1]]))
     rows = np.concatenate([tail_rows, rest])
     ref = oracle.replay_attention(pair.orc, s, 0, q, scale, rows=rows)
     out = pair.gpu.replay_attn(s, 0, dev(q))
