@@ -3,7 +3,8 @@ never to itself.  Each pin takes the oracle *module* so that the mutation tests
 can run the same pins against copies of the oracle with a planted mistake.
 
   pin_bruteforce   - a separately written dense masked softmax (numpy einsum
-                     over contiguous arrays) on tiny paged crop+replay cases
+                     over contiguous arrays) on tiny paged crop+replay cases,
+                     for every query row and for a subset of rows in reverse
   pin_library      - P = 0 (plain causal self-attention) against torch's SDPA
                      in float64, a library routine
   pin_closed_forms - one key, constant V, Q = 0, one dominant logit, and a
@@ -94,6 +95,11 @@ def pin_bruteforce(orc, full=True):
                         assert np.allclose(got, want, rtol=1e-12, atol=1e-12), \
                             f"brute force mismatch ps={ps} hq={hq} hkv={hkv} d={d} T={T} tau={tau}: " \
                             f"{np.max(np.abs(got - want))}"
+                        if S >= 2:  # a subset of query rows, last first, against the same dense rows
+                            sub = np.arange(S - 1, -1, -2)
+                            got_sub = orc.replay_attention(c, s, 0, qc[:S], scale, rows=sub)
+                            assert np.allclose(got_sub, want[sub], rtol=1e-12, atol=1e-12), \
+                                f"row-subset mismatch ps={ps} hq={hq} hkv={hkv} d={d} T={T} tau={tau}"
 
 
 def pin_library(orc):

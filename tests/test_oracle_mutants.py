@@ -20,6 +20,12 @@ MUTANTS = [
     ("top_left_alignment", "attention.c", "const int64_t a = jb->n_keys - jb->n_q + i;", "const int64_t a = i;"),
     ("value_from_keys", "attention.c", "const uint16_t *vrow = jb->v +", "const uint16_t *vrow = jb->k +"),
     ("unnormalised", "attention.c", "o[c] /= den;", "o[c] /= 1.0;"),
+    ("keys_head_major", "attention.c", "jb->k + (j * jb->hkv + kvh) * (int64_t)d",
+     "jb->k + (kvh * jb->n_keys + j) * (int64_t)d"),
+    ("query_from_output_row", "attention.c", "jb->q + (i * jb->hq + h) * (int64_t)d",
+     "jb->q + (r * jb->hq + h) * (int64_t)d"),
+    ("output_head_major", "attention.c", "jb->out + (r * jb->hq + h) * (int64_t)d",
+     "jb->out + (h * jb->n_rows + r) * (int64_t)d"),
     ("crop_keeps_tau", "kvcache.py", "new_len = tau - 1\n", "new_len = min(tau, n)\n"),
     ("push_ascending", "kvcache.py", "for p in reversed(pages):", "for p in pages:"),
     ("slot_shift", "kvcache.py", "page, slot = tbl[pos // self.ps], pos % self.ps",
