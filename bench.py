@@ -669,7 +669,7 @@ def run_reference(args, rank, world):
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "f64",
-        "data": "synthetic (seeded N(0,1)/sqrt(128) bf16 Q/K/V; no dataset)",
+        "data": f"synthetic (seeded N(0,{w.std:.4g}^2) bf16 Q/K/V; no dataset)",
         "config": {**w.describe(), "parallelism": "host cores (oracle)"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                          "sample": f"per step: {samples[-1]}"},

@@ -29,3 +29,27 @@ def test_kernel_source_spans_are_found():
     for wl, t in bench.NCU_TRAFFIC.items():
         assert t.get("kernel", "prefill") in bench.KERNEL_SRC, wl
         assert t["bytes"] > 0 and t["profile"].startswith("profiles/"), wl
+
+
+def test_reference_arm_prints_one_contract_line():
+    """`bench.py --impl reference` times the fp64 oracle on the host cores and prints one JSON line
+    with the contract's keys; it needs no GPU."""
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "2", "--warmup", "1", "--ref-step-budget", "0.3"],
+                       capture_output=True, text=True, timeout=300, cwd=root)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["steps"] == 2 and d["warmup"] == 1 and d["n_gpus"] == 1
+    assert d["value"] > 0 and d["higher_is_better"] is True and d["config"]["workload"] == "tiny"
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
+    assert d["cpu_baseline"]["value"] == d["value"] and d["e2e"]["value"] == d["value"]
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
+    assert d["unit"] == d["e2e"]["unit"] == d["cpu_baseline"]["unit"]
+    assert "N(0,1^2)" in d["data"]  # the tiny workload draws unscaled N(0, 1) values
