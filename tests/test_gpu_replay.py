@@ -53,10 +53,14 @@ def test_peaked_logits_exercise_rescaling(scale_mult):
 
 
 @pytest.mark.parametrize("split", [0, 1])
-def test_reference_moves_on_large_jump(split):
-    """Keys after the first 128 are scaled by 16 (exact in bf16), so for nearly
+@pytest.mark.parametrize("jump", [128, 192])
+def test_reference_moves_on_large_jump(split, jump):
+    """Keys from `jump` on are scaled by 16 (exact in bf16), so for nearly
     every row a later tile's logits exceed the first tile's max by far more
-    than 64 in log2 units: the row's reference must move and O be rescaled."""
+    than 64 in log2 units: the row's reference must move and O be rescaled.
+    At 128 the jump starts a key tile; at 192 it falls in the middle of one,
+    so that tile mixes weights near the old reference with weights far above
+    it."""
     d, hq, hkv, ps, P, S = 128, 32, 8, 16, 600, 100
     T = P + S
     npg = -(-T // ps) + 3
@@ -66,7 +70,7 @@ def test_reference_moves_on_large_jump(split):
     g = synth.rng(61, 1)
     f = synth.bf16_bits_to_f32
     k0 = f(synth.normal_bf16(g, (1, T, hkv, d)))
-    k0[:, 128:] *= 16.0
+    k0[:, jump:] *= 16.0
     k0 = synth.f32_to_bf16_bits(k0)
     v0 = synth.normal_bf16(g, (1, T, hkv, d))
     q = synth.normal_bf16(g, (S, hq, d))
@@ -76,7 +80,7 @@ def test_reference_moves_on_large_jump(split):
     out = pair.gpu.replay_attn(s, 0, dev(q), softmax_scale=scale)
     ref = oracle.replay_attention(pair.orc, s, 0, q, scale)
     vmax = float(np.abs(f(v0)).max())
-    assert_within_rounding_bound(out, ref, vmax, f"large jump split={split}")
+    assert_within_rounding_bound(out, ref, vmax, f"large jump at {jump} split={split}")
 
 
 def test_multilayer_and_pool_contents():
