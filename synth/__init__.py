@@ -5,16 +5,24 @@ it holds none of the method's arithmetic (no attention, no paging policy).
 Tests, the benchmark and the smoke check import it to feed the CUDA library and
 the fp64 oracle the very same bf16 bit patterns.
 
-Values are drawn with numpy's PCG64 generator (``SeedSequence([base, stream,
-index])``) as float32 standard normals, multiplied by the workload's standard
-deviation in float32 and rounded once to bf16 (round-to-nearest-even).  Every
-independent quantity has its own stream so that, e.g., the counterfactual
-suffix of an agent never shares draws with its original ("contaminated")
-suffix.
+Values are drawn with numpy's PCG64 generator as float32 standard normals,
+multiplied by the workload's standard deviation in float32 and rounded once to
+bf16 (round-to-nearest-even).  Every independent quantity has its own stream so
+that, e.g., the counterfactual suffix of an agent never shares draws with its
+original ("contaminated") suffix.
+
+A workload's per-position tensors (K, V, Q of a session) are drawn in blocks
+of ``SESSION_BLOCK`` positions of one layer, each block from its own generator
+``SeedSequence([base, stream, agent, tensor, layer, block])``.  The value at a
+position therefore does not depend on which range of positions is asked for
+(the sanitized suffix of any tau is a slice of one sanitized session), and the
+blocks are drawn on all host cores at once.
 """
 from __future__ import annotations
 
 import math
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -26,7 +34,6 @@ STREAM_PERM = 1          # physical page pop order of the pool
 STREAM_KV_ORIG = 2       # K/V of the original session, positions [0, T)
 STREAM_KV_CF = 3         # K'/V' of the counterfactual (sanitized) suffix
 STREAM_Q_CF = 4          # Q' of the counterfactual suffix
-STREAM_Q_PREFIX = 5      # Q of the prefix positions (full-reset comparator)
 STREAM_LENGTHS = 6       # per-agent T and tau/T (agent batch)
 STREAM_SAMPLE = 7        # query rows sampled for large-size checks
 STREAM_TURNS = 8         # per-agent turn lengths of the suffix (turn-structured workload)
@@ -51,7 +58,11 @@ def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
         raise ValueError("non-finite value in synthetic draw")
     u = x.view(np.uint32)
     # finite inputs: u + 0x8000 stays below 2^32, so uint32 arithmetic is exact
-    r = (u + (np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1)))) >> np.uint32(16)
+    r = u >> np.uint32(16)
+    r &= np.uint32(1)
+    r += np.uint32(0x7FFF)
+    r += u
+    r >>= np.uint32(16)
     return r.astype(np.uint16)
 
 
@@ -73,6 +84,51 @@ def normal_bf16(g: np.random.Generator, shape, std: float = 1.0, chunk: int = 1 
             x = x * s32
         out[lo:hi] = f32_to_bf16_bits(x)
     return out.reshape(shape)
+
+
+SESSION_BLOCK = 256      # positions of one layer drawn from one generator
+
+
+def host_threads() -> int:
+    try:
+        return max(1, len(os.sched_getaffinity(0)))
+    except (AttributeError, OSError):
+        return max(1, os.cpu_count() or 1)
+
+
+def session_bf16(seed: int, stream: int, index: int, tensor: int, num_layers: int, lo: int, hi: int,
+                 width: int, std: float) -> np.ndarray:
+    """Positions [lo, hi) of a per-position session tensor, all layers: bf16 bits
+    [num_layers][hi - lo][width] of i.i.d. N(0, std^2).  Block b of layer l
+    (positions [b B, (b + 1) B), B = SESSION_BLOCK) is drawn whole from
+    SeedSequence([seed, stream, index, tensor, l, b]), so a position's value is
+    the same whatever range contains it."""
+    if not 0 <= lo <= hi:
+        raise ValueError("bad position range")
+    out = np.empty((num_layers, hi - lo, width), dtype=np.uint16)
+    if hi == lo or num_layers == 0 or width == 0:
+        return out
+    B = SESSION_BLOCK
+    s32 = np.float32(std)
+    tasks = [(l, b) for l in range(num_layers) for b in range(lo // B, -(-hi // B))]
+
+    def draw(task):
+        l, b = task
+        g = np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, stream, index, tensor, l, b])))
+        x = g.standard_normal(B * width, dtype=np.float32)
+        if std != 1.0:
+            x *= s32
+        a, z = max(lo, b * B), min(hi, (b + 1) * B)
+        out[l, a - lo:z - lo] = f32_to_bf16_bits(x[(a - b * B) * width:(z - b * B) * width]).reshape(z - a, width)
+
+    n = min(host_threads(), len(tasks))
+    if n <= 1:
+        for t in tasks:
+            draw(t)
+    else:
+        with ThreadPoolExecutor(max_workers=n) as ex:
+            list(ex.map(draw, tasks))
+    return out
 
 
 def page_permutation(seed: int, num_pages: int) -> np.ndarray:
@@ -154,27 +210,25 @@ class Workload:
         }
 
     # -- draws ---------------------------------------------------------------
+    def _session(self, stream, agent, tensor, lo, hi, heads):
+        x = session_bf16(self.seed, stream, agent.index, tensor, self.num_layers, lo, hi, heads * self.head_dim,
+                         self.std)
+        return x.reshape(self.num_layers, hi - lo, heads, self.head_dim)
+
     def kv_original(self, agent: Agent):
-        """K, V of the original session: bf16 bits [L][T][Hkv][d] each."""
-        g = rng(self.seed, STREAM_KV_ORIG, agent.index)
-        shp = (self.num_layers, agent.T, self.num_kv_heads, self.head_dim)
-        return normal_bf16(g, shp, self.std), normal_bf16(g, shp, self.std)
+        """K, V of the original session, positions [0, T): bf16 bits [L][T][Hkv][d] each."""
+        return (self._session(STREAM_KV_ORIG, agent, 0, 0, agent.T, self.num_kv_heads),
+                self._session(STREAM_KV_ORIG, agent, 1, 0, agent.T, self.num_kv_heads))
 
     def kv_counterfactual(self, agent: Agent):
-        """K', V' of the sanitized suffix: bf16 bits [L][S][Hkv][d] each."""
-        g = rng(self.seed, STREAM_KV_CF, agent.index)
-        shp = (self.num_layers, agent.S, self.num_kv_heads, self.head_dim)
-        return normal_bf16(g, shp, self.std), normal_bf16(g, shp, self.std)
+        """K', V' of the sanitized suffix, positions [P, T) of the agent's sanitized
+        session: bf16 bits [L][S][Hkv][d] each."""
+        return (self._session(STREAM_KV_CF, agent, 0, agent.P, agent.T, self.num_kv_heads),
+                self._session(STREAM_KV_CF, agent, 1, agent.P, agent.T, self.num_kv_heads))
 
     def q_counterfactual(self, agent: Agent):
-        """Q' of the sanitized suffix: bf16 bits [L][S][Hq][d]."""
-        g = rng(self.seed, STREAM_Q_CF, agent.index)
-        return normal_bf16(g, (self.num_layers, agent.S, self.num_q_heads, self.head_dim), self.std)
-
-    def q_prefix(self, agent: Agent):
-        """Q of the prefix positions (only the full-reset comparator needs it): [L][P][Hq][d]."""
-        g = rng(self.seed, STREAM_Q_PREFIX, agent.index)
-        return normal_bf16(g, (self.num_layers, agent.P, self.num_q_heads, self.head_dim), self.std)
+        """Q' of the sanitized suffix, positions [P, T): bf16 bits [L][S][Hq][d]."""
+        return self._session(STREAM_Q_CF, agent, 0, agent.P, agent.T, self.num_q_heads)
 
     def init_free_order(self) -> np.ndarray:
         return page_permutation(self.seed, self.num_pages)
@@ -278,6 +332,17 @@ def replica(w: Workload, r: int) -> Workload:
     import copy
     w2 = copy.deepcopy(w)
     w2.seed = seed
+    return w2
+
+
+def with_std(w: Workload, std: float) -> Workload:
+    """The same shapes, lengths and page order with Q/K/V drawn at another
+    standard deviation (std 1: logits q.k / sqrt(d) of standard deviation 1,
+    a sharper softmax than the workloads' own N(0, 1/128) draws)."""
+    import copy
+    w2 = copy.deepcopy(w)
+    w2.std = float(std)
+    w2.name = f"{w.name}_std{std:g}"
     return w2
 
 

@@ -22,3 +22,18 @@ def pytest_sessionstart(session):
     pe_build.build()
     import oracle
     oracle.build()
+
+
+def pytest_sessionfinish(session, exitstatus):
+    # PE_PARITY_REPORT=<file>: the errors of every block the GPU parity tests
+    # checked (absolute and normalised by the oracle's size), one JSON object.
+    path = os.environ.get("PE_PARITY_REPORT")
+    if not path:
+        return
+    try:
+        import gpu_common
+    except Exception:
+        return
+    import json
+    with open(path, "w") as f:
+        json.dump([{"what": w, **e} for w, e in gpu_common.PARITY_LOG], f, indent=0)

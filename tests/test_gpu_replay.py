@@ -43,11 +43,15 @@ def test_peaked_logits_exercise_rescaling(scale_mult):
     """Logit std 4 to 64: running maxima jump between key tiles; at 64 later
     tiles exceed the first tile's max by far more than 2^64 in weight, so the
     reference moves and O in TMEM is rescaled.  The output is then close to
-    single value rows (|O| up to max|V|), so the check uses the derived
-    rounding bound."""
+    single value rows (|O| up to max|V|): at x4 the stated 2e-2 gate still
+    holds and is applied; beyond it the check uses the derived rounding bound
+    (both with the normalised gates)."""
     d = 128
     pair, s, outs, refs, inputs = replay_case(1, 32, 8, d, 16, 700, 300, seed=5, scale=scale_mult / math.sqrt(d),
                                               split=0)
+    if scale_mult <= 4.0:
+        assert_close(outs[0], refs[0], f"peaked x{scale_mult}")
+        return
     vmax = float(np.abs(synth.bf16_bits_to_f32(np.concatenate([inputs[1], inputs[3]], 1))).max())
     assert_within_rounding_bound(outs[0], refs[0], vmax, f"peaked x{scale_mult}")
 

@@ -3,7 +3,13 @@
 launch per layer).  Bookkeeping is compared with the oracle in full; attention
 on sampled query rows (first/last rows, tile boundaries, random rows), each
 computed by the oracle from the counterfactual sequence's definition (retained
-prefix of the original session followed by the sanitized suffix)."""
+prefix of the original session followed by the sanitized suffix).
+
+Every attention block passes the absolute gate and the gate normalised by the
+oracle's size (tests/parity.py), so an output of the right magnitude but the
+wrong values (zeros, another page table, a dropped key split) fails.  Each
+shape also runs with std-1 draws (logits of standard deviation 1 instead of
+the workloads' ~0.008), where a wrong key changes the output visibly."""
 import numpy as np
 import pytest
 import torch
@@ -27,7 +33,7 @@ def _rows(w, a, n_random, edge_tiles=4):
     return np.array(sorted(x for x in rows if 0 <= x < a.S), dtype=np.int64)
 
 
-def _draw(w, agents=None):
+def _draw(w):
     """Host bf16 draws of the workload, shared by the driver and the oracle."""
     out = {}
     for i, a in enumerate(w.agents):
@@ -59,6 +65,7 @@ def _check_bookkeeping(drv, steps=1):
 
 
 def _check_attention(drv, inputs, agents, layers, n_random):
+    """Each (agent, layer) block of sampled rows through both gates."""
     w = drv.w
     worst = (0.0, 0.0)
     for i in agents:
@@ -86,6 +93,7 @@ def _run(w):
 
 
 def test_tiny_full():
+    """Config 1 draws N(0, 1) values already (logits of standard deviation 1)."""
     w = synth.tiny()
     drv, inputs = _run(w)
     _check_bookkeeping(drv)
@@ -93,7 +101,7 @@ def test_tiny_full():
     k0, v0, kc, vc, qc = inputs[0]
     ref = oracle.causal_attention(qc[0], np.concatenate([k0[0, : a.P], kc[0]]),
                                   np.concatenate([v0[0, : a.P], vc[0]]), w.softmax_scale)
-    assert_close(drv.out[0], ref, "tiny (all rows)")
+    assert_close(drv.out[0], ref, f"{w.name} (all rows)")
 
 
 def test_agent_batch():
@@ -109,6 +117,13 @@ def test_agent_batch():
     _check_bookkeeping(drv, steps=2)
 
 
+def test_agent_batch_std1():
+    """The 5256-CTA launch of the agent batch with logits of standard deviation 1."""
+    w = synth.with_std(synth.agent_batch(), 1.0)
+    drv, inputs = _run(w)
+    _check_attention(drv, inputs, range(len(w.agents)), [0], n_random=16)
+
+
 def test_decode_batch():
     """Decode after replay: one new token per agent (n_q = 1) over the full cache."""
     w = synth.decode_batch()
@@ -121,24 +136,45 @@ def test_decode_batch():
     assert torch.equal(first, drv.out)
 
 
-def test_short_suffix_splitkv():
-    w = synth.short_suffix()
+def test_decode_batch_std1():
+    w = synth.with_std(synth.decode_batch(), 1.0)
     drv, inputs = _run(w)
+    _check_attention(drv, inputs, range(len(w.agents)), [0], n_random=0)
+
+
+@pytest.mark.parametrize("std", [None, 1.0])
+def test_short_suffix_splitkv(std):
+    """32k-token prefixes, 16 queries: the split-KV launch (7 key splits) and its combine."""
+    w = synth.short_suffix() if std is None else synth.with_std(synth.short_suffix(), std)
+    drv, inputs = _run(w)
+    split, n_splits, _ = drv.cache.last_attn_plan()
+    assert split and n_splits > 1
     _check_bookkeeping(drv)
     _check_attention(drv, inputs, [0, 7], [0], n_random=16)
     _check_attention(drv, inputs, range(1, 7), [0], n_random=2)
 
 
-def test_long_suffix():
-    w = synth.long_suffix()
+@pytest.mark.parametrize("std", [None, 1.0])
+def test_long_suffix(std):
+    """ps = 64, 16k-query suffixes over 4k prefixes, 64 q-heads on 8 kv-heads."""
+    w = synth.long_suffix() if std is None else synth.with_std(synth.long_suffix(), std)
     drv, inputs = _run(w)
     _check_bookkeeping(drv)
     _check_attention(drv, inputs, range(len(w.agents)), [0], n_random=32)
 
 
-@pytest.mark.parametrize("ratio", [0.1, 0.7, 0.9])
+@pytest.mark.parametrize("ratio", [0.1, 0.3, 0.5, 0.7, 0.9, 0.0])
 def test_tau_sweep(ratio):
+    """Every tau/T of the sweep and the full-reset comparator (ratio 0: an empty
+    prefix, the whole counterfactual sequence recomputed), 32 layers."""
     w = synth.tau_sweep(ratio)
     drv, inputs = _run(w)
     _check_bookkeeping(drv)
-    _check_attention(drv, inputs, [0], [0, w.num_layers - 1], n_random=24)
+    _check_attention(drv, inputs, [0], [0, 17, w.num_layers - 1], n_random=24)
+
+
+@pytest.mark.parametrize("ratio", [0.3, 0.9])
+def test_tau_sweep_std1(ratio):
+    w = synth.with_std(synth.tau_sweep(ratio), 1.0)
+    drv, inputs = _run(w)
+    _check_attention(drv, inputs, [0], [0, 13, w.num_layers - 1], n_random=16)
