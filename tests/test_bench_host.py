@@ -53,3 +53,5 @@ def test_reference_arm_prints_one_contract_line():
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
     assert d["unit"] == d["e2e"]["unit"] == d["cpu_baseline"]["unit"]
     assert "N(0,1^2)" in d["data"]  # the tiny workload draws unscaled N(0, 1) values
+    # ms_per_step is the measured wall time of a step's bounded sample, not an extrapolation
+    assert d["ms_per_step"] < 5000 and d["full_step_ms_extrapolated"] > 0
