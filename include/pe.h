@@ -28,7 +28,16 @@
  *   - All tensors are bf16, row-major, contiguous, 16-byte aligned device
  *     memory unless stated otherwise.
  *   - On any error the cache state is unchanged and pe_last_error() describes
- *     the failure.  A cache is not thread-safe: calls on one cache must not run
+ *     the failure.  This includes a failure of a device step after the
+ *     bookkeeping was applied (e.g. an append's kernel launch failing after its
+ *     pages were taken): the call undoes its host changes and rewrites the
+ *     device page-table rows and lengths of the sequences it touched from the
+ *     host, on `stream`, before returning PE_ERR_CUDA.  Pool slots the failed
+ *     call already wrote belong to pages or positions outside every
+ *     sequence's valid range afterwards, so no later result reads them
+ *     (exception: with "debug_poison" on, a batched crop that fails after its
+ *     first launch may leave poisoned slots in pages it had already freed).
+ *     A cache is not thread-safe: calls on one cache must not run
  *     concurrently.
  *   - Allocation policy: the free list is a LIFO stack whose initial pop order
  *     is `init_free_order`; an append pops one page per new logical page; crop
@@ -195,7 +204,8 @@ pe_status pe_replay_schedule(int32_t n, const int32_t *cu_turns, const int32_t *
  * The rounds must cover each agent's rows exactly (sum over r of take = its
  * row count).  Every argument, the pages all rounds need (checked up front,
  * including copy-on-write) and the page-table capacity are checked before any
- * state changes; a CUDA error (CUDA) may leave the earlier rounds applied.
+ * state changes; a CUDA error (CUDA) in any round undoes the bookkeeping of
+ * every round of the call (the outputs of earlier rounds may have been written).
  * On a host-only cache only the bookkeeping runs (Q, out unused).
  * Errors: INVALID, RANGE, OOM, UNSUPPORTED, CUDA. */
 pe_status pe_replay_rounds(pe_cache *cache, int32_t n, const int32_t *seqs, int32_t n_rounds, const int32_t *take,
@@ -246,7 +256,10 @@ pe_status pe_cache_pools(const pe_cache *cache, void **k_pool, void **v_pool);
  * whose n_q x (Hq/Hkv) query rows fit in 16 take a decode kernel with the
  * split-KV merge done in-kernel -- 1: tcgen05 with keys on the MMA's M side
  * for d = 128, CUDA cores for d = 64; 2: CUDA cores for both; 0: no decode
- * kernel (the prefill kernel serves every call).  Split
+ * kernel (the prefill kernel serves every call); "fail_launch_after" = k >= 0
+ * (test hook): the device step after the next k fails with PE_ERR_CUDA
+ * without being launched, once (-1 = off); on a host-only cache the steps a
+ * device cache would launch are counted the same way.  Split
  * partials and the decode kernel's merge counters live in the cache's
  * workspace, so attention calls on one cache must not overlap on the GPU
  * (issue them on one stream, or order the streams). */

@@ -70,6 +70,28 @@ int32_t pe::report_error(int32_t code, const char *msg)
     return code;
 }
 
+// Undo log of one C-ABI call's changes to the host bookkeeping.  Every change
+// a call makes goes through the journal helpers below; a call that fails after
+// changing the state (a kernel launch failed after pages were taken or given
+// back) replays the log backwards and re-mirrors the touched sequences'
+// device rows, so an error leaves the cache as it was before the call.
+struct SeqSave {
+    int32_t seq;
+    int32_t from;                // table entries [from, size0) are saved in `tail`
+    int32_t size0;               // table size before the call
+    std::vector<int32_t> tail;
+    int64_t len, appended;
+    std::vector<int64_t> ckpt;
+    uint8_t alive;
+};
+
+struct Journal {
+    std::vector<std::pair<int8_t, int32_t>> stack_ops;  // (+1 push / -1 pop, page), in call order
+    std::vector<std::pair<int32_t, int32_t>> refs;      // (page, reference count before the change)
+    std::vector<SeqSave> seqs;                          // one per touched sequence
+    std::vector<int32_t> seq_index;                     // sequence -> index in seqs, -1 when untouched
+};
+
 struct pe_cache {
     pe_cache_config cfg{};
     bool host_only = false;
@@ -98,6 +120,8 @@ struct pe_cache {
     int splitkv = -1, num_splits = 0, debug_poison = 0, decode_kernel = 1, dec_chunks_per_sm = 3;
     int64_t launches = 0;
     int32_t last_split = 0, last_splits = 0, last_ctas = 0;  // plan of the last attention launch
+    Journal jr;                   // changes of the call in progress
+    int64_t fail_after = -1;      // test hook "fail_launch_after": device steps left before an injected failure
 };
 
 namespace {
@@ -110,6 +134,126 @@ pe_status check_seq(const pe_cache *c, int32_t seq)
 }
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// ---- journal: every bookkeeping change of a call, undone if the call fails
+// Saves sequence `seq`'s state before the call changes its table entries at
+// index >= from (or its length, counter, checkpoints, liveness).
+void j_seq(pe_cache *c, int32_t seq, int32_t from)
+{
+    Journal &j = c->jr;
+    if (j.seq_index.empty()) j.seq_index.assign(c->cfg.max_seqs, -1);
+    const std::vector<int32_t> &t = c->table[seq];
+    int32_t &ix = j.seq_index[seq];
+    if (ix < 0) {
+        ix = static_cast<int32_t>(j.seqs.size());
+        SeqSave sv;
+        sv.seq = seq;
+        sv.size0 = static_cast<int32_t>(t.size());
+        sv.from = std::min(from, sv.size0);
+        sv.tail.assign(t.begin() + sv.from, t.end());
+        sv.len = c->len[seq];
+        sv.appended = c->appended[seq];
+        sv.ckpt = c->ckpt[seq];
+        sv.alive = c->alive[seq];
+        j.seqs.push_back(std::move(sv));
+        return;
+    }
+    SeqSave &sv = j.seqs[ix];
+    if (from < sv.from) {  // entries [from, sv.from) are still unchanged: save them too
+        sv.tail.insert(sv.tail.begin(), t.begin() + from, t.begin() + sv.from);
+        sv.from = from;
+    }
+}
+
+void free_push(pe_cache *c, int32_t pg)
+{
+    c->free_stack.push_back(pg);
+    c->jr.stack_ops.emplace_back(static_cast<int8_t>(1), pg);
+}
+
+int32_t free_pop(pe_cache *c)
+{
+    const int32_t pg = c->free_stack.back();
+    c->free_stack.pop_back();
+    c->jr.stack_ops.emplace_back(static_cast<int8_t>(-1), pg);
+    return pg;
+}
+
+void set_ref(pe_cache *c, int32_t pg, int32_t v)
+{
+    c->jr.refs.emplace_back(pg, c->refs[pg]);
+    c->refs[pg] = v;
+}
+
+void journal_clear(pe_cache *c)
+{
+    Journal &j = c->jr;
+    for (const SeqSave &sv : j.seqs) j.seq_index[sv.seq] = -1;
+    j.seqs.clear();
+    j.refs.clear();
+    j.stack_ops.clear();
+}
+
+// Undoes the call's changes (newest first) and rewrites the device mirror
+// (table row and length) of every touched live sequence on `st`, after any
+// device work the call already enqueued.
+void rollback(pe_cache *c, cudaStream_t st)
+{
+    Journal &j = c->jr;
+    for (auto it = j.refs.rbegin(); it != j.refs.rend(); ++it) c->refs[it->first] = it->second;
+    for (auto it = j.stack_ops.rbegin(); it != j.stack_ops.rend(); ++it) {
+        if (it->first > 0) c->free_stack.pop_back();
+        else c->free_stack.push_back(it->second);
+    }
+    for (const SeqSave &sv : j.seqs) {
+        std::vector<int32_t> &t = c->table[sv.seq];
+        t.resize(sv.size0);
+        std::copy(sv.tail.begin(), sv.tail.end(), t.begin() + sv.from);
+        c->len[sv.seq] = sv.len;
+        c->appended[sv.seq] = sv.appended;
+        c->ckpt[sv.seq] = sv.ckpt;
+        c->alive[sv.seq] = sv.alive;
+        if (!c->host_only && sv.alive) {
+            const int64_t row = static_cast<int64_t>(sv.seq) * c->cfg.max_pages_per_seq;
+            if (!t.empty())
+                cudaMemcpyAsync(c->d_table + row, t.data(), sizeof(int32_t) * t.size(), cudaMemcpyHostToDevice, st);
+            cudaMemcpyAsync(c->d_len + sv.seq, &c->len[sv.seq], sizeof(int64_t), cudaMemcpyHostToDevice, st);
+        }
+    }
+    if (!c->host_only) cudaStreamSynchronize(st);  // the copies read host memory the next call may change
+    journal_clear(c);
+}
+
+// One C-ABI call that changes bookkeeping: end() keeps the changes on success
+// and rolls them back on any error.
+struct CallTxn {
+    pe_cache *c;
+    cudaStream_t st;
+    CallTxn(pe_cache *c_, cudaStream_t st_) : c(c_), st(st_) { journal_clear(c); }
+    pe_status end(pe_status s)
+    {
+        if (s != PE_OK) rollback(c, st);
+        else journal_clear(c);
+        return s;
+    }
+    ~CallTxn() { journal_clear(c); }
+};
+
+// Test hook: with "fail_launch_after" = k, the device step after the next k
+// fails with PE_ERR_CUDA without running (on a host-only cache the steps a
+// device cache would launch are counted the same way).
+bool injected_failure(pe_cache *c)
+{
+    if (c->fail_after < 0) return false;
+    if (c->fail_after-- > 0) return false;
+    c->fail_after = -1;
+    return true;
+}
+
+pe_status launch_fault(const char *what)
+{
+    return fail(PE_ERR_CUDA, "%s: launch failure injected by the fail_launch_after test hook", what);
+}
 
 pe_status encode_2d(CUtensorMap *m, void *base, uint64_t cols, uint64_t rows, uint32_t box_cols, uint32_t box_rows)
 {
@@ -175,12 +319,14 @@ struct CropPlan {
 // last reference goes is pushed onto the free list.
 void apply_crop(pe_cache *c, CropPlan &pl, int32_t *freed_out)
 {
+    j_seq(c, pl.seq, pl.keep);
     std::vector<int32_t> &t = c->table[pl.seq];
     std::vector<int32_t> freed_desc;
     for (int32_t e = pl.old_n - 1; e >= pl.keep; --e) {
         const int32_t pg = t[e];
-        if (--c->refs[pg] == 0) {
-            c->free_stack.push_back(pg);
+        set_ref(c, pg, c->refs[pg] - 1);
+        if (c->refs[pg] == 0) {
+            free_push(c, pg);
             freed_desc.push_back(pg);
         }
     }
@@ -198,7 +344,6 @@ void apply_crop(pe_cache *c, CropPlan &pl, int32_t *freed_out)
 
 pe_status launch_crops(pe_cache *c, const std::vector<CropPlan> &plans, cudaStream_t st)
 {
-    if (c->host_only) return PE_OK;
     std::vector<char> buf(sizeof(CropParams));
     CropParams &p = *reinterpret_cast<CropParams *>(buf.data());
     std::memset(&p, 0, sizeof p);
@@ -233,6 +378,8 @@ pe_status launch_crops(pe_cache *c, const std::vector<CropPlan> &plans, cudaStre
             nf += sg.n_freed;
             sg.tail_page = pl.tail_page;
         }
+        if (injected_failure(c)) return launch_fault("crop kernel");
+        if (c->host_only) continue;
         cudaError_t e = launch_crop(p, st);
         if (e != cudaSuccess) return cuda_fail(e, "crop kernel launch");
         c->launches++;
@@ -285,17 +432,40 @@ pe_status plan_append(const pe_cache *c, int32_t seq, int64_t n, AppendPlan *pl)
     return PE_OK;
 }
 
+// A batch is planned as if its sequences were appended one after another: a
+// copy-on-write planned for an earlier sequence drops one reference of the
+// shared page, so a later sequence sharing that page may hold it alone by its
+// turn and need no copy (and no extra page).
+void settle_batch_cow(const pe_cache *c, std::vector<AppendPlan> &plans)
+{
+    std::vector<std::pair<int32_t, int32_t>> dropped;  // (page, references dropped by earlier plans)
+    for (AppendPlan &pl : plans) {
+        if (!pl.cow) continue;
+        const int32_t pg = c->table[pl.seq].back();
+        auto it = std::find_if(dropped.begin(), dropped.end(), [&](const auto &x) { return x.first == pg; });
+        const int32_t d = it == dropped.end() ? 0 : it->second;
+        if (c->refs[pg] - d <= 1) {
+            pl.cow = false;
+            pl.need -= 1;
+            continue;
+        }
+        if (it == dropped.end()) dropped.emplace_back(pg, 1);
+        else it->second += 1;
+    }
+}
+
 // Copy-on-write of a sequence's shared, partially filled last page: pop a
 // fresh page, copy the valid slots on the device, drop one reference.
 pe_status apply_cow(pe_cache *c, int32_t seq, cudaStream_t st)
 {
+    j_seq(c, seq, static_cast<int32_t>(c->table[seq].size()) - 1);
     std::vector<int32_t> &t = c->table[seq];
     const int32_t src = t.back();
-    const int32_t dst = c->free_stack.back();
-    c->free_stack.pop_back();
-    c->refs[dst] = 1;
-    c->refs[src] -= 1;
+    const int32_t dst = free_pop(c);
+    set_ref(c, dst, 1);
+    set_ref(c, src, c->refs[src] - 1);
     t.back() = dst;
+    if (injected_failure(c)) return launch_fault("copy-on-write");
     if (!c->host_only) {
         const int32_t slots = static_cast<int32_t>(c->len[seq] % c->cfg.page_size);
         int32_t *entry = c->d_table + static_cast<int64_t>(seq) * c->cfg.max_pages_per_seq + (t.size() - 1);
@@ -315,12 +485,10 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
                         int64_t n_total, cudaStream_t st)
 {
     const int ps = c->cfg.page_size;
-    AppendParams *p = nullptr;
-    std::vector<char> pbuf;
-    if (!c->host_only) {
-        pbuf.resize(sizeof(AppendParams));
-        p = reinterpret_cast<AppendParams *>(pbuf.data());
-        std::memset(p, 0, sizeof(AppendParams));
+    std::vector<char> pbuf(sizeof(AppendParams));
+    AppendParams *p = reinterpret_cast<AppendParams *>(pbuf.data());
+    std::memset(p, 0, sizeof(AppendParams));
+    {
         p->K = static_cast<const uint4 *>(K);
         p->V = static_cast<const uint4 *>(V);
         p->k_pool = static_cast<uint4 *>(c->k_pool);
@@ -335,10 +503,11 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
         p->n_total = static_cast<int32_t>(n_total);
     }
     auto flush = [&]() -> pe_status {
-        if (c->host_only || p->n_segs == 0) return PE_OK;
+        if (p->n_segs == 0) return PE_OK;
         p->seg_tokens = p->segs[p->n_segs - 1].cum0 + p->segs[p->n_segs - 1].n_tokens;
         const int64_t chunks = static_cast<int64_t>(p->L) * p->seg_tokens * p->hkv * p->dvec;
-        if (chunks > 0 || p->n_segs > 0) {
+        if (injected_failure(c)) return launch_fault("append kernel");
+        if (!c->host_only) {
             cudaError_t e = launch_append(*p, chunks, st);
             if (e != cudaSuccess) return cuda_fail(e, "append kernel launch");
             c->launches++;
@@ -348,11 +517,14 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
     };
     int32_t pages_in_launch = 0;
     for (const AppendPlan &pl : plans) {
-        if (pl.cow) {
+        // decided now, on the current references (the planners' page counts agree: settle_batch_cow)
+        const std::vector<int32_t> &tt = c->table[pl.seq];
+        if (pl.n > 0 && c->len[pl.seq] % ps != 0 && c->refs[tt.back()] > 1) {
             pe_status s = apply_cow(c, pl.seq, st);
             if (s != PE_OK) return s;
         }
         int32_t done = 0;
+        if (pl.n > 0) j_seq(c, pl.seq, static_cast<int32_t>(c->table[pl.seq].size()));
         while (done < pl.n) {
             const int64_t len0 = c->len[pl.seq];
             std::vector<int32_t> &t = c->table[pl.seq];
@@ -362,7 +534,7 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
             int64_t take = pl.n - done;
             const int64_t max_take = have_slots + room_pages * ps;
             if (take > max_take) take = max_take;
-            if (!c->host_only && (take <= 0 || p->n_segs == kMaxSegs)) {
+            if (take <= 0 || p->n_segs == kMaxSegs) {
                 pe_status s = flush();
                 if (s != PE_OK) return s;
                 pages_in_launch = 0;
@@ -370,7 +542,7 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
             }
             const int32_t first_new_lp = static_cast<int32_t>(t.size());
             const int32_t need = static_cast<int32_t>(ceil_div(len0 + take, ps) - static_cast<int64_t>(t.size()));
-            if (!c->host_only) {
+            {
                 AppendSeg &sg = p->segs[p->n_segs];
                 sg.tok0 = pl.tok0 + done;
                 sg.cum0 = p->n_segs == 0 ? 0 : p->segs[p->n_segs - 1].cum0 + p->segs[p->n_segs - 1].n_tokens;
@@ -384,16 +556,13 @@ pe_status apply_appends(pe_cache *c, const std::vector<AppendPlan> &plans, const
                 sg.seq = pl.seq;
             }
             for (int32_t i = 0; i < need; ++i) {
-                const int32_t pg = c->free_stack.back();
-                c->free_stack.pop_back();
-                c->refs[pg] = 1;
+                const int32_t pg = free_pop(c);
+                set_ref(c, pg, 1);
                 t.push_back(pg);
-                if (!c->host_only) p->new_pages[pages_in_launch + i] = pg;
+                p->new_pages[pages_in_launch + i] = pg;
             }
-            if (!c->host_only) {
-                pages_in_launch += need;
-                p->n_segs++;
-            }
+            pages_in_launch += need;
+            p->n_segs++;
             c->len[pl.seq] = len0 + take;
             c->appended[pl.seq] += take;
             done += static_cast<int32_t>(take);
@@ -514,6 +683,7 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
             c->last_split = any_split ? 1 : 0;
             c->last_splits = p.seqs[0].n_splits;
             c->last_ctas = p.total_ctas;
+            if (injected_failure(c)) return launch_fault("decode attention");
             cudaError_t e = launch_decode_attn(d, rb, true, c->tm_kd, c->tm_vd, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
             c->launches++;
@@ -583,6 +753,7 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
         c->last_split = p.seqs[0].n_splits > 1 ? 1 : 0;
         c->last_splits = p.seqs[0].n_splits;
         c->last_ctas = p.total_ctas;
+        if (injected_failure(c)) return launch_fault("decode attention");
         cudaError_t e = launch_decode_attn(d, rb, tc, c->tm_kd, c->tm_vd, p, st);
         if (e != cudaSuccess) return cuda_fail(e, "decode attention launch");
         c->launches++;
@@ -789,10 +960,12 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         c->last_split = split || tail ? 1 : 0;
         c->last_splits = tail ? static_cast<int32_t>(tp.splits) : (split ? p.seqs[0].n_splits : 1);
         c->last_ctas = p.total_items + (tail ? static_cast<int32_t>(tp.pairs * hkv * tp.splits) : 0);
+        if (injected_failure(c)) return launch_fault("replay attention");
         cudaError_t e = launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, p, st);
         if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
         c->launches++;
         if (split) {
+            if (injected_failure(c)) return launch_fault("split-KV combine");
             e = launch_splitkv_combine(d, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
             c->launches++;
@@ -810,9 +983,11 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             p.total_comb = static_cast<int32_t>(tp.qtiles * hkv * kBM);  // q-tiles [0, 2 cut)
             p.part_o = c->d_ws;
             p.part_lse = c->d_ws + tp.qtiles * hkv * tp.splits * kBM * d;
+            if (injected_failure(c)) return launch_fault("replay attention tail");
             e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "replay attention tail launch");
             c->launches++;
+            if (injected_failure(c)) return launch_fault("split-KV combine");
             e = launch_splitkv_combine(d, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
             c->launches++;
@@ -984,10 +1159,11 @@ pe_status pe_seq_release(pe_cache *c, int32_t seq, void *stream)
     std::vector<CropPlan> pl(1);
     pe_status s = plan_crop(c, seq, 1, &pl[0]);
     if (s != PE_OK) return s;
+    CallTxn tx(c, static_cast<cudaStream_t>(stream));
     apply_crop(c, pl[0], nullptr);
     c->alive[seq] = 0;
     c->ckpt[seq].clear();
-    return launch_crops(c, pl, static_cast<cudaStream_t>(stream));
+    return tx.end(launch_crops(c, pl, static_cast<cudaStream_t>(stream)));
 }
 
 pe_status pe_seq_fork(pe_cache *c, int32_t seq, int32_t *new_seq, void *stream)
@@ -999,21 +1175,24 @@ pe_status pe_seq_fork(pe_cache *c, int32_t seq, int32_t *new_seq, void *stream)
     for (int32_t q = 0; q < c->cfg.max_seqs; ++q)
         if (!c->alive[q]) { ns = q; break; }
     if (ns < 0) return fail(PE_ERR_OOM, "no free sequence slot (max_seqs = %d)", c->cfg.max_seqs);
+    CallTxn tx(c, static_cast<cudaStream_t>(stream));
+    j_seq(c, ns, 0);
     c->alive[ns] = 1;
     c->table[ns] = c->table[seq];
-    for (int32_t pg : c->table[ns]) c->refs[pg] += 1;
+    for (int32_t pg : c->table[ns]) set_ref(c, pg, c->refs[pg] + 1);
     c->len[ns] = c->len[seq];
     c->appended[ns] = c->appended[seq];
     c->ckpt[ns] = c->ckpt[seq];
-    *new_seq = ns;
+    if (injected_failure(c)) return tx.end(launch_fault("fork table copy"));
     if (!c->host_only) {
         cudaError_t e = launch_table_copy(c->d_table, seq * c->cfg.max_pages_per_seq, ns * c->cfg.max_pages_per_seq,
                                           static_cast<int32_t>(c->table[ns].size()), c->d_len, ns, c->len[ns],
                                           static_cast<cudaStream_t>(stream));
-        if (e != cudaSuccess) return cuda_fail(e, "fork table copy launch");
+        if (e != cudaSuccess) return tx.end(cuda_fail(e, "fork table copy launch"));
         c->launches++;
     }
-    return PE_OK;
+    *new_seq = ns;
+    return tx.end(PE_OK);
 }
 
 pe_status pe_checkpoint_add(pe_cache *c, int32_t seq, int64_t offset)
@@ -1084,9 +1263,11 @@ pe_status pe_crop(pe_cache *c, int32_t seq, int64_t tau, int32_t *freed_out, int
     if (s != PE_OK) return s;
     const int32_t nf = pl[0].n_freed;
     if (freed_out && freed_cap < nf) return fail(PE_ERR_RANGE, "freed_cap %d < %d freed pages", freed_cap, nf);
+    CallTxn tx(c, static_cast<cudaStream_t>(stream));
     apply_crop(c, pl[0], freed_out);
-    if (n_freed) *n_freed = nf;
-    return launch_crops(c, pl, static_cast<cudaStream_t>(stream));
+    s = tx.end(launch_crops(c, pl, static_cast<cudaStream_t>(stream)));
+    if (s == PE_OK && n_freed) *n_freed = nf;
+    return s;
 }
 
 pe_status pe_crop_batch(pe_cache *c, int32_t n, const int32_t *seqs, const int64_t *taus, void *stream)
@@ -1101,8 +1282,9 @@ pe_status pe_crop_batch(pe_cache *c, int32_t n, const int32_t *seqs, const int64
         if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice in the batch", seqs[i]);
         seen[seqs[i]] = 1;
     }
+    CallTxn tx(c, static_cast<cudaStream_t>(stream));
     for (CropPlan &pl : plans) apply_crop(c, pl, nullptr);
-    return launch_crops(c, plans, static_cast<cudaStream_t>(stream));
+    return tx.end(launch_crops(c, plans, static_cast<cudaStream_t>(stream)));
 }
 
 pe_status pe_append_kv(pe_cache *c, int32_t seq, const void *K, const void *V, int32_t n_tokens, void *stream)
@@ -1117,7 +1299,8 @@ pe_status pe_append_kv(pe_cache *c, int32_t seq, const void *K, const void *V, i
     if (pl.need > static_cast<int32_t>(c->free_stack.size()))
         return fail(PE_ERR_OOM, "append needs %d pages, %zu free", pl.need, c->free_stack.size());
     pl.tok0 = 0;
-    return apply_appends(c, {pl}, K, V, n_tokens, static_cast<cudaStream_t>(stream));
+    CallTxn tx(c, static_cast<cudaStream_t>(stream));
+    return tx.end(apply_appends(c, {pl}, K, V, n_tokens, static_cast<cudaStream_t>(stream)));
 }
 
 pe_status pe_append_kv_batch(pe_cache *c, int32_t n, const int32_t *seqs, const void *K, const void *V,
@@ -1128,7 +1311,6 @@ pe_status pe_append_kv_batch(pe_cache *c, int32_t n, const int32_t *seqs, const 
     if (n > 0 && cu_tokens[0] != 0) return fail(PE_ERR_INVALID, "cu_tokens[0] must be 0");
     std::vector<AppendPlan> plans(n);
     std::vector<uint8_t> seen(c->cfg.max_seqs, 0);
-    int64_t need = 0;
     for (int32_t i = 0; i < n; ++i) {
         if (cu_tokens[i + 1] < cu_tokens[i]) return fail(PE_ERR_INVALID, "cu_tokens must be non-decreasing");
         pe_status s = plan_append(c, seqs[i], cu_tokens[i + 1] - cu_tokens[i], &plans[i]);
@@ -1136,8 +1318,10 @@ pe_status pe_append_kv_batch(pe_cache *c, int32_t n, const int32_t *seqs, const 
         if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice in the batch", seqs[i]);
         seen[seqs[i]] = 1;
         plans[i].tok0 = cu_tokens[i];
-        need += plans[i].need;
     }
+    settle_batch_cow(c, plans);
+    int64_t need = 0;
+    for (const AppendPlan &pl : plans) need += pl.need;
     const int64_t total = n > 0 ? cu_tokens[n] : 0;
     if (!c->host_only && total > 0) {
         if (!K || !V) return fail(PE_ERR_INVALID, "null K or V");
@@ -1146,7 +1330,8 @@ pe_status pe_append_kv_batch(pe_cache *c, int32_t n, const int32_t *seqs, const 
     if (need > static_cast<int64_t>(c->free_stack.size()))
         return fail(PE_ERR_OOM, "batch append needs %lld pages, %zu free", static_cast<long long>(need),
                     c->free_stack.size());
-    return apply_appends(c, plans, K, V, total, static_cast<cudaStream_t>(stream));
+    CallTxn tx(c, static_cast<cudaStream_t>(stream));
+    return tx.end(apply_appends(c, plans, K, V, total, static_cast<cudaStream_t>(stream)));
 }
 
 pe_status pe_replay_attn(pe_cache *c, int32_t seq, int32_t layer, const void *Q, void *out, int32_t n_q,
@@ -1211,14 +1396,13 @@ pe_status pe_replay_rounds(pe_cache *c, int32_t n, const int32_t *seqs, int32_t 
     // every agent: a live, distinct sequence whose rounds cover its rows exactly,
     // and room for all of its positions (pages counted once, up front)
     std::vector<uint8_t> seen(c->cfg.max_seqs, 0);
-    int64_t need = 0;
+    std::vector<AppendPlan> whole(n);
     for (int32_t i = 0; i < n; ++i) {
         if (cu_tok[i + 1] < cu_tok[i]) return fail(PE_ERR_INVALID, "cu_tok must be non-decreasing");
-        AppendPlan pl{};
+        AppendPlan &pl = whole[i];
         if ((s = plan_append(c, seqs[i], cu_tok[i + 1] - cu_tok[i], &pl)) != PE_OK) return s;
         if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice", seqs[i]);
         seen[seqs[i]] = 1;
-        need += pl.need;
         int64_t sum = 0;
         for (int32_t r = 0; r < n_rounds; ++r) {
             const int32_t t = take[static_cast<int64_t>(r) * n + i];
@@ -1229,11 +1413,16 @@ pe_status pe_replay_rounds(pe_cache *c, int32_t n, const int32_t *seqs, int32_t 
             return fail(PE_ERR_INVALID, "agent %d: rounds cover %lld of its %d rows", i, static_cast<long long>(sum),
                         cu_tok[i + 1] - cu_tok[i]);
     }
+    // a sequence copies its shared last page in its first round with work, in agent order
+    settle_batch_cow(c, whole);
+    int64_t need = 0;
+    for (const AppendPlan &pl : whole) need += pl.need;
     if (need > static_cast<int64_t>(c->free_stack.size()))
         return fail(PE_ERR_OOM, "the rounds need %lld pages, %zu free", static_cast<long long>(need),
                     c->free_stack.size());
 
     const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    CallTxn tx(c, st);
     const int64_t row_bytes = static_cast<int64_t>(num_q_heads) * c->cfg.head_dim * 2;  // one bf16 [Hq][d] row
     std::vector<int32_t> done(n, 0);
     std::vector<AppendPlan> plans;
@@ -1252,16 +1441,16 @@ pe_status pe_replay_rounds(pe_cache *c, int32_t n, const int32_t *seqs, int32_t 
             done[i] += t;
         }
         if (plans.empty()) continue;
-        if ((s = apply_appends(c, plans, K, V, N, st)) != PE_OK) return s;
+        if ((s = apply_appends(c, plans, K, V, N, st)) != PE_OK) return tx.end(s);
         if (c->host_only) continue;
         for (int32_t layer = 0; layer < c->cfg.num_layers; ++layer) {
             const int64_t off = static_cast<int64_t>(layer) * N * row_bytes;
             s = run_attention(c, items, layer, static_cast<const char *>(Q) + off, N, static_cast<char *>(out) + off,
                               num_q_heads, softmax_scale, st);
-            if (s != PE_OK) return s;
+            if (s != PE_OK) return tx.end(s);
         }
     }
-    return PE_OK;
+    return tx.end(PE_OK);
 }
 
 pe_status pe_replay_attn_static_scratch(pe_cache *c, int32_t seq, int32_t layer, const void *Q, void *out,
@@ -1332,9 +1521,11 @@ pe_status pe_replay_attn_static_scratch(pe_cache *c, int32_t seq, int32_t layer,
     p.part_o = scratch;
     p.part_lse = scratch + prow * d;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (injected_failure(c)) return launch_fault("replay attention");
     e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, p, st);
     if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
     c->launches++;
+    if (injected_failure(c)) return launch_fault("split-KV combine");
     e = launch_splitkv_combine(d, p, st);
     if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
     c->launches++;
@@ -1415,6 +1606,9 @@ pe_status pe_set_option(pe_cache *c, const char *key, int64_t value)
     } else if (!std::strcmp(key, "decode_kernel")) {
         if (value < 0 || value > 2) return fail(PE_ERR_INVALID, "decode_kernel must be 0, 1 or 2");
         c->decode_kernel = static_cast<int>(value);
+    } else if (!std::strcmp(key, "fail_launch_after")) {
+        if (value < -1) return fail(PE_ERR_INVALID, "fail_launch_after must be -1 (off) or >= 0");
+        c->fail_after = value;
     } else {
         return fail(PE_ERR_INVALID, "unknown option '%s'", key);
     }
