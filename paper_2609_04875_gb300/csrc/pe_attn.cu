@@ -211,9 +211,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (op_on) ptx::tma_load_2d(v_smem0 + s * C::kTileBytes + op_off, &tm_v, op_reg * 64, y, b_v_full + 8 * s);
         return true;
     };
+    // Launched with programmatic serialization: the next kernel in the stream may
+    // start its set-up once every CTA of this grid has started (it waits for this
+    // grid's completion before touching memory), and this grid's set-up overlaps
+    // the previous kernel; griddepcontrol.wait comes before the first read of
+    // memory an earlier kernel wrote (page table, pool, Q) and before any write.
+    ptx::griddep_launch_dependents();
     int page_next = -1;
     if (warp == 8) {
-        if (n_all > 0) page_next = page_of(0);   // global load in flight during the set-up
         if (lane == 0) {
             ptx::mbar_init(b_q_full, 1);
             for (int s = 0; s < C::kStages; ++s) {
@@ -233,6 +238,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::prefetch_tensormap(&tm_q);
             ptx::prefetch_tensormap(&tm_k);
             ptx::prefetch_tensormap(&tm_v);
+        }
+        ptx::griddep_wait();
+        if (n_all > 0) page_next = page_of(0);
+        if (lane == 0) {
             if (n_all > 0) {
                 const int nq = geo[1].qt >= 0 ? 2 : 1;
                 ptx::mbar_arrive_expect_tx(b_q_full, nq * C::kTileBytes);
@@ -336,6 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp < 8) {
         // =================================================== softmax / epilogue
+        ptx::griddep_wait();                     // before this role's first global write
         const int t = warp >> 2;                 // q-tile of this warpgroup
         const TileGeo &G = geo[t];
         const int row = threadIdx.x & 127;       // TMEM lane
@@ -529,6 +539,10 @@ cudaError_t launch_bounded_wait_selftest(int32_t *status, uint64_t limit_ns, cud
 template <int HD>
 __global__ void __launch_bounds__(256) splitkv_combine_kernel(const __grid_constant__ AttnParams p)
 {
+    // launched with programmatic serialization after the attention grid: wait
+    // for its partials; the next kernel may start its own set-up meanwhile
+    ptx::griddep_launch_dependents();
+    ptx::griddep_wait();
     const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (gw >= p.total_comb) return;
@@ -613,8 +627,17 @@ static cudaError_t launch_attn_t(const CUtensorMap &q, const CUtensorMap &k, con
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    replay_attn_kernel<HD, SPLIT><<<p.total_items, kThreads, C::kDynSmem, st>>>(q, k, v, p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(p.total_items));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::kDynSmem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, replay_attn_kernel<HD, SPLIT>, q, k, v, p);
 }
 
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
@@ -635,13 +658,19 @@ cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream
     if (p.total_comb <= 0) return cudaSuccess;
     const int warps_per_block = 8;
     const int blocks = (p.total_comb + warps_per_block - 1) / warps_per_block;
-    if (head_dim == 128)
-        splitkv_combine_kernel<128><<<blocks, 256, 0, st>>>(p);
-    else if (head_dim == 64)
-        splitkv_combine_kernel<64><<<blocks, 256, 0, st>>>(p);
-    else
-        return cudaErrorInvalidValue;
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(blocks));
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (head_dim == 128) return cudaLaunchKernelEx(&cfg, splitkv_combine_kernel<128>, p);
+    if (head_dim == 64) return cudaLaunchKernelEx(&cfg, splitkv_combine_kernel<64>, p);
+    return cudaErrorInvalidValue;
 }
 
 }  // namespace pe

@@ -819,15 +819,18 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         // splits add their fp32 partials' HBM round trip and a combine launch.
         const double W = C > 0 ? static_cast<double>(tiles) / C : 0.0;
         const int64_t row_bytes = static_cast<int64_t>(d) * 4 + 4;
+        // (the combine kernel is a programmatic dependent of the attention grid: about 3 us more)
         auto cost = [&](int64_t sp) {
             const double waves = std::ceil(static_cast<double>(C * sp) / c->num_sms);
             double t = std::max(waves * (W / sp + 2.0), static_cast<double>(max_tiles) / sp + 2.0) * 1.5e-6;
-            if (sp > 1) t += static_cast<double>(valid_rows * sp * row_bytes * 2) / 6.0e12 + 5e-6;
+            if (sp > 1) t += static_cast<double>(valid_rows * sp * row_bytes * 2) / 6.0e12 + 3e-6;
             return t;
         };
         int64_t best = 1;
         if (splitkv != 0) {
-            const int64_t s_max = std::min<int64_t>(128, std::max<int64_t>(1, max_tiles / 4));
+            // at least 4 key tiles per split, unless the CTAs are too few to fill the SMs
+            int64_t s_max = std::min<int64_t>(128, std::max<int64_t>(1, max_tiles / 4));
+            if (C > 0 && C * 2 <= c->num_sms) s_max = std::max(s_max, std::min<int64_t>(max_tiles, c->num_sms / C));
             double best_t = splitkv == 1 ? 1e30 : cost(1);
             for (int64_t sp = 2; sp <= s_max; ++sp) {
                 if (rows * sp * row_bytes > c->ws_bytes) break;
