@@ -14,7 +14,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libpe.so")
-SOURCES = ["pe_host.cu", "pe_kv.cu", "pe_attn.cu", "pe_decode.cu", "pe_prov.cpp", "pe_sched.cpp"]
+SOURCES = ["pe_host.cu", "pe_kv.cu", "pe_attn.cu", "pe_attn_sk.cu", "pe_decode.cu", "pe_prov.cpp", "pe_sched.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -118,6 +118,8 @@ struct pe_cache {
     CUtensorMap tm_kd{}, tm_vd{};  // decode kernel: 64 x min(ps, 64) boxes
     // options
     int splitkv = -1, num_splits = 0, debug_poison = 0, decode_kernel = 1, dec_chunks_per_sm = 3;
+    int attn_kernel = 1;          // prefill kernel: 1 auto, 2 persistent stream-K, 0 one work item per CTA
+    int attn_ctas = 0;            // persistent kernel's CTA count (0 = chosen by the planner)
     int64_t launches = 0;
     int32_t last_split = 0, last_splits = 0, last_ctas = 0;  // plan of the last attention launch
     Journal jr;                   // changes of the call in progress
@@ -761,6 +763,207 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
     return PE_OK;
 }
 
+// ---- persistent stream-K plan of one launch group (replay_attn_sk_kernel)
+// Units are (sequence, kv-head, q-tile pair) in the kernel's order: sequences
+// as given (longest first), kv-head fastest, pairs heaviest first.  A unit
+// costs its key tiles plus kSkUnitCost for loading Q and writing the output;
+// CTA c takes the work between boundaries c and c + 1 at c / P of the total.
+// With cuts allowed a boundary falls inside a unit (at a key tile, each piece
+// at least kSkMinPiece tiles), else at the unit boundary nearest to it; cuts
+// are kept when the cost model (the busiest CTA, plus the combine launch)
+// prefers them by 5 %, or always with "splitkv" = 1.
+constexpr double kSkUnitCost = 2.0;
+constexpr int kSkMinPiece = 2;
+
+struct SkBound {
+    int32_t u, t;  // unit and key tile (t = 0: the start of unit u)
+    bool operator==(const SkBound &o) const { return u == o.u && t == o.t; }
+};
+
+pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, size_t hi, int32_t layer, void *out,
+                  int32_t hq, float scale, SkParams &P)
+{
+    const pe_cache_config &cf = c->cfg;
+    const int hkv = cf.num_kv_heads, d = cf.head_dim, g = hq / hkv, bmq = kBM / g;
+    std::memset(&P, 0, sizeof P);
+    AttnParams &p = P.a;
+    p.page_table = c->d_table;
+    p.out = out;
+    p.status = c->d_status;
+    p.hq = hq;
+    p.hkv = hkv;
+    p.group = g;
+    p.layer = layer;
+    p.num_pages = cf.num_pages;
+    p.ps = cf.page_size;
+    p.oob_row = static_cast<int32_t>(c->pool_rows);
+    p.scale_log2 = scale * 1.4426950408889634f;
+    std::vector<int32_t> n_all;   // key tiles per unit
+    std::vector<double> cum{0.0};  // cost before each unit
+    for (size_t i = lo; i < hi; ++i) {
+        const AttnItem &it = order[i];
+        AttnSeq &q = p.seqs[p.n_seqs++];
+        q.table_row = it.seq * cf.max_pages_per_seq;
+        q.n_pages = static_cast<int32_t>(c->table[it.seq].size());
+        q.q_row0 = it.q_row0;
+        q.n_q = it.n_q;
+        q.n_keys = static_cast<int32_t>(c->len[it.seq]);
+        q.n_qtiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(it.n_q) * g, kBM));
+        q.pair_top = (q.n_qtiles + 1) / 2;
+        q.n_splits = 1;
+        q.item0 = static_cast<int32_t>(n_all.size());
+        for (int32_t local = 0; local < q.pair_top * hkv; ++local) {
+            const int32_t pair = q.pair_top - 1 - local / hkv;
+            const int32_t qt_last = std::min(2 * pair + 1, q.n_qtiles - 1);
+            const int64_t q_last = std::min<int64_t>((qt_last + 1) * static_cast<int64_t>(bmq), it.n_q) - 1;
+            const int32_t n = static_cast<int32_t>(ceil_div(c->len[it.seq] - it.n_q + q_last + 1, kBN));
+            n_all.push_back(n);
+            cum.push_back(cum.back() + n + kSkUnitCost);
+        }
+    }
+    const int32_t U = static_cast<int32_t>(n_all.size());
+    auto unit_at = [&](double x) {  // the unit whose cost range holds x
+        return static_cast<int32_t>(std::upper_bound(cum.begin(), cum.end(), x) - cum.begin()) - 1;
+    };
+
+    // A plan for nc CTAs.  Whole units first, in lockstep rounds: in round r CTA k takes unit
+    // r nc + k (k reversed in odd rounds), so the CTAs running at once work on neighbouring units
+    // and share their K/V in L2.  The last one to two rounds of units (the tail) are spread so that
+    // every CTA ends with about the same total: CTA k's contiguous tail stretch is what its rounds
+    // lack of the mean.  b[k] = (unit, key tile) where CTA k's tail stretch starts, b[nc] = (U, 0).
+    struct Plan {
+        int32_t nc = 1, R = 0;
+        std::vector<double> own;
+        std::vector<SkBound> b;
+    };
+    auto make = [&](int32_t nc, bool cuts, Plan &pl) {
+        pl.nc = nc;
+        pl.R = U >= 2 * nc ? U / nc - 1 : 0;
+        const int32_t T0 = pl.R * nc;  // first tail unit
+        pl.own.assign(nc, 0.0);
+        for (int32_t r = 0; r < pl.R; ++r)
+            for (int32_t k = 0; k < nc; ++k)
+                pl.own[k] += n_all[r * nc + ((r & 1) ? nc - 1 - k : k)] + kSkUnitCost;
+        const double W = cum.back() - cum[T0];
+        const double mean = cum.back() / nc;
+        std::vector<double> want(nc), pos(nc + 1, 0.0);
+        double sum_want = 0.0;
+        for (int32_t k = 0; k < nc; ++k) sum_want += (want[k] = std::max(0.0, mean - pl.own[k]));
+        for (int32_t k = 0; k < nc; ++k) pos[k + 1] = pos[k] + (sum_want > 0 ? want[k] * W / sum_want : W / nc);
+        pl.b.assign(nc + 1, SkBound{T0, 0});
+        pl.b[nc] = SkBound{U, 0};
+        for (int32_t k = 1; k < nc; ++k) {
+            const double x = cum[T0] + pos[k];
+            SkBound bd{U, 0};
+            if (x < cum.back()) {
+                const int32_t u = std::min(unit_at(x), U - 1);
+                const double off = x - cum[u];
+                const int32_t t = static_cast<int32_t>(std::lround(off - kSkUnitCost));
+                bd = SkBound{u, 0};
+                if (cuts && t >= kSkMinPiece && n_all[u] - t >= kSkMinPiece) bd.t = t;
+                else if (off > 0.5 * (n_all[u] + kSkUnitCost)) bd = SkBound{u + 1, 0};
+            }
+            const SkBound &prev = pl.b[k - 1];
+            if (bd.u < prev.u || (bd.u == prev.u && bd.t < prev.t)) bd = prev;  // an empty stretch
+            pl.b[k] = bd;
+        }
+    };
+    // the busiest CTA: its rounds plus its tail stretch (a cut piece pays its own set-up)
+    auto busiest = [&](const Plan &pl) {
+        auto at = [&](const SkBound &x) {
+            return (x.u < U ? cum[x.u] : cum.back()) + (x.t > 0 ? kSkUnitCost + x.t : 0.0);
+        };
+        double worst = 0.0;
+        for (int32_t k = 0; k < pl.nc; ++k) {
+            double tail = at(pl.b[k + 1]) - at(pl.b[k]);
+            if (tail > 0 && pl.b[k].t > 0) tail += kSkUnitCost;
+            worst = std::max(worst, pl.own[k] + tail);
+        }
+        return worst;
+    };
+    // cut units of a plan: slots and part counts; false when the partials do not fit
+    std::vector<int32_t> slot_of;
+    std::vector<int32_t> cuts_in;  // interior boundaries per cut unit
+    int32_t n_slots = 0, max_parts = 1;
+    auto slots_for = [&](const std::vector<SkBound> &bb) {
+        slot_of.assign(U, -1);
+        cuts_in.clear();
+        n_slots = 0;
+        max_parts = 1;
+        for (const SkBound &x : bb) {
+            if (x.t <= 0 || x.u >= U) continue;
+            if (slot_of[x.u] < 0) {
+                slot_of[x.u] = n_slots++;
+                cuts_in.push_back(0);
+            }
+            cuts_in[slot_of[x.u]] += 1;
+        }
+        for (int32_t k = 0; k < n_slots; ++k) max_parts = std::max(max_parts, cuts_in[k] + 1);
+        const int64_t rows = static_cast<int64_t>(n_slots) * max_parts * 2 * kBM;
+        return n_slots <= kMaxSkCtas && max_parts <= 32 && rows * (static_cast<int64_t>(d) * 4 + 4) <= c->ws_bytes;
+    };
+
+    // CTAs: one per SM, fewer when the work is small (about 3 cost units each at least)
+    int32_t n_cta = static_cast<int32_t>(std::min<int64_t>(
+        std::min<int64_t>(c->num_sms, kMaxSkCtas), std::max<int64_t>(1, static_cast<int64_t>(cum.back() / 3.0))));
+    if (c->attn_ctas > 0) n_cta = std::min(c->attn_ctas, kMaxSkCtas);
+    Plan whole, cut;
+    make(n_cta, false, whole);
+    bool cuts = false;
+    if (c->splitkv != 0) {
+        // fewer CTAs when a unit would be cut into more than 32 parts or the partials overflow the workspace
+        for (int32_t nc = n_cta; nc >= 2; nc = std::min(nc - 1, nc * 31 / std::max<int32_t>(max_parts, 32))) {
+            make(nc, true, cut);
+            if (!slots_for(cut.b)) continue;
+            if (n_slots > 0 && (c->splitkv == 1 || busiest(cut) + 2.0 < 0.95 * busiest(whole))) cuts = true;
+            break;
+        }
+    }
+    const Plan &pl = cuts ? cut : whole;
+    if (!cuts) {
+        n_slots = 0;
+        max_parts = 1;
+    }
+    P.n_ctas = pl.nc;
+    P.rounds = pl.R;
+    P.n_slots = n_slots;
+    P.max_parts = max_parts;
+    if (cuts) {
+        for (int32_t u = 0; u < U; ++u)
+            if (slot_of[u] >= 0) P.slots[slot_of[u]] = SkSlot{u, cuts_in[slot_of[u]] + 1};
+        p.part_o = c->d_ws;
+        p.part_lse = c->d_ws + static_cast<int64_t>(n_slots) * max_parts * 2 * kBM * d;
+    }
+    for (int32_t k = 0; k < pl.nc; ++k) {
+        const SkBound &a = pl.b[k], &z = pl.b[k + 1];
+        SkCta &w = P.cta[k];
+        w.slot0 = w.slot1 = -1;
+        w.part0 = w.part1 = 0;
+        if (a == z) {  // no tail stretch
+            w.u0 = 1;
+            w.u1 = 0;
+            w.t0 = w.t1 = 0;
+            continue;
+        }
+        w.u0 = a.u;
+        w.t0 = a.t;
+        w.u1 = z.u;
+        w.t1 = z.t;
+        if (cuts && slot_of[a.u] >= 0) {
+            w.slot0 = slot_of[a.u];
+            int32_t part = 0;  // interior boundaries of unit a.u at or before tile a.t
+            for (const SkBound &x : pl.b)
+                if (x.u == a.u && x.t > 0 && x.t <= a.t) ++part;
+            w.part0 = part;
+        }
+        if (cuts && z.u != a.u && z.t > 0) {
+            w.slot1 = slot_of[z.u];
+            w.part1 = 0;
+        }
+    }
+    return PE_OK;
+}
+
 pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t layer, const void *Q,
                         int64_t q_rows, void *out, int32_t hq, float scale, cudaStream_t st)
 {
@@ -948,6 +1151,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
 
     std::vector<char> pbuf(sizeof(AttnParams));
     AttnParams &p = *reinterpret_cast<AttnParams *>(pbuf.data());
+    std::vector<char> sbuf;
     for (size_t lo = 0; lo < order.size(); lo += kMaxSegs) {
         const size_t hi = std::min(order.size(), lo + kMaxSegs);
         bool split = false;
@@ -955,6 +1159,37 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         if (s != PE_OK) return s;
         TailPlan tp;
         const bool tail = hi - lo == 1 && c->splitkv == -1 && c->num_splits == 0 && plan_tail(order[lo], tp);
+        // The persistent stream-K kernel where the one-item plan leaves SMs idle (it needs key splits
+        // or a tail launch) and its units fill between a quarter of the SMs and two waves: one CTA
+        // per SM, whole units in rounds, the rest cut into equal stretches.  Elsewhere the one-item
+        // kernel, whose tile loop runs a little faster (measured: short suffix 195 -> 184 us and
+        // tau/T 0.9 311 -> 303 us with the persistent kernel; tau/T 0.7 716 -> 749 us and the
+        // 8-unit tiny launch 14 -> 16 us without it).
+        int64_t units = 0;
+        for (size_t i = lo; i < hi; ++i)
+            units += ceil_div(ceil_div(static_cast<int64_t>(order[i].n_q) * g, kBM), 2) * hkv;
+        const bool sk_fits = 4 * units >= c->num_sms && units < 2 * static_cast<int64_t>(c->num_sms);
+        const bool sk = c->num_splits == 0 &&
+                        (c->attn_kernel == 2 || (c->attn_kernel == 1 && (split || tail) && sk_fits));
+        if (sk) {
+            if (sbuf.empty()) sbuf.resize(sizeof(SkParams));
+            SkParams &P = *reinterpret_cast<SkParams *>(sbuf.data());
+            if ((s = plan_sk(c, order, lo, hi, layer, out, hq, scale, P)) != PE_OK) return s;
+            c->last_split = P.n_slots > 0 ? 1 : 0;
+            c->last_splits = P.max_parts;
+            c->last_ctas = P.n_ctas;
+            if (injected_failure(c)) return launch_fault("replay attention");
+            cudaError_t e = launch_replay_attn_sk(d, tm_q, c->tm_k, c->tm_v, P, st);
+            if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
+            c->launches++;
+            if (P.n_slots > 0) {
+                if (injected_failure(c)) return launch_fault("split-KV combine");
+                e = launch_sk_combine(d, P, st);
+                if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
+                c->launches++;
+            }
+            continue;
+        }
         if (tail && split) {  // the first launch runs unsplit: re-plan the group without splits
             s = plan_group(lo, hi, p, split, 0);
             if (s != PE_OK) return s;
@@ -1609,6 +1844,12 @@ pe_status pe_set_option(pe_cache *c, const char *key, int64_t value)
     } else if (!std::strcmp(key, "decode_kernel")) {
         if (value < 0 || value > 2) return fail(PE_ERR_INVALID, "decode_kernel must be 0, 1 or 2");
         c->decode_kernel = static_cast<int>(value);
+    } else if (!std::strcmp(key, "attn_kernel")) {
+        if (value < 0 || value > 2) return fail(PE_ERR_INVALID, "attn_kernel must be 0, 1 or 2");
+        c->attn_kernel = static_cast<int>(value);
+    } else if (!std::strcmp(key, "attn_ctas")) {
+        if (value < 0 || value > kMaxSkCtas) return fail(PE_ERR_INVALID, "attn_ctas must be 0..%d", kMaxSkCtas);
+        c->attn_ctas = static_cast<int>(value);
     } else if (!std::strcmp(key, "fail_launch_after")) {
         if (value < -1) return fail(PE_ERR_INVALID, "fail_launch_after must be -1 (off) or >= 0");
         c->fail_after = value;

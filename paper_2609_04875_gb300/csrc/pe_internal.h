@@ -16,6 +16,7 @@ constexpr int kAppendMaxPages = 3072;  // new page ids carried by one append lau
 
 // Device status word codes (pe_device_status).
 constexpr int kStatusWaitTimeout = 1;
+constexpr int kStatusBadPlan = 3;      // the persistent kernel met a partial slot outside its workspace (skipped)
 
 // ---------------------------------------------------------------- append
 struct AppendSeg {
@@ -98,6 +99,37 @@ struct AttnParams {
     AttnSeq seqs[kMaxSegs];
 };
 
+// ---------------------------------------------------------------- persistent (stream-K) attention
+// A launch group's work units are (sequence, kv-head, q-tile pair), numbered
+// sequence by sequence from AttnSeq::item0 (kv-head fastest, pairs heaviest
+// first); a unit loads the key tiles [0, n) of its pair.  The persistent
+// kernel runs one CTA per SM: whole units in lockstep rounds, then CTA c's
+// contiguous stretch of the remaining (unit, key tile) work; the pieces of
+// units cut by a stretch boundary write fp32 partials (O / l and log2-sum-exp)
+// into slot `slot`, part `part`, and a combine launch merges each slot's parts.
+constexpr int kMaxSkCtas = 160;        // >= SMs of the GPU
+
+struct SkCta {
+    int32_t u0, t0;        // first unit and its first key tile
+    int32_t u1, t1;        // last unit and the key tile it stops before (t1 = 0: u1 is not taken)
+    int32_t slot0, part0;  // partial slot and part of u0's piece (slot -1: the whole unit, written directly)
+    int32_t slot1, part1;  // the same for u1's piece when u1 > u0
+};
+
+struct SkSlot {
+    int32_t unit;          // the unit cut into parts
+    int32_t n_parts;
+};
+
+struct SkParams {
+    AttnParams a;          // sequences, shapes, output; part_o / part_lse hold the partials
+    int32_t n_ctas, n_slots, max_parts;
+    int32_t rounds;        // whole units first: in round r < rounds CTA k takes unit r n_ctas + k (odd r:
+                           // r n_ctas + n_ctas - 1 - k); then its tail stretch (cta[k], u0 > u1: none)
+    SkCta cta[kMaxSkCtas];
+    SkSlot slots[kMaxSkCtas];
+};
+
 // ---------------------------------------------------------------- decode attention
 // Sequences whose queries pack into at most kDecMaxRows rows per kv-head
 // (n_q x group) take the decode kernel (pe_decode.cu): CUDA cores, 64-key
@@ -160,6 +192,10 @@ cudaError_t launch_cow_copy(uint4 *k_pool, uint4 *v_pool, int32_t src, int32_t d
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
                                const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);
+// Persistent stream-K attention (p.n_ctas CTAs) and the merge of its cut units (p.n_slots > 0).
+cudaError_t launch_replay_attn_sk(int head_dim, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
+                                  const CUtensorMap &tm_v, const SkParams &p, cudaStream_t st);
+cudaError_t launch_sk_combine(int head_dim, const SkParams &p, cudaStream_t st);
 // rows_cap: 4, 8 or 16 (every sequence's n_q x group fits).
 // tm_k / tm_v: the pools as 2-D maps {d, L*num_pages*Hkv*ps} with 64 x min(ps, 64) boxes, 128-byte swizzle.
 // tensor_core (d = 128 only): keys on the MMA's M side, 128-key tiles (split_tiles

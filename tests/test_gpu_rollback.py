@@ -81,8 +81,9 @@ def test_failed_calls_leave_cache_and_mirror_unchanged():
             assert_close(out, ref, f"after rollbacks, seq {s} layer {layer}")
     # an attention call that fails leaves nothing behind either
     pair.gpu.set_option("splitkv", 1)
+    pair.gpu.set_option("num_splits", 2)          # two key splits: an attention launch, then a combine launch
     q = dev(synth.normal_bf16(g, (30, hq, d)))
-    pair.gpu.set_option("fail_launch_after", 1)   # the combine launch after the split-KV attention
+    pair.gpu.set_option("fail_launch_after", 1)   # the combine launch
     with pytest.raises(binding.PEError):
         pair.gpu.replay_attn(a, 0, q, softmax_scale=scale)
     pair.gpu.set_option("fail_launch_after", -1)

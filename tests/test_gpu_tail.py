@@ -1,6 +1,7 @@
-"""The tail launch of the replay-attention path: one sequence whose q-tile
-pairs leave the last wave of CTAs mostly empty runs its lightest pairs in a
-second, split-KV launch over every SM.  Rows of both launches against the
+"""The tail launch of the one-work-item-per-CTA attention kernel (option
+"attn_kernel" = 0): one sequence whose q-tile pairs leave the last wave of
+CTAs mostly empty runs its lightest pairs in a second, split-KV launch over
+every SM.  Rows of both launches against the
 oracle (every row of the tail pairs, a sample of the rest), and the same rows
 with the tail launch off (uniform plan) for comparison."""
 import math
@@ -20,6 +21,7 @@ def _case(n_q, prefix, seed, d=128, hq=32, hkv=8, ps=16):
     n = prefix + n_q
     npg = -(-n // ps) + 4
     pair = Pair(1, hkv, d, ps, npg, 1, npg, seed=seed)
+    pair.gpu.set_option("attn_kernel", 0)
     g = synth.rng(seed, 41)
     s = pair.seq()
     pair.append(s, synth.normal_bf16(g, (1, n, hkv, d)), synth.normal_bf16(g, (1, n, hkv, d)))
