@@ -308,18 +308,27 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "agent_batch": {"bytes": 696.787712e6 + 328.413184e6, "profile": "profiles/replay_attn_agent_batch.md",
-                    "src_sha256": "7189e778c5f940b1c537cf93b422f5087750bc5f64e748a579bd47bb8bdff10d"},
-    "short_suffix": {"bytes": 1.076235e9 + 21.172736e6, "profile": "profiles/replay_attn_splitkv_short_suffix.md",
-                     "src_sha256": "7189e778c5f940b1c537cf93b422f5087750bc5f64e748a579bd47bb8bdff10d"},
+    "tiny": {"bytes": 1.518592e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
+             "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100"}},
+    "agent_batch": {"bytes": 695.139072e6 + 327.651328e6, "profile": "profiles/replay_attn_agent_batch.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100"}},
+    "short_suffix": {"bytes": 1.077033216e9 + 6.493184e6, "profile": "profiles/replay_attn_sk_short_suffix.md",
+                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f3856241b4b16f861c6be6b07d1731e7f4f0f11fd357d69f392aef397889e2ee"}},
+    "long_suffix": {"bytes": 4.61800832e9 + 1.176607232e9, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100"}},
+    # mean over the 160 attention launches of one sweep step (5 forget requests x 32 layers)
+    "tau_sweep": {"bytes": 198.352832e6 + 41.8683744e6, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100", "prefill_sk": "f3856241b4b16f861c6be6b07d1731e7f4f0f11fd357d69f392aef397889e2ee"}},
     "decode_batch": {"bytes": 341.564672e6 + 4.737536e6, "profile": "profiles/decode_tc_decode_batch.md",
-                     "kernel": "decode",
-                     "src_sha256": "ebdfb149b87b25a869e6dbdd23d758b653f850efdd292555c54f0ecf44542551"},
+                     "kernels": ["decode"],
+                     "src_sha256": {"decode": "ebdfb149b87b25a869e6dbdd23d758b653f850efdd292555c54f0ecf44542551"}},
 }
 CSRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc")
 # (file, first line of the kernel's source, the text that follows it): the span that is hashed
 KERNEL_SRC = {
     "prefill": ("pe_attn.cu", "template <int HD, bool SPLIT>\n__global__", "// Exercises the bounded wait on its own"),
+    "prefill_sk": ("pe_attn_sk.cu", "template <int HD>\n__global__ void __launch_bounds__(kThreads, 1)\n"
+                   "    replay_attn_sk_kernel", "// One warp per row of a cut unit's q-tile"),
     "decode": ("pe_decode.cu", "template <int RB>\n__global__ void __launch_bounds__(kTcThreads, 1)",
                "template <int RB>\ncudaError_t launch_tc("),
 }
@@ -341,8 +350,10 @@ def _src_sha(kernel="prefill"):
 
 
 def traffic_for(workload):
+    """Recorded DRAM bytes per attention launch of `workload`, or None when any
+    kernel it launches has changed since the capture."""
     t = NCU_TRAFFIC.get(workload)
-    if not t or t["src_sha256"] != _src_sha(t.get("kernel", "prefill")):
+    if not t or any(t["src_sha256"][k] != _src_sha(k) for k in t["kernels"]):
         return None, None
     return t["bytes"], t["profile"]
 
@@ -654,14 +665,17 @@ def measure(name, args, rank, world, local_rank, dev, peaks, peak_src, headline)
         "gated_definition": "the same attention launches timed behind a busy kernel, so no host gap is inside "
                             "the events",
     }
+    tr, prof = traffic_for(name)
+    rep["roofline"]["traffic"], rep["roofline"]["traffic_profile"] = tr, prof
     if len(units) == 1:
         rep["roofline"]["plan"] = reports[0]["plan"]
         rep["roofline"]["units_per_launch"] = reports[0]["units_per_launch"]
-        tr, prof = traffic_for(units[0].w.name)
-        rep["roofline"]["traffic"], rep["roofline"]["traffic_profile"] = tr, prof
         rep.update({k: reports[0][k] for k in ("append_ms", "attention_ms_all_layers")})
     else:
-        rep["roofline"]["traffic"] = None
+        rep["roofline"]["units_per_launch"] = {
+            "requests": len(units), "suffix_tokens": sum(u.S for u in units),
+            "keys": sum(a.T for u in units for a in u.w.agents), "layers": units[0].L,
+            "note": "per-launch figures are means over the step's launches (one per layer and request)"}
         rep["per_request"] = {u.label: r for u, r in zip(units, reports)}
     rep["crop_us"] = {"kernel_median": median([g["crop_kernel_us"] for g in gated]),
                       "host_call_median": median([g["crop_host_us"] for g in gated]),

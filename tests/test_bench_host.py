@@ -1,8 +1,12 @@
 """Host-side pieces of bench.py that need no GPU: the workload table, the
 algorithmic units, and the kernel-source hashes that keep recorded ncu
 traffic valid only for the kernel version it was captured on."""
+import os
+
 import bench
 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def test_every_named_workload_builds():
@@ -27,8 +31,10 @@ def test_kernel_source_spans_are_found():
         h = bench._src_sha(kernel)
         assert h is not None and len(h) == 64, kernel
     for wl, t in bench.NCU_TRAFFIC.items():
-        assert t.get("kernel", "prefill") in bench.KERNEL_SRC, wl
+        assert t["kernels"] and all(k in bench.KERNEL_SRC for k in t["kernels"]), wl
+        assert set(t["src_sha256"]) == set(t["kernels"]), wl
         assert t["bytes"] > 0 and t["profile"].startswith("profiles/"), wl
+        assert os.path.exists(os.path.join(ROOT, t["profile"])), wl
 
 
 def test_reference_arm_prints_one_contract_line():
