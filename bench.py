@@ -329,8 +329,8 @@ KERNEL_SRC = {
     "prefill": ("pe_attn.cu", "template <int HD, bool SPLIT>\n__global__", "// Exercises the bounded wait on its own"),
     "prefill_sk": ("pe_attn_sk.cu", "template <int HD>\n__global__ void __launch_bounds__(kThreads, 1)\n"
                    "    replay_attn_sk_kernel", "// One warp per row of a cut unit's q-tile"),
-    "decode": ("pe_decode.cu", "template <int RB>\n__global__ void __launch_bounds__(kTcThreads, 1)",
-               "template <int RB>\ncudaError_t launch_tc("),
+    "decode": ("pe_decode.cu", "template <int HD, int RB>\n__global__ void __launch_bounds__(kTcThreads, 1)",
+               "template <int HD, int RB>\ncudaError_t launch_tc("),
 }
 
 
@@ -388,9 +388,7 @@ def kernel_name(w, plan):
     rows = max(a.S for a in w.agents) * (w.num_q_heads // w.num_kv_heads)
     if rows <= 16:  # every sequence's query rows fit the decode kernel
         rb = 4 if rows <= 4 else (8 if rows <= 8 else 16)
-        if w.head_dim == 128:
-            return f"decode_tc_kernel<{rb}> (+ decode_tc_combine_kernel<{rb}> for split items)"
-        return f"decode_attn_kernel<{w.head_dim},{rb}> (split-KV merged in-kernel)"
+        return f"decode_tc_kernel<{w.head_dim},{rb}> (+ decode_tc_combine_kernel<{w.head_dim},{rb}> for split items)"
     return f"replay_attn_kernel<{w.head_dim},{'split' if plan[0] else 'single'}> (+ splitkv_combine when split)"
 
 

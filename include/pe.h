@@ -253,10 +253,16 @@ pe_status pe_cache_pools(const pe_cache *cache, void **k_pool, void **v_pool);
  * fills freed pages and the stale tail of the last kept page with a finite
  * sentinel (bf16 2^100), so that a kernel reading them unmasked gives a
  * visibly wrong result; "decode_kernel" = 1 (default) / 2 / 0: sequences
- * whose n_q x (Hq/Hkv) query rows fit in 16 take a decode kernel with the
- * split-KV merge done in-kernel -- 1: tcgen05 with keys on the MMA's M side
- * for d = 128, CUDA cores for d = 64; 2: CUDA cores for both; 0: no decode
- * kernel (the prefill kernel serves every call); "fail_launch_after" = k >= 0
+ * whose n_q x (Hq/Hkv) query rows fit in 16 take a decode kernel -- 1:
+ * tcgen05 with keys on the MMA's M side (d = 64 and 128), split items merged
+ * by a combine launch; 2: CUDA cores, split-KV merged in-kernel; 0: no
+ * decode kernel (the prefill kernel serves every call); "attn_kernel" = 1
+ * (default) / 2 / 0: the prefill kernel -- 1: the persistent stream-K kernel
+ * for launch groups whose one-work-item-per-CTA plan would need key splits or
+ * a tail launch and whose q-tile pairs x Hkv number between a quarter of the
+ * SMs and two waves, the one-item kernel otherwise; 2: always persistent; 0:
+ * always one-item; "attn_ctas" = 0 (auto) or the persistent kernel's CTA
+ * count; "fail_launch_after" = k >= 0
  * (test hook): the device step after the next k fails with PE_ERR_CUDA
  * without being launched, once (-1 = off); on a host-only cache the steps a
  * device cache would launch are counted the same way.  Split

@@ -440,13 +440,15 @@ __global__ void __launch_bounds__(kDecThreads, DecCfg<HD, RB>::kMinBlocks)
 }
 
 // ============================================================================
-// d = 128: tensor-core form.  With keys on the M side of the MMA the few query
-// rows become N = 16 (rows padded):
+// Tensor-core form (d = 128 and d = 64).  With keys on the M side of the MMA
+// the few query rows become N = 16 (rows padded):
 //     S^T [128 keys x 16] = K [128 x d] . Q^T          (A = K tile, B = Q; K-major)
 //     O^T [d x 16]       += V^T [d x 128 keys] . P^T   (A = V tile, MN-major; B = P^T, K-major)
 // both accumulated in TMEM (lane = key for S^T, lane = d-column for O^T), so a
 // softmax thread owns one key and touches only its RB valid row values per
-// 128-key tile.
+// 128-key tile.  For d = 64 the O^T GEMM keeps M = 128: the A operand's second
+// 64-row half (d-columns 64..127) is a zero-filled shared-memory region beside
+// each V stage, so O^T rows 64..127 stay zero and only the first 64 are read.
 //
 // Persistent, dynamically scheduled: every (sequence, kv-head) item's 128-key
 // tiles are cut into chunks of at most 8 tiles (the host picks about three
@@ -495,10 +497,12 @@ constexpr int kDescInts = 8 + 8 * 16;              // header, then the row of bo
 constexpr int kBarSoftmax = 2;                     // named barrier of the softmax warps
 constexpr float kTcWeightLimit = 1.8446744e19f;    // 2^64
 
-template <int RB>
+template <int HD, int RB>
 struct TcCfg {
+    static constexpr int kRegs = HD / 64;                   // 64-column halves of a K, V or Q row
     static constexpr int kRegionBytes = kTcKeys * 128;      // 128 keys x 64 columns (bf16), 128-byte swizzle
-    static constexpr int kTileBytes = 2 * kRegionBytes;     // one K or V tile
+    static constexpr int kTileBytes = 2 * kRegionBytes;     // one K or V stage (d = 64: V's second half is zeros)
+    static constexpr int kLoadBytes = kTcKeys * HD * 2;     // bytes the TMA boxes of one tile deliver
     static constexpr int kOffV = kTcKStages * kTileBytes;   // K ring, then V ring
     static constexpr int kOffQ = (kTcKStages + kTcVStages) * kTileBytes;  // Q x2: [16 rows][128] bf16, 2 x 2 KB each
     static constexpr int kOffP = kOffQ + 2 * 4096;          // P^T x2: [16 rows][128 keys] bf16, 2 regions x 2 KB each
@@ -517,6 +521,7 @@ struct TcCfg {
     static constexpr uint32_t kTmemCols = 64;               // S^T buffers at 0 and 16, O^T buffers at 32 and 48
     static_assert(kDynSmem <= 232448, "shared memory budget");
     static_assert(RB == 4 || RB == 8 || RB == 16, "row capacity");
+    static_assert(HD == 64 || HD == 128, "head dim");
 };
 
 // A chunk: tiles [t0, t1) of item (sequence si, kv-head kvh).  An item has
@@ -568,13 +573,12 @@ __device__ __forceinline__ ChunkInfo tc_chunk(const DecodeParams &p, const Decod
     return ci;
 }
 
-template <int RB>
+template <int HD, int RB>
 __global__ void __launch_bounds__(kTcThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                      const __grid_constant__ DecodeParams p)
 {
-    using C = TcCfg<RB>;
-    constexpr int HD = 128;
+    using C = TcCfg<HD, RB>;
     constexpr int R = kChunkRing;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -664,6 +668,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // both P^T buffers start at zero (rows past RB stay zero)
         for (int e = threadIdx.x; e < 2 * 4096 / 16; e += 128)
             reinterpret_cast<uint4 *>(smem + C::kOffP)[e] = make_uint4(0u, 0u, 0u, 0u);
+        if (HD == 64) {  // the zero second half of every V stage (d-columns 64..127 of the O^T GEMM's A)
+            for (int s = 0; s < kTcVStages; ++s)
+                for (int e = threadIdx.x; e < C::kRegionBytes / 16; e += 128)
+                    reinterpret_cast<uint4 *>(smem + C::kOffV + s * C::kTileBytes + C::kRegionBytes)[e] =
+                        make_uint4(0u, 0u, 0u, 0u);
+        }
         ptx::fence_proxy_async_smem();
     } else if (warp >= 7) {
         // the sequence table and the remainder order, read at every chunk by every role
@@ -687,15 +697,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (warp == 4 || warp == 6) {
         // ============================================================ producers (warp 4: K, warp 6: V)
-        // Each chunk's TMA rows come ready from the loader warp; lane 2 j + h issues box j (keys
+        // Each chunk's TMA rows come ready from the loader warp; lane kRegs j + h issues box j (keys
         // [j kpc, (j + 1) kpc) of the tile) of 64-column half h.
         const bool is_v = warp == 6;
         const CUtensorMap *map = is_v ? &tm_v : &tm_k;
         const int n_stages = is_v ? kTcVStages : kTcKStages;
         const int kpc = p.ps < kDecKeys ? p.ps : kDecKeys;  // keys per box (<= 64)
-        const int n_ops = (kTcKeys / kpc) * 2;              // boxes per tile, <= 32
-        const int op_slot = lane >> 1;
-        const int op_reg = lane & 1;
+        const int n_ops = (kTcKeys / kpc) * C::kRegs;       // boxes per tile, <= 32
+        const int op_slot = lane / C::kRegs;
+        const int op_reg = lane % C::kRegs;
         const bool op_on = lane < n_ops;
         int i = 0;  // tile ordinal in this CTA
         for (int n = 0;; ++n) {
@@ -713,7 +723,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     ok = false;
                     break;
                 }
-                if (lane == 0) ptx::mbar_arrive_expect_tx(b_full, C::kTileBytes);
+                if (lane == 0) ptx::mbar_arrive_expect_tx(b_full, C::kLoadBytes);
                 __syncwarp();
                 if (op_on) {
                     const uint32_t dst = sbase + (is_v ? C::kOffV : 0) + s * C::kTileBytes +
@@ -785,29 +795,33 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(b_desc_full + 8 * d);  // release: the producers read the rows
             if (c < 0) break;
-            // the chunk's Q rows into buffer n & 1 as [16 rows][128] bf16 (128-byte swizzle), rows past
-            // n_q x g zero; the buffer's previous chunk (n - 2) must be done with it
+            // the chunk's Q rows into buffer n & 1 as [16 rows][d] bf16 (128-byte swizzle, 64-column
+            // halves 2 KB apart), rows past n_q x g zero; the buffer's previous chunk (n - 2) must be
+            // done with it
             {
                 const ChunkInfo ci = tc_chunk(p, s_seqs, s_rem_seq, c);
                 const DecodeSeq &sq = s_seqs[ci.si];
                 const int n_rows = sq.n_q * g;
-                uint4 qv[8];
+                constexpr int kCols = HD / 8;     // 16-byte columns of a row
+                constexpr int kQj = 16 * kCols / 32;
+                uint4 qv[kQj];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {  // piece e = 32 j + lane: row e / 16, 16-byte column e % 16
+                for (int j = 0; j < kQj; ++j) {  // piece e = 32 j + lane: row e / kCols, 16-byte column e % kCols
                     const int e = 32 * j + lane;
-                    const int r = e >> 4;
+                    const int r = e / kCols;
                     qv[j] = make_uint4(0u, 0u, 0u, 0u);
                     if (r < n_rows)
                         qv[j] = *reinterpret_cast<const uint4 *>(
                             static_cast<const __nv_bfloat16 *>(p.q) +
-                            (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + ci.kvh * g + r % g) * HD + (e & 15) * 8);
+                            (static_cast<int64_t>(sq.q_row0 + r / g) * p.hq + ci.kvh * g + r % g) * HD +
+                            (e % kCols) * 8);
                 }
                 if (n >= 2 && !wait_bar_warp(b_q_free + 8 * (n & 1), ((n - 2) >> 1) & 1, wctx)) break;
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
+                for (int j = 0; j < kQj; ++j) {
                     const int e = 32 * j + lane;
-                    const int r = e >> 4;
-                    const int cc = e & 15;
+                    const int r = e / kCols;
+                    const int cc = e % kCols;
                     *reinterpret_cast<uint4 *>(smem + C::kOffQ + (n & 1) * 4096 + (cc >> 3) * 2048 + r * 128 +
                                                (((cc & 7) ^ (r & 7)) << 4)) = qv[j];
                 }
@@ -860,7 +874,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                         const uint32_t ka = sbase + s * C::kTileBytes;
                         const uint32_t qa = q_smem + (ns_chunk & 1) * 4096;
 #pragma unroll
-                        for (int kk = 0; kk < 8; ++kk) {
+                        for (int kk = 0; kk < HD / 16; ++kk) {
                             const uint32_t off = (kk >> 2) * C::kRegionBytes + (kk & 3) * 32;
                             const uint32_t qoff = (kk >> 2) * 2048 + (kk & 3) * 32;
                             ptx::mma_bf16(t_s + 16 * (ns & 1), ptx::smem_desc_sw128(ka + off, 16, 1024),
@@ -1104,7 +1118,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             if (ci.cpi == 1) {
 #pragma unroll
                 for (int r = 0; r < RB; ++r) {
-                    if (r < n_rows) {
+                    if (r < n_rows && t < HD) {  // d = 64: O^T rows 64..127 are the zero half
                         const float inv = lsum[r] > 0.f ? 1.0f / lsum[r] : 0.f;
                         static_cast<__nv_bfloat16 *>(p.out)[(static_cast<int64_t>(sq.q_row0 + r / g) * p.hq +
                                                              ci.kvh * g + r % g) * HD + t] = __float2bfloat16_rn(o[r] * inv);
@@ -1117,8 +1131,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             float *po = p.part + static_cast<int64_t>(c) * RB * HD;
             float *pm = p.part + static_cast<int64_t>(p.total_tiles) * RB * HD;
             float *pl = pm + static_cast<int64_t>(p.total_tiles) * RB;
+            if (t < HD) {
 #pragma unroll
-            for (int r = 0; r < RB; ++r) po[r * HD + t] = o[r];
+                for (int r = 0; r < RB; ++r) po[r * HD + t] = o[r];
+            }
             if (et < RB) {
                 float mv = -INFINITY, lv = 0.f;
 #pragma unroll
@@ -1159,11 +1175,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // Merge of an item's chunk partials (one block per (sequence, kv-head), thread = d-column), after
 // the decode kernel: M = max_k m_k, O = sum_k 2^(m_k - M) O_k / sum_k 2^(m_k - M) l_k over the item's
 // chunks in its chunk order.  Items held in one chunk were written by the decode kernel itself.
-template <int RB>
+template <int HD, int RB>
 __global__ void __launch_bounds__(128) decode_tc_combine_kernel(const __grid_constant__ DecodeParams p)
 {
-    constexpr int HD = 128;
     ptx::griddep_wait();  // launched with programmatic serialization: the decode kernel's partials
+    if (static_cast<int>(threadIdx.x) >= HD) return;
     const int si = static_cast<int>(blockIdx.x) / p.hkv;
     const int kvh = static_cast<int>(blockIdx.x) - si * p.hkv;
     if (si >= p.n_seqs) return;
@@ -1229,14 +1245,14 @@ __global__ void __launch_bounds__(128) decode_tc_combine_kernel(const __grid_con
     }
 }
 
-template <int RB>
+template <int HD, int RB>
 cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st)
 {
-    using C = TcCfg<RB>;
+    using C = TcCfg<HD, RB>;
     static bool configured = false;
     if (!configured) {
         cudaError_t e =
-            cudaFuncSetAttribute(decode_tc_kernel<RB>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kDynSmem);
+            cudaFuncSetAttribute(decode_tc_kernel<HD, RB>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kDynSmem);
         if (e != cudaSuccess) return e;
         configured = true;
     }
@@ -1251,7 +1267,7 @@ cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const De
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<RB>, tm_k, tm_v, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<HD, RB>, tm_k, tm_v, p);
     if (e != cudaSuccess) return e;
     // the merges, also with programmatic serialization (its launch overlaps the decode grid's end)
     cudaLaunchConfig_t ccfg = {};
@@ -1261,7 +1277,7 @@ cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const De
     ccfg.stream = st;
     ccfg.attrs = attr;
     ccfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&ccfg, decode_tc_combine_kernel<RB>, p);
+    return cudaLaunchKernelEx(&ccfg, decode_tc_combine_kernel<HD, RB>, p);
 }
 
 template <int HD, int RB>
@@ -1286,10 +1302,15 @@ cudaError_t launch_decode_attn(int head_dim, int rows_cap, bool tensor_core, con
 {
     if (p.total_ctas <= 0) return cudaSuccess;
     if (tensor_core) {
-        if (head_dim != 128) return cudaErrorInvalidValue;
-        if (rows_cap == 4) return launch_tc<4>(tm_k, tm_v, p, st);
-        if (rows_cap == 8) return launch_tc<8>(tm_k, tm_v, p, st);
-        if (rows_cap == 16) return launch_tc<16>(tm_k, tm_v, p, st);
+        if (head_dim == 128) {
+            if (rows_cap == 4) return launch_tc<128, 4>(tm_k, tm_v, p, st);
+            if (rows_cap == 8) return launch_tc<128, 8>(tm_k, tm_v, p, st);
+            if (rows_cap == 16) return launch_tc<128, 16>(tm_k, tm_v, p, st);
+        } else if (head_dim == 64) {
+            if (rows_cap == 4) return launch_tc<64, 4>(tm_k, tm_v, p, st);
+            if (rows_cap == 8) return launch_tc<64, 8>(tm_k, tm_v, p, st);
+            if (rows_cap == 16) return launch_tc<64, 16>(tm_k, tm_v, p, st);
+        }
         return cudaErrorInvalidValue;
     }
     if (head_dim == 128) {

@@ -590,8 +590,8 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
     const int hkv = cf.num_kv_heads;
     const int d = cf.head_dim;
     const int g = hq / hkv;
-    // d = 128: tensor-core form (128-key tiles, one CTA per SM); otherwise CUDA cores (64-key tiles, two per SM)
-    const bool tc = d == 128 && c->decode_kernel == 1;
+    // tensor-core form (128-key tiles, one CTA per SM) unless "decode_kernel" = 2: CUDA cores (64-key tiles)
+    const bool tc = (d == 128 || d == 64) && c->decode_kernel == 1;
     const int64_t tile_keys = tc ? 128 : kDecKeys;
     std::vector<char> pbuf(sizeof(DecodeParams));
     DecodeParams &p = *reinterpret_cast<DecodeParams *>(pbuf.data());
@@ -978,7 +978,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     for (const AttnItem &it : items) {
         if (it.n_q <= 0) continue;
         // (the tcgen05 decode kernel always splits keys across CTAs: "splitkv" = 0 keeps the prefill kernel)
-        const bool tc_nosplit = d == 128 && c->decode_kernel == 1 && c->splitkv == 0;
+        const bool tc_nosplit = c->decode_kernel == 1 && c->splitkv == 0;
         if (c->decode_kernel && static_cast<int64_t>(it.n_q) * g <= kDecMaxRows && (d == 64 || d == 128) && !tc_nosplit)
             dec.push_back(it);
         else

@@ -136,6 +136,18 @@ def test_decode_batch():
     assert torch.equal(first, drv.out)
 
 
+def test_decode_batch_d64():
+    """The decode batch with head dim 64: the tensor-core decode kernel's d = 64 form (O^T GEMM
+    over a zero upper half), split items merged by its combine launch."""
+    import copy
+    import math
+    w = copy.deepcopy(synth.decode_batch())
+    w.head_dim, w.softmax_scale, w.name = 64, 1.0 / math.sqrt(64), "decode_batch_d64"
+    drv, inputs = _run(w)
+    _check_bookkeeping(drv)
+    _check_attention(drv, inputs, range(len(w.agents)), [0], n_random=0)
+
+
 def test_decode_batch_std1():
     w = synth.with_std(synth.decode_batch(), 1.0)
     drv, inputs = _run(w)
