@@ -395,12 +395,16 @@ def kernel_name(w, plan):
 # ------------------------------------------------------------------ GPU timing passes
 def timed_pass(units, steps, stream, dist):
     """`steps` steps of every unit back to back, inputs resident in HBM.  Events
-    on the launching stream bracket each unit's step, its append and each of
-    its attention launches.  Returns the elapsed ms (max over ranks) and the
-    per-unit event times."""
+    on the launching stream bracket each attention launch, and each unit's step
+    when there are several units (the sweep's requests); a lone unit's step time
+    is the region's.  Few events per step, so that a host-bound step (the tiny
+    configuration) is not slowed by them.  Returns the elapsed ms (max over
+    ranks), the per-unit event times and the library's launch count."""
     import torch
     E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    ev = [[(E(), E(), E(), [(E(), E()) for _ in range(u.L)], E()) for _ in range(steps)] for u in units]
+    many = len(units) > 1
+    ev = [[((E(), E()) if many else None, [(E(), E()) for _ in range(u.L)]) for _ in range(steps)] for u in units]
+    calls = [u.drv._calls(None, None) for u in units]  # the step's prepared C-ABI calls
     launches0 = sum(u.drv.cache.kernel_launches() for u in units)
     barrier(dist)
     torch.cuda.synchronize()
@@ -408,31 +412,30 @@ def timed_pass(units, steps, stream, dist):
     with no_gc():
         t0.record(stream)
         for k in range(steps):
-            for u, e in zip(units, ev):
-                s0, a0, a1, attn, s1 = e[k]
-                drv = u.drv
-                s0.record(stream)
-                drv.crop()
-                a0.record(stream)
-                drv.append()
-                a1.record(stream)
-                for layer in range(u.L):
+            for (crop, append, attend), e in zip(calls, ev):
+                se, attn = e[k]
+                if many:
+                    se[0].record(stream)
+                crop()
+                append()
+                for layer, call in enumerate(attend):
                     attn[layer][0].record(stream)
-                    drv.attend(layer)
+                    call()
                     attn[layer][1].record(stream)
-                s1.record(stream)
+                if many:
+                    se[1].record(stream)
         t1.record(stream)
         torch.cuda.synchronize()
     barrier(dist)
     launches = sum(u.drv.cache.kernel_launches() for u in units) - launches0
+    elapsed = t0.elapsed_time(t1)
     per_unit = []
     for u, e in zip(units, ev):
         per_unit.append({
-            "step_ms": [s0.elapsed_time(s1) for s0, _, _, _, s1 in e],
-            "append_ms": [a0.elapsed_time(a1) for _, a0, a1, _, _ in e],
-            "attn_ms": [b.elapsed_time(c) for _, _, _, at, _ in e for b, c in at],
+            "step_ms": [se[0].elapsed_time(se[1]) for se, _ in e] if many else [elapsed / steps],
+            "attn_ms": [b.elapsed_time(c) for _, at in e for b, c in at],
         })
-    return reduce_max(t0.elapsed_time(t1), dist), per_unit, launches
+    return reduce_max(elapsed, dist), per_unit, launches
 
 
 def gated_pass(units, reps, stream):
@@ -482,10 +485,11 @@ def gated_pass(units, reps, stream):
 
 
 def unit_report(u, t, gated, peaks, peak_src, steps):
-    """Numbers of one unit from its timed-pass events `t` and gated times."""
+    """Numbers of one unit from its timed-pass events `t` and gated times (the
+    append's device time comes from the gated pass)."""
     ms_step = statistics.mean(t["step_ms"])
     attn_launch_s = statistics.mean(t["attn_ms"]) / 1e3
-    app_ms = statistics.mean(t["append_ms"])
+    app_ms = gated["append_ms"]
     kern = roofline(u.flops_launch, u.bytes_launch, attn_launch_s, peaks, peak_src)
     attn_step_ms = attn_launch_s * 1e3 * u.L
     step = roofline(u.flops_step, u.bytes_step, (app_ms + attn_step_ms) / 1e3, peaks, peak_src)
@@ -658,7 +662,8 @@ def measure(name, args, rank, world, local_rank, dev, peaks, peak_src, headline)
         "roofline_ms_per_launch": kern["roofline_s"] * 1e3 / n_launch,
         "step_frac": step_roof / step_meas,
         "step_frac_definition": "roofline time of append + attention (max of FLOP at bf16 peak, step bytes at "
-                                "HBM peak) over their measured device time",
+                                "HBM peak) over their measured device time (attention: the timed region's "
+                                "events; append: the busy-gated pass)",
         "gated_frac": kern_g["frac"],
         "gated_definition": "the same attention launches timed behind a busy kernel, so no host gap is inside "
                             "the events",

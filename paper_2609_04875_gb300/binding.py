@@ -391,6 +391,55 @@ class PagedKVCache:
                                      Q.shape[2], scale, self._s(stream)))
         return out
 
+    # -- prepared calls ----------------------------------------------------------
+    # A caller repeating the same call (the same sequences, buffers and stream,
+    # e.g. one step of a benchmark loop) can validate and marshal its arguments
+    # once: each prepare_* checks them like the plain method and returns a
+    # function of no arguments that only calls the library.  The tensors are
+    # kept alive by the returned function; their contents may change between
+    # calls, their storage may not.
+    def prepare_crop_batch(self, seqs, taus, stream=None):
+        args = (self._h, len(seqs), _i32_array(seqs), _i64_array(taus), self._s(stream))
+        fn = _lib.pe_crop_batch
+
+        def call():
+            rc = fn(*args)
+            if rc:
+                _check(rc)
+        return call
+
+    def prepare_append_kv_batch(self, seqs, K, V, cu_tokens, stream=None):
+        self._check_kv(K, V)
+        if K.shape[1] != cu_tokens[-1]:
+            raise ValueError("K token count does not match cu_tokens")
+        keep = (K, V)
+        args = (self._h, len(seqs), _i32_array(seqs), _dev_ptr(K, "K"), _dev_ptr(V, "V"), _i32_array(cu_tokens),
+                self._s(stream))
+        fn = _lib.pe_append_kv_batch
+
+        def call():
+            rc = fn(*args)
+            if rc:
+                _check(rc)
+            return keep
+        return call
+
+    def prepare_replay_attn_batch(self, seqs, layer, Q, cu_q, out, softmax_scale=None, stream=None):
+        if Q.dim() != 3 or Q.shape[2] != self.head_dim or Q.shape[0] != cu_q[-1] or out.shape != Q.shape:
+            raise ValueError("Q and out must be [cu_q[-1]][Hq][d]")
+        scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
+        keep = (Q, out)
+        args = (self._h, len(seqs), _i32_array(seqs), int(layer), _dev_ptr(Q, "Q"), _i32_array(cu_q),
+                _dev_ptr(out, "out"), Q.shape[1], ctypes.c_float(scale), self._s(stream))
+        fn = _lib.pe_replay_attn_batch
+
+        def call():
+            rc = fn(*args)
+            if rc:
+                _check(rc)
+            return keep
+        return call
+
     def replay_attn_static_scratch(self, seq, layer, Q, out=None, softmax_scale=None, stream=None):
         """pe_replay_attn_static_scratch: split-KV replay attention whose partials
         live in the library's fixed device array (the call allocates nothing)."""

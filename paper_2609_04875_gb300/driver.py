@@ -63,6 +63,7 @@ class ReplayDriver:
             self.Qc[:, lo:hi] = _dev(q, self.device)
             del k, v, q
         self.out = torch.empty_like(self.Qc)
+        self._prepared = {}
         if fill:
             self.fill_original()
 
@@ -79,29 +80,48 @@ class ReplayDriver:
         """The step's device buffers (K', V', Q', out)."""
         return self.Kc, self.Vc, self.Qc, self.out
 
+    def _calls(self, stream, bufs):
+        """The step's C-ABI calls for (stream, buffer set), validated and marshalled
+        once (binding.prepare_*): crop, append, one attention call per layer."""
+        from .binding import _stream
+        key = (_stream(stream).value,  # the stream the calls will use (the current one when None)
+               None if bufs is None else tuple(t.data_ptr() for t in bufs))
+        calls = self._prepared.get(key)
+        if calls is None:
+            K, V, Q, out = bufs or self.buffers()
+            c = self.cache
+            st = key[0]
+            calls = (c.prepare_crop_batch(self._seqs_c, self._taus_c, stream=st),
+                     c.prepare_append_kv_batch(self._seqs_c, K, V, self._cu_c, stream=st),
+                     [c.prepare_replay_attn_batch(self._seqs_c, layer, Q[layer], self._cu_c, out[layer],
+                                                  softmax_scale=self.w.softmax_scale, stream=st)
+                      for layer in range(self.w.num_layers)])
+            self._prepared[key] = calls
+        return calls
+
     def crop(self, stream=None):
-        self.cache.crop_batch(self._seqs_c, self._taus_c, stream=stream)
+        self._calls(stream, None)[0]()
 
     def append(self, stream=None, bufs=None):
-        K, V = (bufs or self.buffers())[:2]
-        self.cache.append_kv_batch(self._seqs_c, K, V, self._cu_c, stream=stream)
+        self._calls(stream, bufs)[1]()
 
     def attend(self, layer, stream=None, bufs=None):
-        Q, out = (bufs or self.buffers())[2:]
-        self.cache.replay_attn_batch(self._seqs_c, layer, Q[layer], self._cu_c, out=out[layer],
-                                     softmax_scale=self.w.softmax_scale, stream=stream)
+        self._calls(stream, bufs)[2][layer]()
 
     def step(self, stream=None, attn_events=None, bufs=None):
         """One forget request for every agent.  attn_events: optional list of
         (start, end) CUDA event pairs, one per layer, recorded around attention.
         bufs: optional (K', V', Q', out) device tensors shaped like buffers()."""
-        self.crop(stream)
-        self.append(stream, bufs)
-        for layer in range(self.w.num_layers):
-            if attn_events is not None:
+        crop, append, attend = self._calls(stream, bufs)
+        crop()
+        append()
+        if attn_events is None:
+            for call in attend:
+                call()
+        else:
+            for layer, call in enumerate(attend):
                 attn_events[layer][0].record(stream)
-            self.attend(layer, stream, bufs)
-            if attn_events is not None:
+                call()
                 attn_events[layer][1].record(stream)
         return (bufs or self.buffers())[3]
 
