@@ -26,6 +26,9 @@ __global__ void __launch_bounds__(256) append_kv_kernel(const __grid_constant__ 
 {
     // the attention launch that follows may start its set-up now; it waits for this grid's writes
     ptx::griddep_launch_dependents();
+    // launched with programmatic serialization: only the launch overlaps the previous kernel; every
+    // read and write here waits for it (a crop before may still be poisoning freed pages)
+    ptx::griddep_wait();
     // 1) mirror the new page ids and lengths into the device tables
     if (blockIdx.x == 0) {
         for (int s = 0; s < p.n_segs; ++s) {
@@ -79,8 +82,16 @@ cudaError_t launch_append(const AppendParams &p, int64_t chunks, cudaStream_t st
     const int64_t cap = static_cast<int64_t>(sms) * 8;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    append_kv_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(p, chunks);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(blocks));
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, append_kv_kernel, p, chunks);
 }
 
 // One block per cropped sequence.  Debug poison first overwrites the pages
@@ -89,6 +100,10 @@ cudaError_t launch_append(const AppendParams &p, int64_t chunks, cudaStream_t st
 // the table entries [keep, old_n) of this sequence become -1.
 __global__ void __launch_bounds__(256) crop_kernel(const __grid_constant__ CropParams p)
 {
+    // launched with programmatic serialization: the launch overlaps the previous kernel (an attention
+    // launch that may still read the pages this crop frees); every write here waits for it
+    ptx::griddep_launch_dependents();
+    ptx::griddep_wait();
     const CropSeg &sg = p.segs[blockIdx.x];
     int32_t *row = p.page_table + sg.table_row;
     if (p.poison) {
@@ -131,8 +146,16 @@ __global__ void __launch_bounds__(256) crop_kernel(const __grid_constant__ CropP
 cudaError_t launch_crop(const CropParams &p, cudaStream_t st)
 {
     if (p.n <= 0) return cudaSuccess;
-    crop_kernel<<<p.n, 256, 0, st>>>(p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(p.n));
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, crop_kernel, p);
 }
 
 __global__ void __launch_bounds__(256) table_copy_kernel(int32_t *page_table, int32_t src_row, int32_t dst_row,
