@@ -319,9 +319,9 @@ NCU_TRAFFIC = {
     # mean over the 160 attention launches of one sweep step (5 forget requests x 32 layers)
     "tau_sweep": {"bytes": 198.352832e6 + 41.8683744e6, "profile": "profiles/traffic_attention_configs.md",
                   "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100", "prefill_sk": "f3856241b4b16f861c6be6b07d1731e7f4f0f11fd357d69f392aef397889e2ee"}},
-    "decode_batch": {"bytes": 341.564672e6 + 4.737536e6, "profile": "profiles/decode_tc_decode_batch.md",
+    "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
-                     "src_sha256": {"decode": "ebdfb149b87b25a869e6dbdd23d758b653f850efdd292555c54f0ecf44542551"}},
+                     "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},
 }
 CSRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc")
 # (file, first line of the kernel's source, the text that follows it): the span that is hashed

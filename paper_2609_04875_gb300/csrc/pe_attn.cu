@@ -523,17 +523,23 @@ __global__ void __launch_bounds__(256) splitkv_combine_kernel(const __grid_const
     const int qi = qt * (kBM / g) + row / g;
     if (qi >= sq.n_q) return;
     const int64_t base = sq.part_row0 + static_cast<int64_t>(unit) * sq.n_splits * kBM + row;
-    float mx = -INFINITY;
-    for (int s = 0; s < sq.n_splits; ++s) mx = fmaxf(mx, p.part_lse[base + static_cast<int64_t>(s) * kBM]);
+    const int ns = sq.n_splits;
+    // the splits' LSEs in one round of loads (lane s holds split s's, s < 32), then their max
+    float my = lane < ns ? p.part_lse[base + static_cast<int64_t>(lane) * kBM] : -INFINITY;
+    float mx = my;
+    for (int s = 32 + lane; s < ns; s += 32) mx = fmaxf(mx, p.part_lse[base + static_cast<int64_t>(s) * kBM]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     constexpr int kPer = HD / 32;
     float acc[kPer];
 #pragma unroll
     for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
     float den = 0.f;
     if (mx != -INFINITY) {
-        for (int s = 0; s < sq.n_splits; ++s) {
+#pragma unroll 4
+        for (int s = 0; s < ns; ++s) {
             const int64_t r = base + static_cast<int64_t>(s) * kBM;
-            const float lse = p.part_lse[r];
+            const float lse = s < 32 ? __shfl_sync(0xffffffffu, my, s) : p.part_lse[r];
             if (lse == -INFINITY) continue;
             const float w = ex2(lse - mx);
             den += w;

@@ -73,8 +73,12 @@ int32_t pe::report_error(int32_t code, const char *msg)
 // Undo log of one C-ABI call's changes to the host bookkeeping.  Every change
 // a call makes goes through the journal helpers below; a call that fails after
 // changing the state (a kernel launch failed after pages were taken or given
-// back) replays the log backwards and re-mirrors the touched sequences'
-// device rows, so an error leaves the cache as it was before the call.
+// back) undoes them and re-mirrors the touched sequences' device rows, so an
+// error leaves the cache as it was before the call.  Kept small: a touched
+// sequence saves its table from the first changed entry; the free list saves
+// only the entries popped below its start height; reference counts are not
+// logged at all, since every change to one goes with a change of a table entry
+// of a touched sequence and is undone from the two tables' difference.
 struct SeqSave {
     int32_t seq;
     int32_t from;                // table entries [from, size0) are saved in `tail`
@@ -86,10 +90,10 @@ struct SeqSave {
 };
 
 struct Journal {
-    std::vector<std::pair<int8_t, int32_t>> stack_ops;  // (+1 push / -1 pop, page), in call order
-    std::vector<std::pair<int32_t, int32_t>> refs;      // (page, reference count before the change)
-    std::vector<SeqSave> seqs;                          // one per touched sequence
-    std::vector<int32_t> seq_index;                     // sequence -> index in seqs, -1 when untouched
+    size_t low = 0;                    // lowest free-list height the call reached (its start height first)
+    std::vector<int32_t> popped;       // entries of the start free list popped below `low`, in pop order
+    std::vector<SeqSave> seqs;         // one per touched sequence
+    std::vector<int32_t> seq_index;    // sequence -> index in seqs, -1 when untouched
 };
 
 struct pe_cache {
@@ -167,48 +171,51 @@ void j_seq(pe_cache *c, int32_t seq, int32_t from)
     }
 }
 
-void free_push(pe_cache *c, int32_t pg)
-{
-    c->free_stack.push_back(pg);
-    c->jr.stack_ops.emplace_back(static_cast<int8_t>(1), pg);
-}
+void free_push(pe_cache *c, int32_t pg) { c->free_stack.push_back(pg); }
 
 int32_t free_pop(pe_cache *c)
 {
     const int32_t pg = c->free_stack.back();
     c->free_stack.pop_back();
-    c->jr.stack_ops.emplace_back(static_cast<int8_t>(-1), pg);
+    Journal &j = c->jr;
+    if (c->free_stack.size() < j.low) {  // an entry of the start free list
+        j.low = c->free_stack.size();
+        j.popped.push_back(pg);
+    }
     return pg;
 }
 
-void set_ref(pe_cache *c, int32_t pg, int32_t v)
-{
-    c->jr.refs.emplace_back(pg, c->refs[pg]);
-    c->refs[pg] = v;
-}
+void set_ref(pe_cache *c, int32_t pg, int32_t v) { c->refs[pg] = v; }
 
 void journal_clear(pe_cache *c)
 {
     Journal &j = c->jr;
     for (const SeqSave &sv : j.seqs) j.seq_index[sv.seq] = -1;
     j.seqs.clear();
-    j.refs.clear();
-    j.stack_ops.clear();
+    j.popped.clear();
+    j.low = c->free_stack.size();
 }
 
-// Undoes the call's changes (newest first) and rewrites the device mirror
+// Undoes the call's changes and rewrites the device mirror
 // (table row and length) of every touched live sequence on `st`, after any
 // device work the call already enqueued.
 void rollback(pe_cache *c, cudaStream_t st)
 {
     Journal &j = c->jr;
-    for (auto it = j.refs.rbegin(); it != j.refs.rend(); ++it) c->refs[it->first] = it->second;
-    for (auto it = j.stack_ops.rbegin(); it != j.stack_ops.rend(); ++it) {
-        if (it->first > 0) c->free_stack.pop_back();
-        else c->free_stack.push_back(it->second);
-    }
+    // the free list: back to its start entries below `low`, then the popped ones in reverse pop order
+    c->free_stack.resize(j.low);
+    for (auto it = j.popped.rbegin(); it != j.popped.rend(); ++it) c->free_stack.push_back(*it);
     for (const SeqSave &sv : j.seqs) {
         std::vector<int32_t> &t = c->table[sv.seq];
+        // reference counts: one more for an entry the call removed or replaced, one fewer for one it added
+        const size_t now = t.size(), end = std::max<size_t>(now, static_cast<size_t>(sv.size0));
+        for (size_t i = sv.from; i < end; ++i) {
+            const int32_t was = i < static_cast<size_t>(sv.size0) ? sv.tail[i - sv.from] : -1;
+            const int32_t is = i < now ? t[i] : -1;
+            if (was == is) continue;
+            if (was >= 0) c->refs[was] += 1;
+            if (is >= 0) c->refs[is] -= 1;
+        }
         t.resize(sv.size0);
         std::copy(sv.tail.begin(), sv.tail.end(), t.begin() + sv.from);
         c->len[sv.seq] = sv.len;
@@ -323,16 +330,18 @@ void apply_crop(pe_cache *c, CropPlan &pl, int32_t *freed_out)
 {
     j_seq(c, pl.seq, pl.keep);
     std::vector<int32_t> &t = c->table[pl.seq];
-    std::vector<int32_t> freed_desc;
+    // the freed pages' ids are kept only for the caller and the debug poison
+    const bool keep_ids = freed_out != nullptr || c->debug_poison;
+    pl.freed.clear();
     for (int32_t e = pl.old_n - 1; e >= pl.keep; --e) {
         const int32_t pg = t[e];
         set_ref(c, pg, c->refs[pg] - 1);
         if (c->refs[pg] == 0) {
             free_push(c, pg);
-            freed_desc.push_back(pg);
+            if (keep_ids) pl.freed.push_back(pg);
         }
     }
-    pl.freed.assign(freed_desc.rbegin(), freed_desc.rend());
+    std::reverse(pl.freed.begin(), pl.freed.end());  // ascending logical order
     if (freed_out) std::copy(pl.freed.begin(), pl.freed.end(), freed_out);
     t.resize(pl.keep);
     c->len[pl.seq] = pl.new_len;
