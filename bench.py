@@ -508,7 +508,7 @@ def unit_report(u, t, gated, peaks, peak_src, steps):
         "roofline_ms_per_launch": kern["roofline_s"] * 1e3,
         "kernel_frac": kern["frac"], "kernel_bound": kern["bound"],
         "kernel_achieved": kern["achieved"], "kernel_unit": kern["unit"],
-        # section 8(d)'s step fraction: roofline time of append + attention over their measured time
+        # the step fraction: roofline time of append + attention over their measured device time
         "step_frac": step["frac"], "step_bound": step["bound"], "step_roofline_ms": step["roofline_s"] * 1e3,
         "append_ms": app_ms, "attention_ms_all_layers": attn_step_ms,
         "gated": {**gated, "attn_ms_per_launch": gated["attn_ms_all_layers"] / u.L, "kernel_frac": gk["frac"]},
@@ -640,7 +640,7 @@ def measure(name, args, rank, world, local_rank, dev, peaks, peak_src, headline)
         "value": world * S_step * steps / (elapsed_ms / 1e3), "unit": UNIT, "steps": steps,
         "ms_per_step": ms_per_step, "suffix_tokens_per_step": S_step, "gpu_launches": launches, "clocks": clk,
     }
-    # the attention kernel over every launch of the step, and the step fraction of section 8(d)
+    # the attention kernel over every launch of the step, and the step fraction (append + attention)
     attn_s = sum(statistics.mean(t["attn_ms"]) / 1e3 * u.L for u, t in zip(units, per_unit))
     flops = sum(u.flops_step for u in units)
     n_launch = sum(u.L for u in units)
