@@ -327,8 +327,7 @@ CSRC = os.path.join(ROOT, "paper_2609_04875_gb300", "csrc")
 # (file, first line of the kernel's source, the text that follows it): the span that is hashed
 KERNEL_SRC = {
     "prefill": ("pe_attn.cu", "template <int HD, bool SPLIT>\n__global__", "// Exercises the bounded wait on its own"),
-    "prefill_sk": ("pe_attn_sk.cu", "template <int HD>\n__global__ void __launch_bounds__(kThreads, 1)\n"
-                   "    replay_attn_sk_kernel", "// One warp per row of a cut unit's q-tile"),
+    "prefill_sk": ("pe_attn_sk.cu", "// Merge of one row of a cut unit's q-tile", "template <int HD>\ncudaError_t launch_sk_t("),
     "decode": ("pe_decode.cu", "template <int HD, int RB>\n__global__ void __launch_bounds__(kTcThreads, 1)",
                "template <int HD, int RB>\ncudaError_t launch_tc("),
 }

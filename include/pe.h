@@ -266,16 +266,18 @@ pe_status pe_cache_pools(const pe_cache *cache, void **k_pool, void **v_pool);
  * (test hook): the device step after the next k fails with PE_ERR_CUDA
  * without being launched, once (-1 = off); on a host-only cache the steps a
  * device cache would launch are counted the same way.  Split
- * partials and the decode kernel's merge counters live in the cache's
- * workspace, so attention calls on one cache must not overlap on the GPU
- * (issue them on one stream, or order the streams). */
+ * partials and the merge counters (decode kernel, persistent kernel) live in
+ * the cache's workspace, so attention calls on one cache must not overlap on
+ * the GPU (issue them on one stream, or order the streams). */
 pe_status pe_set_option(pe_cache *cache, const char *key, int64_t value);
 
 /* Synchronises `stream` and reads the device status word.  *code = 0 when no
  * kernel reported a problem, else the first recorded code (1 = a bounded
  * wait ran out; 2 = the decode kernel met a page id outside the pool and
- * skipped it).  clear != 0 resets it, and after a nonzero code also the decode
- * kernel's split-merge and scheduling counters.  Returns DEVICE_TIMEOUT if
+ * skipped it; 3 = the persistent kernel met a partial slot outside its
+ * workspace and skipped it).  clear != 0 resets it, and after a nonzero code
+ * also the split-merge counters of the decode and persistent kernels and the
+ * decode scheduler's.  Returns DEVICE_TIMEOUT if
  * *code != 0. */
 pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *stream);
 
@@ -288,8 +290,9 @@ pe_status pe_device_status(pe_cache *cache, int32_t *code, int32_t clear, void *
 pe_status pe_selftest_bounded_wait(pe_cache *cache, int64_t limit_ns, void *stream);
 
 /* Plan of the most recent replay-attention launch group on this cache: split
- * = 1 when the split-KV path ran (a combine launch followed the attention, or
- * the CUDA-core decode kernel merged in-kernel), n_splits = key splits of its
+ * = 1 when the split-KV path ran (a combine launch followed the attention, the
+ * persistent kernel cut units and merged their parts in-kernel, or the
+ * CUDA-core decode kernel merged in-kernel), n_splits = key splits of its
  * first sequence (of the tail launch, when one ran: a group of one sequence
  * whose last wave of CTAs would be mostly empty runs its lightest q-tile pairs
  * in a second, split-KV launch), ctas = attention CTAs launched in all. */

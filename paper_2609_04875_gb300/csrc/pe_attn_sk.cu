@@ -11,11 +11,13 @@
 // stretch of (unit, key tile) work, chosen on the host so that every CTA has
 // about the same number of key tiles plus per-unit overhead.  A unit cut by a
 // stretch boundary is computed in pieces (key ranges) by consecutive CTAs, each
-// writing fp32 partials (O / l and the row's log2-sum-exp); sk_combine_kernel
-// merges them.  Whole units write bf16 output directly.  So the last wave of
-// a launch is as full as the first, and a CTA's next unit starts loading while
-// its previous unit's epilogue runs (no CTA launch, TMEM allocation or barrier
-// set-up between units).
+// writing fp32 partials (O / l and the row's log2-sum-exp); per warp of 32 rows
+// a ticket counts the parts written, and the warp that writes a unit's last
+// part merges the parts into the bf16 output (no combine launch).  Whole units
+// write bf16 output directly.  So the last wave of a launch is as full as the
+// first, and a CTA's next unit starts loading while its previous unit's last
+// tile and epilogue run (no CTA launch, TMEM allocation or barrier set-up
+// between units).
 //
 // Roles (320 threads) as in replay_attn_kernel: softmax warpgroups 0 and 1
 // (one per q-tile, thread r owns row r), producer warp 8 (page table -> TMA
@@ -23,8 +25,8 @@
 // same sequence of pieces, computed from the kernel parameters; barrier phases
 // run on across pieces (per q-tile tile counts for S / P / O, a global key
 // tile count for the K and V rings, a piece count for Q).  Two more barriers
-// than the one-unit kernel: q_empty (the MMA's S GEMMs of a piece are done, so
-// Q may be reloaded) and o_free[t] (the softmax warps have read O_t out of
+// than the one-unit kernel: q_empty (the piece's last S GEMMs are done, so the
+// next piece's Q may load while its last tile's softmax and P V run) and o_free[t] (the softmax warps have read O_t out of
 // TMEM, so the next piece's first P V GEMM may overwrite it).
 //
 // Key tiles start at logical key 0 (multiples of 128 keys) whatever the
@@ -158,6 +160,134 @@ __device__ __forceinline__ bool piece_of(const SkParams &P, const SkCta &cw, int
     return pc.hi > pc.lo;
 }
 
+// Merge of one row of a cut unit's q-tile t from its n parts (slot `slot`):
+// O = sum_p 2^(lse_p - m) O_p / sum_p 2^(lse_p - m), m = max_p lse_p, where
+// O_p is part p's O / l and lse_p its log2-sum-exp (-inf: no visible key).
+// The parts were written by other CTAs of this grid: read through L2.
+template <int HD>
+__device__ __forceinline__ void merge_parts_row(const SkParams &P, int slot, int t, int row, int n, uint4 *dst)
+{
+    const AttnParams &p = P.a;
+    constexpr int64_t kStride = 2 * kBM;  // rows from one part to the next
+    const int64_t r0 = static_cast<int64_t>(slot) * P.max_parts * kStride + t * kBM + row;
+    float mx = -INFINITY;
+    for (int q = 0; q < n; ++q) mx = fmaxf(mx, __ldcg(p.part_lse + r0 + q * kStride));
+    float den = 0.f;
+    for (int q = 0; q < n; ++q) {
+        const float lse = __ldcg(p.part_lse + r0 + q * kStride);
+        if (lse != -INFINITY) den += ex2(lse - mx);
+    }
+    const float inv = den > 0.f ? 1.0f / den : 0.f;
+    constexpr int kCh = 64;  // columns per pass
+#pragma unroll 1
+    for (int c0 = 0; c0 < HD; c0 += kCh) {
+        float acc[kCh];
+#pragma unroll
+        for (int i = 0; i < kCh; ++i) acc[i] = 0.f;
+#pragma unroll 1
+        for (int q = 0; q < n; ++q) {
+            const float lse = __ldcg(p.part_lse + r0 + q * kStride);
+            if (lse == -INFINITY) continue;
+            const float w = ex2(lse - mx);
+            const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (r0 + q * kStride) * HD + c0);
+#pragma unroll
+            for (int i = 0; i < kCh / 4; ++i) {
+                const float4 v = __ldcg(src + i);
+                acc[4 * i + 0] += w * v.x;
+                acc[4 * i + 1] += w * v.y;
+                acc[4 * i + 2] += w * v.z;
+                acc[4 * i + 3] += w * v.w;
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < kCh / 8; ++i)
+            dst[c0 / 8 + i] = make_uint4(pack_bf16(acc[8 * i + 0] * inv, acc[8 * i + 1] * inv),
+                                         pack_bf16(acc[8 * i + 2] * inv, acc[8 * i + 3] * inv),
+                                         pack_bf16(acc[8 * i + 4] * inv, acc[8 * i + 5] * inv),
+                                         pack_bf16(acc[8 * i + 6] * inv, acc[8 * i + 7] * inv));
+    }
+}
+
+// The same merge by the warp whose part of the unit comes last (n <= 4 parts):
+// its own part is still in TMEM (unnormalised O at tO, with l and m_ref) and
+// is not written; the other parts are read through L2.  Own values are formed
+// exactly as a written part holds them (O * (1 / l), m_ref + log2 l) and the
+// parts are summed in index order, so the bits do not depend on which part's
+// warp merges.  has_tmem = false: this piece has no key for the q-tile (TMEM
+// is not read).  kOwn = false: every part, this warp's too, is read from L2
+// (own, tO, l and m_ref unused).  Whole warp.
+constexpr int kMaxOwnMergeParts = 4;
+template <int HD, bool kOwn>
+__device__ __forceinline__ void merge_own_row(const SkParams &P, int slot, int t, int row, int n, int own,
+                                              bool has_tmem, uint32_t tO, float l, float m_ref, bool valid,
+                                              uint4 *dst)
+{
+    if (!kOwn) own = -1;
+    const AttnParams &p = P.a;
+    constexpr int64_t kStride = 2 * kBM;
+    const int64_t r0 = static_cast<int64_t>(slot) * P.max_parts * kStride + t * kBM + row;
+    const float lse_own = (has_tmem && l > 0.f) ? m_ref + __log2f(l) : -INFINITY;
+    const float inv_own = l > 0.f ? 1.0f / l : 0.f;
+    float lse[kMaxOwnMergeParts];
+#pragma unroll
+    for (int q = 0; q < kMaxOwnMergeParts; ++q)
+        lse[q] = q == own ? lse_own : (valid && q < n) ? __ldcg(p.part_lse + r0 + q * kStride) : -INFINITY;
+    float mx = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < kMaxOwnMergeParts; ++q)
+        if (q < n) mx = fmaxf(mx, lse[q]);
+    float den = 0.f;
+#pragma unroll
+    for (int q = 0; q < kMaxOwnMergeParts; ++q)
+        if (q < n && lse[q] != -INFINITY) den += ex2(lse[q] - mx);
+    const float inv = den > 0.f ? 1.0f / den : 0.f;
+    constexpr int kCh = 64;  // columns per pass
+#pragma unroll 1
+    for (int c0 = 0; c0 < HD; c0 += kCh) {
+        float acc[kCh];
+#pragma unroll
+        for (int i = 0; i < kCh; ++i) acc[i] = 0.f;
+#pragma unroll
+        for (int q = 0; q < kMaxOwnMergeParts; ++q) {
+            if (q >= n) break;
+            if (kOwn && q == own) {  // warp-uniform: the TMEM loads are collective
+                if (has_tmem) {
+#pragma unroll
+                    for (int h = 0; h < kCh; h += 32) {
+                        float o[32];
+                        ptx::tmem_ld32(tO + c0 + h, o);
+                        ptx::tmem_wait_ld();
+                        if (lse[q] != -INFINITY) {
+                            const float w = ex2(lse[q] - mx);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) acc[h + i] += w * (o[i] * inv_own);
+                        }
+                    }
+                }
+            } else if (valid && lse[q] != -INFINITY) {
+                const float w = ex2(lse[q] - mx);
+                const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (r0 + q * kStride) * HD + c0);
+#pragma unroll
+                for (int i = 0; i < kCh / 4; ++i) {
+                    const float4 v = __ldcg(src + i);
+                    acc[4 * i + 0] += w * v.x;
+                    acc[4 * i + 1] += w * v.y;
+                    acc[4 * i + 2] += w * v.z;
+                    acc[4 * i + 3] += w * v.w;
+                }
+            }
+        }
+        if (valid) {
+#pragma unroll
+            for (int i = 0; i < kCh / 8; ++i)
+                dst[c0 / 8 + i] = make_uint4(pack_bf16(acc[8 * i + 0] * inv, acc[8 * i + 1] * inv),
+                                             pack_bf16(acc[8 * i + 2] * inv, acc[8 * i + 3] * inv),
+                                             pack_bf16(acc[8 * i + 4] * inv, acc[8 * i + 5] * inv),
+                                             pack_bf16(acc[8 * i + 6] * inv, acc[8 * i + 7] * inv));
+        }
+    }
+}
+
 template <int HD>
 __global__ void __launch_bounds__(kThreads, 1)
     replay_attn_sk_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -246,7 +376,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int k = 0; ok && piece_of(P, cw, k, pc, U); ++k) {
             const AttnSeq &sq = p.seqs[U.si];
             const bool two = 2 * U.pair + 1 < sq.n_qtiles;
-            // Q of this piece once the previous piece's GEMMs have read theirs
+            auto page_of = [&](int kt) -> int {  // this lane's page id of key tile kt (or -1)
+                const int lp = kt * ppt + lane;
+                return (lane < ppt && lp < sq.n_pages) ? p.page_table[sq.table_row + lp] : -1;
+            };
+            int page_next = page_of(pc.lo);  // read while the previous piece's last S GEMMs run
+            // Q of this piece once the previous piece's S GEMMs have read theirs
             if (q_issued > 0 && !wait_bar_warp(b_q_empty, (q_issued - 1) & 1, wctx)) { ok = false; break; }
             if (lane == 0) {
                 const int nq = two ? 2 : 1;
@@ -258,11 +393,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             __syncwarp();
             ++q_issued;
-            auto page_of = [&](int kt) -> int {  // this lane's page id of key tile kt (or -1)
-                const int lp = kt * ppt + lane;
-                return (lane < ppt && lp < sq.n_pages) ? p.page_table[sq.table_row + lp] : -1;
-            };
-            int page_next = page_of(pc.lo);
             for (int kt = pc.lo; kt < pc.hi; ++kt, ++gk) {
                 const int page = page_next;
                 if (kt + 1 < pc.hi) page_next = page_of(kt + 1);
@@ -344,9 +474,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 ptx::tc_fence_after();
+                const int n_s = max(n0, n1);  // key tiles with S GEMMs; Q is free after the last one
                 if (n0 > 0) issue_s(0, gk % C::kStages);
                 if (n1 > 0) issue_s(1, gk % C::kStages);
                 ptx::mma_commit(b_k_empty + 8 * (gk % C::kStages));
+                if (n_s <= 1) ptx::mma_commit(b_q_empty);
                 for (int j = 0; j < n_all; ++j) {
                     const int gj = gk + j;
                     const int s = gj % C::kStages;
@@ -370,10 +502,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         issue_pv(1, s, j > 0);
                     }
                     if (j + 1 < n1) issue_s(1, s1);
+                    if (j + 2 == n_s) ptx::mma_commit(b_q_empty);    // the piece's last S GEMMs read Q
                     if (more) ptx::mma_commit(b_k_empty + 8 * s1);  // K of tile j+1 consumed by its S GEMMs
                     ptx::mma_commit(b_v_empty + 8 * s);              // V of tile j consumed by its P V GEMMs
                 }
-                ptx::mma_commit(b_q_empty);  // every GEMM of this piece (and so its Q reads) is done
                 gk += n_all;
                 cnt0 += n0;
                 cnt1 += n1;
@@ -504,6 +636,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int64_t prow = pc.slot >= 0
                 ? (static_cast<int64_t>(pc.slot) * P.max_parts + pc.part) * (2 * kBM) + t * kBM + row
                 : 0;
+            uint4 *out_row = reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(p.out) +
+                                                       (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD);
+            // A part of a cut unit: per warp of 32 rows a ticket counts the parts written.  When
+            // every other part is in already, this warp merges them with its own part straight
+            // from TMEM; else it writes its part and counts it.
+            int *ticket = P.tickets + (max(pc.slot, 0) * 2 + t) * 4 + (warp & 3);
+            const int n_parts = pc.slot >= 0 ? P.slots[pc.slot].n_parts : 0;
+            int seen = 0;
+            if (pc.slot >= 0 && lane == 0) seen = *reinterpret_cast<volatile int *>(ticket);
+            const bool last = pc.slot >= 0 && n_parts <= kMaxOwnMergeParts &&
+                              __shfl_sync(0xffffffffu, seen, 0) == n_parts - 1;
+            if (last) __threadfence();  // the other parts' rows, written before their tickets
             if (G.ntiles > 0) {
                 // ---- epilogue: O / l, bf16 output or fp32 partial
                 if (!wait_bar_warp(b_o, (cnt + G.ntiles - 1) & 1, wctx)) { ok = false; break; }
@@ -527,6 +671,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                    pack_bf16(o[8 * q + 6] * inv, o[8 * q + 7] * inv));
                         }
                     }
+                } else if (last) {
+                    merge_own_row<HD, true>(P, pc.slot, t, row, n_parts, pc.part, true, tO, l, m_ref, valid,
+                                            out_row);
                 } else if (pc.slot >= 0) {
                     float *dst = p.part_o + prow * HD;
 #pragma unroll
@@ -547,8 +694,29 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // O_t has been read: the next piece's first P V GEMM may overwrite it
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(b_f);
+            } else if (last) {
+                merge_own_row<HD, true>(P, pc.slot, t, row, n_parts, pc.part, false, tO, 0.f, 0.f, valid, out_row);
             } else if (pc.slot >= 0 && valid) {
                 p.part_lse[prow] = -INFINITY;  // no key of this piece is visible to these rows
+            }
+            if (last) {
+                if (lane == 0) *ticket = 0;  // zero again for the next launch
+            } else if (pc.slot >= 0) {
+                // this warp's 32 rows of the part are written: count them; the warp that brings
+                // the count to the part count (another part finished meanwhile) merges from L2
+                __threadfence();
+                __syncwarp();
+                int arrived = 0;
+                if (lane == 0) arrived = atomicAdd(ticket, 1);
+                if (__shfl_sync(0xffffffffu, arrived, 0) == n_parts - 1) {
+                    __threadfence();
+                    if (n_parts <= kMaxOwnMergeParts)
+                        merge_own_row<HD, false>(P, pc.slot, t, row, n_parts, -1, false, tO, 0.f, 0.f, valid,
+                                                 out_row);
+                    else if (valid)
+                        merge_parts_row<HD>(P, pc.slot, t, row, n_parts, out_row);
+                    if (lane == 0) *ticket = 0;
+                }
             }
             cnt += G.ntiles;
         }
@@ -559,62 +727,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 9) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, C::kTmemCols);
-    }
-}
-
-// One warp per row of a cut unit's q-tile: LSE-weighted merge of the unit's parts.
-template <int HD>
-__global__ void __launch_bounds__(256) sk_combine_kernel(const __grid_constant__ SkParams P)
-{
-    ptx::griddep_launch_dependents();
-    ptx::griddep_wait();  // the attention grid's partials
-    const AttnParams &p = P.a;
-    const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (gw >= P.n_slots * 2 * kBM) return;
-    const int slot = gw / (2 * kBM);
-    const int t = (gw / kBM) & 1;
-    const int row = gw % kBM;
-    const UnitGeo U = unit_geo(p, P.slots[slot].unit);
-    const AttnSeq &sq = p.seqs[U.si];
-    const int g = p.group;
-    const int qt = 2 * U.pair + t;
-    if (qt >= sq.n_qtiles) return;
-    const int qi = qt * (kBM / g) + row / g;
-    if (qi >= sq.n_q) return;
-    const int n_parts = P.slots[slot].n_parts;
-    const int64_t base = static_cast<int64_t>(slot) * P.max_parts * (2 * kBM) + t * kBM + row;
-    constexpr int kPer = HD / 32;
-    // every part's LSE at once (one lane per part), then the weighted sum of their rows
-    float lse = -INFINITY;
-    if (lane < n_parts) lse = p.part_lse[base + static_cast<int64_t>(lane) * (2 * kBM)];
-    float mx = lse;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float acc[kPer];
-#pragma unroll
-    for (int q = 0; q < kPer; ++q) acc[q] = 0.f;
-    float den = 0.f;
-    if (mx != -INFINITY) {
-        for (int part = 0; part < n_parts; ++part) {
-            const float lp = __shfl_sync(0xffffffffu, lse, part & 31);
-            if (lp == -INFINITY) continue;
-            const float w = ex2(lp - mx);
-            den += w;
-            const float *src = p.part_o + (base + static_cast<int64_t>(part) * (2 * kBM)) * HD + lane * kPer;
-#pragma unroll
-            for (int q = 0; q < kPer; ++q) acc[q] += w * src[q];
-        }
-    }
-    const float inv = den > 0.f ? 1.0f / den : 0.f;
-    const int head = U.kvh * g + (row % g);
-    __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) +
-                         (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD + lane * kPer;
-    if constexpr (kPer == 4) {
-        *reinterpret_cast<uint2 *>(dst) =
-            make_uint2(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv));
-    } else {
-        *reinterpret_cast<uint32_t *>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
     }
 }
 
@@ -652,26 +764,6 @@ cudaError_t launch_replay_attn_sk(int head_dim, const CUtensorMap &tm_q, const C
     if (p.n_ctas > kMaxSkCtas) return cudaErrorInvalidValue;
     if (head_dim == 128) return launch_sk_t<128>(tm_q, tm_k, tm_v, p, st);
     if (head_dim == 64) return launch_sk_t<64>(tm_q, tm_k, tm_v, p, st);
-    return cudaErrorInvalidValue;
-}
-
-cudaError_t launch_sk_combine(int head_dim, const SkParams &p, cudaStream_t st)
-{
-    if (p.n_slots <= 0) return cudaSuccess;
-    if (p.max_parts > 32) return cudaErrorInvalidValue;  // one lane per part's LSE
-    const int warps = p.n_slots * 2 * kBM;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>((warps + 7) / 8));
-    cfg.blockDim = dim3(256);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (head_dim == 128) return cudaLaunchKernelEx(&cfg, sk_combine_kernel<128>, p);
-    if (head_dim == 64) return cudaLaunchKernelEx(&cfg, sk_combine_kernel<64>, p);
     return cudaErrorInvalidValue;
 }
 

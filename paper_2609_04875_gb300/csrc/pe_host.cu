@@ -44,6 +44,10 @@ pe_status cuda_fail(cudaError_t e, const char *what)
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// Merge counters in one zeroed device array: decode's per (sequence, kv-head)
+// of a launch, its scheduler's two, then the persistent attention's per slot.
+int64_t ticket_count(int32_t hkv) { return static_cast<int64_t>(kMaxSegs) * hkv + 2 + kMaxSkCtas * kSkTicketsPerSlot; }
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -116,7 +120,8 @@ struct pe_cache {
     int32_t *d_status = nullptr;
     float *d_ws = nullptr;
     int64_t ws_bytes = 0;
-    int32_t *d_tickets = nullptr;  // decode split merge: one counter per (sequence, kv-head) of a launch
+    int32_t *d_tickets = nullptr;  // merge counters: decode (per sequence and kv-head, then the scheduler's
+                                   // two), then the persistent attention's (per slot, q-tile and warp)
     int64_t pool_rows = 0;  // L * num_pages * Hkv * ps
     CUtensorMap tm_k{}, tm_v{};    // tensor-core kernel: 64 x ps boxes
     CUtensorMap tm_kd{}, tm_vd{};  // decode kernel: 64 x min(ps, 64) boxes
@@ -779,8 +784,9 @@ pe_status run_decode(pe_cache *c, const std::vector<AttnItem> &items, int32_t la
 // CTA c takes the work between boundaries c and c + 1 at c / P of the total.
 // With cuts allowed a boundary falls inside a unit (at a key tile, each piece
 // at least kSkMinPiece tiles), else at the unit boundary nearest to it; cuts
-// are kept when the cost model (the busiest CTA, plus the combine launch)
-// prefers them by 5 %, or always with "splitkv" = 1.
+// are kept when the cost model (the busiest CTA, plus the merge of the last
+// parts at the end of the kernel) prefers them by 5 %, or always with
+// "splitkv" = 1.
 constexpr double kSkUnitCost = 2.0;
 constexpr int kSkMinPiece = 2;
 
@@ -943,6 +949,7 @@ pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, si
         p.part_o = c->d_ws;
         p.part_lse = c->d_ws + static_cast<int64_t>(n_slots) * max_parts * 2 * kBM * d;
     }
+    P.tickets = c->d_tickets + kMaxSegs * hkv + 2;
     for (int32_t k = 0; k < pl.nc; ++k) {
         const SkBound &a = pl.b[k], &z = pl.b[k + 1];
         SkCta &w = P.cta[k];
@@ -1191,12 +1198,6 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             cudaError_t e = launch_replay_attn_sk(d, tm_q, c->tm_k, c->tm_v, P, st);
             if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
             c->launches++;
-            if (P.n_slots > 0) {
-                if (injected_failure(c)) return launch_fault("split-KV combine");
-                e = launch_sk_combine(d, P, st);
-                if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
-                c->launches++;
-            }
             continue;
         }
         if (tail && split) {  // the first launch runs unsplit: re-plan the group without splits
@@ -1353,8 +1354,9 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
         if ((e = cudaMalloc(&cc->d_status, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
         if ((e = cudaMemset(cc->d_status, 0, sizeof(int32_t))) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
         if ((e = cudaMalloc(&cc->d_ws, cc->ws_bytes)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc workspace"); break; }
-        // per-(sequence, kv-head) merge tickets, then the decode scheduler's chunk and done counters
-        const size_t tickets = sizeof(int32_t) * (kMaxSegs * c.num_kv_heads + 2);
+        // per-(sequence, kv-head) merge tickets, the decode scheduler's chunk and done counters, then
+        // the persistent attention's merge tickets
+        const size_t tickets = sizeof(int32_t) * ticket_count(c.num_kv_heads);
         if ((e = cudaMalloc(&cc->d_tickets, tickets)) != cudaSuccess) { st = cuda_fail(e, "cudaMalloc"); break; }
         if ((e = cudaMemset(cc->d_tickets, 0, tickets)) != cudaSuccess) { st = cuda_fail(e, "memset"); break; }
         if ((st = encode_2d(&cc->tm_k, cc->k_pool, c.head_dim, pool_rows, 64, ps)) != PE_OK) break;
@@ -1907,7 +1909,7 @@ pe_status pe_device_status(pe_cache *c, int32_t *code, int32_t clear, void *stre
     if (e == cudaSuccess && clear) e = cudaMemset(c->d_status, 0, sizeof(int32_t));
     // after a kernel gave up, its merge tickets and scheduler counters may be mid-count: reset them
     if (e == cudaSuccess && clear && *code != 0)
-        e = cudaMemset(c->d_tickets, 0, sizeof(int32_t) * (kMaxSegs * c->cfg.num_kv_heads + 2));
+        e = cudaMemset(c->d_tickets, 0, sizeof(int32_t) * ticket_count(c->cfg.num_kv_heads));
     if (e != cudaSuccess) return cuda_fail(e, "device status read");
     if (*code != 0) return fail(PE_ERR_DEVICE_TIMEOUT, "a kernel reported status %d", *code);
     return PE_OK;

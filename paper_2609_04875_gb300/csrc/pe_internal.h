@@ -106,8 +106,10 @@ struct AttnParams {
 // kernel runs one CTA per SM: whole units in lockstep rounds, then CTA c's
 // contiguous stretch of the remaining (unit, key tile) work; the pieces of
 // units cut by a stretch boundary write fp32 partials (O / l and log2-sum-exp)
-// into slot `slot`, part `part`, and a combine launch merges each slot's parts.
+// into slot `slot`, part `part`, and the warp that writes a slot's last part
+// (counted on its ticket) merges the slot's parts.
 constexpr int kMaxSkCtas = 160;        // >= SMs of the GPU
+constexpr int kSkTicketsPerSlot = 8;   // one per (q-tile, warp of 32 rows)
 
 struct SkCta {
     int32_t u0, t0;        // first unit and its first key tile
@@ -126,6 +128,7 @@ struct SkParams {
     int32_t n_ctas, n_slots, max_parts;
     int32_t rounds;        // whole units first: in round r < rounds CTA k takes unit r n_ctas + k (odd r:
                            // r n_ctas + n_ctas - 1 - k); then its tail stretch (cta[k], u0 > u1: none)
+    int32_t *tickets;      // [n_slots][2][4] parts written per (slot, q-tile, warp); zero between launches
     SkCta cta[kMaxSkCtas];
     SkSlot slots[kMaxSkCtas];
 };
@@ -192,10 +195,9 @@ cudaError_t launch_cow_copy(uint4 *k_pool, uint4 *v_pool, int32_t src, int32_t d
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
                                const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);
-// Persistent stream-K attention (p.n_ctas CTAs) and the merge of its cut units (p.n_slots > 0).
+// Persistent stream-K attention (p.n_ctas CTAs), cut units merged in the kernel.
 cudaError_t launch_replay_attn_sk(int head_dim, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
                                   const CUtensorMap &tm_v, const SkParams &p, cudaStream_t st);
-cudaError_t launch_sk_combine(int head_dim, const SkParams &p, cudaStream_t st);
 // rows_cap: 4, 8 or 16 (every sequence's n_q x group fits).
 // tm_k / tm_v: the pools as 2-D maps {d, L*num_pages*Hkv*ps} with 64 x min(ps, 64) boxes, 128-byte swizzle.
 // tensor_core (d = 128 only): keys on the MMA's M side, 128-key tiles (split_tiles

@@ -2,8 +2,9 @@
 it; by default it serves the launch groups whose one-item plan would leave
 SMs idle): one CTA per SM, whole (sequence, kv-head, q-tile pair) units in
 lockstep rounds, then balanced stretches of the remaining (unit, key tile)
-work.  Units cut between CTAs are computed in pieces whose fp32 partials a
-combine launch merges.
+work.  Units cut between CTAs are computed in pieces that write fp32
+partials; the warp that finishes a unit's last part merges them in the kernel
+(its own part straight from TMEM when the others are in already).
 
 Checked against the oracle with forced CTA counts that cut units into up to
 tens of parts (pieces where one q-tile of the pair has no key tile, odd q-tile
@@ -107,3 +108,24 @@ def test_whole_units_bitwise_equal_one_item_kernel(d, hq, hkv, ps, P, S):
     torch.cuda.synchronize()
     assert torch.equal(a, b)
     assert_close(a, oracle.replay_attention(pair.orc, s, 0, q, 1 / math.sqrt(d)), "whole units")
+
+
+@pytest.mark.parametrize("ctas", [152, 40, 7])
+def test_cut_unit_merge_is_deterministic(ctas):
+    """Whichever warp finishes a cut unit's last part merges the parts: from
+    TMEM and L2 when the other parts are in before its epilogue, else all from
+    L2 (or the many-part path).  Every path forms the same values in the same
+    order, so repeated launches, whose timing differs, agree bit for bit."""
+    d, hq, hkv, ps, P, S = 128, 32, 8, 16, 3000, 700
+    pair, s, q = _one(d, hq, hkv, ps, P, S, seed=31)
+    pair.gpu.set_option("attn_ctas", ctas)
+    pair.gpu.set_option("splitkv", 1)
+    Q = dev(q)
+    outs = [pair.gpu.replay_attn(s, 0, Q) for _ in range(8)]
+    torch.cuda.synchronize()
+    split, parts, n_ctas = pair.gpu.last_attn_plan()
+    assert split == 1 and parts >= 2, (split, parts, n_ctas)
+    for o in outs[1:]:
+        assert torch.equal(o, outs[0])
+    assert_close(outs[0], oracle.replay_attention(pair.orc, s, 0, q, 1 / math.sqrt(d)), f"ctas={ctas}")
+    assert pair.gpu.device_status() == 0
