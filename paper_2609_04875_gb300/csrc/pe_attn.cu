@@ -12,16 +12,22 @@
 // Roles (320 threads):
 //   warps 0-3, 4-7  softmax of q-tile 0 / q-tile 1: thread r owns row r
 //                   (TMEM lane r); masks, online softmax in fp32 (exp2),
-//                   writes P (bf16) back into TMEM over its S columns,
-//                   rescales O in TMEM when needed, epilogue.
+//                   writes P (bf16) back into TMEM (d = 128: over its S
+//                   columns; d = 64: into its own P columns), rescales O in
+//                   TMEM when needed, epilogue.
 //   warp 8          producer: reads the page table; its lanes issue one TMA
 //                   box per (page, 64-column half) into K and V stage rings.
 //   warp 9          MMA: allocates TMEM; one thread issues tcgen05.mma for
 //                   S_t = Q_t K^T (A, B from shared memory) and
 //                   O_t += P_t V (A = P from TMEM, B = V from shared memory).
-// Tensor-core order per key tile j:  PV_0(j), S_0(j+1), PV_1(j), S_1(j+1), so
-// one softmax group works while the tensor core runs the other group's GEMMs.
+// Tensor-core order per key tile j (d = 128):  PV_0(j), S_0(j+1), PV_1(j),
+// S_1(j+1), so one softmax group works while the tensor core runs the other
+// group's GEMMs; S_t(j+1) waits for PV_t(j), which reads P_t(j) over S_t.
 // TMEM columns: S_0 [0,128), S_1 [128,256), O_0 and O_1 (HD each) from 256.
+// At d = 64 the last 128 columns hold P_0 and P_1, so S_t(j+1) is issued as
+// soon as the softmax has copied S_t(j) into registers (barrier s_free) and
+// runs during the softmax of tile j; the softmax writes P_t(j) once
+// PV_t(j-1) has read P_t(j-1).  Same arithmetic, so the same bits.
 //
 // Key tiles always start at logical key 0 (multiples of 128 keys), whatever
 // the physical pages, so a row's arithmetic depends only on its own keys.
@@ -59,8 +65,12 @@ struct AttnCfg {
     static constexpr int kOffK = kOffQ + 2 * kTileBytes;
     static constexpr int kOffV = kOffK + kStages * kTileBytes;
     static constexpr int kOffBar = kOffV + kStages * kTileBytes;
-    // barriers: q_full, k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_full[2], o_done[2]
-    static constexpr int kNumBars = 1 + 4 * kStages + 6;
+    // barriers: q_full, k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_full[2], o_done[2],
+    // s_free[2]
+    static constexpr int kNumBars = 1 + 4 * kStages + 8;
+    // TMEM columns: S_0, S_1 (128 each), O_0, O_1 (HD each); for d = 64 the 128 left over hold P_0 and
+    // P_1 (64 each), so S(j+1) need not wait for the P V GEMM of tile j (P(j) lives apart from S)
+    static constexpr bool kSepP = HD == 64;
     static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem slot, abort flag
     static constexpr int kSmemBytes = kOffMisc + 16;
     static constexpr int kDynSmem = kSmemBytes + 1024;       // alignment slack
@@ -144,6 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t b_s_full = b_v_empty + 8 * C::kStages;  // [2]
     const uint32_t b_p_full = b_s_full + 16;               // [2]
     const uint32_t b_o_done = b_p_full + 16;               // [2]
+    const uint32_t b_s_free = b_o_done + 16;               // [2] (d = 64) S_t has been read into registers
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 4);
     const WaitCtx wctx{abort_flag, p.status};
@@ -196,6 +207,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ptx::mbar_init(b_s_full + 8 * t, 1);
                 ptx::mbar_init(b_p_full + 8 * t, 128);
                 ptx::mbar_init(b_o_done + 8 * t, 1);
+                ptx::mbar_init(b_s_free + 8 * t, 128);
             }
             *abort_flag = 0;
             ptx::fence_barrier_init();
@@ -270,9 +282,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             };
             auto issue_pv = [&](int t, int s, bool acc) {
                 const uint32_t vb = v_smem0 + s * C::kTileBytes;
+                const uint32_t tp = C::kSepP ? tmem + 256 + 2 * HD + 64 * t : tmem + 128 * t;  // P_t
 #pragma unroll
                 for (int kk = 0; kk < kBN / 16; ++kk)
-                    mma_bf16_ts(tmem + 256 + HD * t, tmem + 128 * t + kk * 8,
+                    mma_bf16_ts(tmem + 256 + HD * t, tp + kk * 8,
                                 ptx::smem_desc_sw128(vb + kk * 16 * 128, C::kRegionBytes, 1024), kIdescPV,
                                 (acc || kk > 0) ? 1u : 0u);
                 ptx::mma_commit(b_o_done + 8 * t);
@@ -284,7 +297,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (n1 > 0) issue_s(1, 0);
                 if (n0 > 0 || n1 > 0) ptx::mma_commit(b_k_empty);
             }
-            for (int j = 0; ok && j < n_all; ++j) {
+            for (int j = 0; ok && C::kSepP && j < n_all; ++j) {
+                // d = 64: S_t(j+1) once the softmax holds S_t(j) in registers, P V_t(j) once P_t(j) is in
+                const int s = j % C::kStages;
+                const int s1 = (j + 1) % C::kStages;
+                const bool more = j + 1 < n_all;
+                if (more && !wait_bar(b_k_full + 8 * s1, ((j + 1) / C::kStages) & 1, wctx)) { ok = false; break; }
+#pragma unroll
+                for (int t = 0; t < 2; ++t) {
+                    if (j + 1 >= (t ? n1 : n0)) continue;
+                    if (!wait_bar(b_s_free + 8 * t, j & 1, wctx)) { ok = false; break; }
+                    ptx::tc_fence_after();
+                    issue_s(t, s1);
+                }
+                if (!ok) break;
+                if (more) ptx::mma_commit(b_k_empty + 8 * s1);  // K of tile j+1 consumed by its S GEMMs
+                if (!wait_bar(b_v_full + 8 * s, (j / C::kStages) & 1, wctx)) { ok = false; break; }
+#pragma unroll
+                for (int t = 0; t < 2; ++t) {
+                    if (j >= (t ? n1 : n0)) continue;
+                    if (!wait_bar(b_p_full + 8 * t, j & 1, wctx)) { ok = false; break; }
+                    ptx::tc_fence_after();
+                    issue_pv(t, s, j > 0);
+                }
+                if (!ok) break;
+                ptx::mma_commit(b_v_empty + 8 * s);              // V of tile j consumed by its PV GEMMs
+            }
+            for (int j = 0; ok && !C::kSepP && j < n_all; ++j) {
                 const int s = j % C::kStages;
                 const int s1 = (j + 1) % C::kStages;
                 const bool more = j + 1 < n_all;
@@ -321,6 +360,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t tS = tmem + 128 * t + lane_off;
         const uint32_t tO = tmem + 256 + HD * t + lane_off;
         const uint32_t b_s = b_s_full + 8 * t, b_p = b_p_full + 8 * t, b_o = b_o_done + 8 * t;
+        const uint32_t tP = C::kSepP ? tmem + 256 + 2 * HD + 64 * t + lane_off : tS;  // P_t (over S_t for d = 128)
         const float sl2 = p.scale_log2;
         const float2 sl2x2 = make_float2(sl2, sl2);
         float m_ref = -INFINITY;
@@ -341,6 +381,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ptx::tmem_ld32(tS + 64, s2);
                 ptx::tmem_ld32(tS + 96, s3);
                 ptx::tmem_wait_ld();
+            }
+            if (C::kSepP) {
+                // S_t(j) is in registers: the next tile's S GEMM may overwrite it
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(b_s_free + 8 * t);
             }
             if (kbase + kBN - 1 > G.pos_first) {  // tile crosses the causal diagonal of some row
 #pragma unroll
@@ -366,7 +411,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                         acc[k & 3] = add2(acc[k & 3], e);
                         pk[k] = pack_bf16(e.x, e.y);
                     }
-                    tmem_st16(tS + ch * 16, pk);
+                    if (C::kSepP && ch == 0 && j > 0) {
+                        // P_t(j) goes to P_t's own columns once P V_t(j-1) has read P_t(j-1)
+                        if (!wait_bar_warp(b_o, (j - 1) & 1, wctx)) ok = false;
+                        ptx::tc_fence_after();
+                    }
+                    tmem_st16(tP + ch * 16, pk);
                 }
                 const float2 a = add2(add2(acc[0], acc[1]), add2(acc[2], acc[3]));
                 return a.x + a.y;
@@ -375,6 +425,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool need = j == 0;
             if (j > 0) {
                 rs = exp_tile(m_ref);
+                if (!ok) break;
                 need = !(rs <= kTileSumLimit);
             }
             if (__any_sync(0xffffffffu, need)) {
@@ -410,6 +461,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 ptx::tmem_wait_st();
                 rs = exp_tile(m_ref);
+                if (!ok) break;
             }
             l += rs;
             ptx::tmem_wait_st();

@@ -1015,6 +1015,9 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
 
     // split-KV decision over the whole launch group; plan_est: the cost model's time of the plan
     double plan_est = 0.0;
+    // time of one key tile per CTA in the cost models: about 1.5 us, compute- or HBM-bound alike; 1 us at
+    // d = 64, whose next S GEMM overlaps the softmax
+    const double tile_s = d == 64 ? 1.0e-6 : 1.5e-6;
     // splitkv: the "splitkv" option's value for this plan (-1 auto, 0 never, 1 always)
     auto plan_group = [&](size_t lo, size_t hi, AttnParams &p, bool &split, int splitkv) -> pe_status {
         // C CTAs (pairs of q-tiles x kv-heads), W key tiles per CTA on average.
@@ -1033,16 +1036,17 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             max_tiles = std::max(max_tiles, ceil_div(len, kBN));
         }
         // Estimated time with s key splits: the CTAs run in ceil(C s / N) waves of
-        // (W/s + 2) tile times (about 1.5 us per tile, compute- or HBM-bound
-        // alike), and never faster than the longest CTA (max_tiles/s + 2);
-        // splits add their fp32 partials' HBM round trip and a combine launch.
+        // (W/s + 2) tile times, and never faster than the longest CTA
+        // (max_tiles/s + 2); splits add their fp32 partials' HBM round trip and
+        // a combine launch.
         const double W = C > 0 ? static_cast<double>(tiles) / C : 0.0;
         const int64_t row_bytes = static_cast<int64_t>(d) * 4 + 4;
-        // (the combine kernel is a programmatic dependent of the attention grid: about 3 us more)
+        // (the combine kernel is a programmatic dependent of the attention grid: about 5 us more, measured
+        // on the 1-agent d = 64 launch: 5 splits + combine 14.0 us, one pass 13.0 us)
         auto cost = [&](int64_t sp) {
             const double waves = std::ceil(static_cast<double>(C * sp) / c->num_sms);
-            double t = std::max(waves * (W / sp + 2.0), static_cast<double>(max_tiles) / sp + 2.0) * 1.5e-6;
-            if (sp > 1) t += static_cast<double>(valid_rows * sp * row_bytes * 2) / 6.0e12 + 3e-6;
+            double t = std::max(waves * (W / sp + 2.0), static_cast<double>(max_tiles) / sp + 2.0) * tile_s;
+            if (sp > 1) t += static_cast<double>(valid_rows * sp * row_bytes * 2) / 6.0e12 + 5e-6;
             return t;
         };
         int64_t best = 1;
@@ -1146,12 +1150,12 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         wb /= static_cast<double>(cut);
         const int64_t qt_b = std::min<int64_t>(nqt, 2 * cut);
         const int64_t row_bytes = static_cast<int64_t>(d) * 4 + 4;
-        const double t_a = std::ceil(static_cast<double>(C - cut * hkv) / N) * (wa + 2.0) * 1.5e-6;
+        const double t_a = std::ceil(static_cast<double>(C - cut * hkv) / N) * (wa + 2.0) * tile_s;
         double best_t = 1e30;
         for (int64_t sp = 2; sp <= std::min<int64_t>(128, std::max<int64_t>(2, ktiles / 4)); ++sp) {
             if (qt_b * hkv * sp * kBM * row_bytes > c->ws_bytes) break;
             const double waves = std::ceil(static_cast<double>(cut * hkv * sp) / N);
-            const double t = t_a + waves * (wb / sp + 2.0) * 1.5e-6 +
+            const double t = t_a + waves * (wb / sp + 2.0) * tile_s +
                              static_cast<double>(qt_b * hkv * kBM * sp * row_bytes * 2) / 6.0e12 + 10e-6;
             if (t < best_t) {
                 best_t = t;
