@@ -308,17 +308,18 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "tiny": {"bytes": 1.518592e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
-             "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100"}},
-    "agent_batch": {"bytes": 695.139072e6 + 327.651328e6, "profile": "profiles/replay_attn_agent_batch.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100"}},
-    "short_suffix": {"bytes": 1.077033216e9 + 6.493184e6, "profile": "profiles/replay_attn_sk_short_suffix.md",
-                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f3856241b4b16f861c6be6b07d1731e7f4f0f11fd357d69f392aef397889e2ee"}},
-    "long_suffix": {"bytes": 4.61800832e9 + 1.176607232e9, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100"}},
-    # mean over the 160 attention launches of one sweep step (5 forget requests x 32 layers)
-    "tau_sweep": {"bytes": 198.352832e6 + 41.8683744e6, "profile": "profiles/traffic_attention_configs.md",
-                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "e59de9879c8bb9d3729810501c170ec0f7ef4d0980ca20c42b09e43b123b2100", "prefill_sk": "f3856241b4b16f861c6be6b07d1731e7f4f0f11fd357d69f392aef397889e2ee"}},
+    "tiny": {"bytes": 1.499136e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
+             "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d"}},
+    "agent_batch": {"bytes": 695.387648e6 + 327.606784e6, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d"}},
+    "short_suffix": {"bytes": 1.078952192e9 + 5.8368e6, "profile": "profiles/traffic_attention_configs.md",
+                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
+    "long_suffix": {"bytes": 4.624238592e9 + 1.177223168e9, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d"}},
+    # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
+    # tail launch runs), per layer: bytes / 160
+    "tau_sweep": {"bytes": (47299.836416e6 + 9032.658944e6) / 160, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d", "prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
     "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
                      "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},
