@@ -506,7 +506,8 @@ def unit_report(u, t, gated, peaks, peak_src, steps):
         "units_per_launch": {"agents": len(u.w.agents), "suffix_tokens": u.S,
                              "keys": sum(a.T for a in u.w.agents)},
         "roofline_ms_per_launch": kern["roofline_s"] * 1e3,
-        "kernel_frac": kern["frac"], "kernel_bound": kern["bound"],
+        "kernel_frac": kern["frac"], "kernel_frac_of_sustained": kern.get("frac_of_sustained"),
+        "kernel_bound": kern["bound"],
         "kernel_achieved": kern["achieved"], "kernel_unit": kern["unit"],
         # the step fraction: roofline time of append + attention over their measured device time
         "step_frac": step["frac"], "step_bound": step["bound"], "step_roofline_ms": step["roofline_s"] * 1e3,
