@@ -56,16 +56,18 @@ def test_peaked_logits_exercise_rescaling(scale_mult):
     assert_within_rounding_bound(outs[0], refs[0], vmax, f"peaked x{scale_mult}")
 
 
+@pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("split", [0, 1])
 @pytest.mark.parametrize("jump", [128, 192])
-def test_reference_moves_on_large_jump(split, jump):
+def test_reference_moves_on_large_jump(split, jump, d):
     """Keys from `jump` on are scaled by 16 (exact in bf16), so for nearly
     every row a later tile's logits exceed the first tile's max by far more
     than 64 in log2 units: the row's reference must move and O be rescaled.
     At 128 the jump starts a key tile; at 192 it falls in the middle of one,
     so that tile mixes weights near the old reference with weights far above
-    it."""
-    d, hq, hkv, ps, P, S = 128, 32, 8, 16, 600, 100
+    it.  At d = 64 P has its own TMEM columns and the next tile's S GEMM runs
+    during the softmax: the rescale must still see this tile's S intact."""
+    hq, hkv, ps, P, S = 32, 8, 16, 600, 100
     T = P + S
     npg = -(-T // ps) + 3
     pair = Pair(1, hkv, d, ps, npg, 1, npg, seed=61)
