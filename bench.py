@@ -310,12 +310,12 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 NCU_TRAFFIC = {
     "tiny": {"bytes": 1.499136e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
              "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d"}},
-    "agent_batch": {"bytes": 695.387648e6 + 327.606784e6, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d"}},
+    "agent_batch": {"bytes": 684.605e6 + 317.062e6, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
     "short_suffix": {"bytes": 1.078952192e9 + 5.8368e6, "profile": "profiles/traffic_attention_configs.md",
                      "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
-    "long_suffix": {"bytes": 4.624238592e9 + 1.177223168e9, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d"}},
+    "long_suffix": {"bytes": 1.41242e9 + 1.03806e9, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
     # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
     # tail launch runs), per layer: bytes / 160
     "tau_sweep": {"bytes": (47299.836416e6 + 9032.658944e6) / 160, "profile": "profiles/traffic_attention_configs.md",

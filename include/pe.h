@@ -262,7 +262,11 @@ pe_status pe_cache_pools(const pe_cache *cache, void **k_pool, void **v_pool);
  * a tail launch and whose q-tile pairs x Hkv number between a quarter of the
  * SMs and two waves, the one-item kernel otherwise; 2: always persistent; 0:
  * always one-item; "attn_ctas" = 0 (auto) or the persistent kernel's CTA
- * count; "fail_launch_after" = k >= 0
+ * count; "attn_order" = -1 (auto) / 0 / 1: how the one-item kernel numbers a
+ * sequence's CTAs -- 0: kv-heads fastest, every head's heaviest q-tile pairs
+ * first; 1: pairs fastest, so the CTAs resident at once share one or two
+ * kv-heads' keys in L2; auto takes 1 for launches of at least 32 CTAs per SM;
+ * "fail_launch_after" = k >= 0
  * (test hook): the device step after the next k fails with PE_ERR_CUDA
  * without being launched, once (-1 = off); on a host-only cache the steps a
  * device cache would launch are counted the same way.  Split

@@ -101,7 +101,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
 
-    // ---- work item -> (sequence, kv-head, split, q-tile pair); heaviest pairs first
+    // ---- work item -> (sequence, kv-head, split, q-tile pair); heaviest pairs first.  Within a
+    // sequence the kv-heads run fastest (every head's heaviest pairs first), or, when p.pairs_fastest
+    // is set (launches of many waves), the pairs: then the CTAs resident at once work on one or two
+    // kv-heads' keys, which stay in L2 while Q and O stream through.
     const int item = blockIdx.x;
     int si = 0, si_hi = p.n_seqs;  // the last sequence whose first item is at most `item` (binary search)
     while (si_hi - si > 1) {
@@ -111,11 +114,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     const AttnSeq &sq = p.seqs[si];
     int local = item - sq.item0;
-    const int kvh = local % p.hkv;
-    local /= p.hkv;
-    const int split = local % sq.n_splits;
-    local /= sq.n_splits;
-    const int pair = sq.pair_top - 1 - local;
+    int kvh, split, pair;
+    if (p.pairs_fastest) {
+        const int seq_items = (si + 1 < p.n_seqs ? p.seqs[si + 1].item0 : p.total_items) - sq.item0;
+        const int n_pairs = seq_items / (p.hkv * sq.n_splits);  // pairs of this sequence in the launch
+        pair = sq.pair_top - 1 - local % n_pairs;
+        local /= n_pairs;
+        split = local % sq.n_splits;
+        kvh = local / sq.n_splits;
+    } else {
+        kvh = local % p.hkv;
+        local /= p.hkv;
+        split = local % sq.n_splits;
+        pair = sq.pair_top - 1 - local / sq.n_splits;
+    }
     const int g = p.group;
     const int bmq = kBM / g;
     const int kt0 = SPLIT ? split * p.split_tiles : 0;

@@ -95,6 +95,7 @@ struct AttnParams {
     int32_t split_tiles;   // key tiles per split
     int32_t total_items;
     int32_t total_comb;
+    int32_t pairs_fastest;  // one-item kernel: number a sequence's items pairs fastest (else kv-heads fastest)
     float scale_log2;      // softmax_scale * log2(e)
     AttnSeq seqs[kMaxSegs];
 };

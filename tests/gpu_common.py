@@ -99,14 +99,17 @@ class Pair:
             assert self.gpu.device_page_table(s, len(tbl)) == tbl
 
 
-def replay_case(L, hq, hkv, d, ps, P, S, seed, scale=None, std=1.0, split=None, slack_pages=3):
+def replay_case(L, hq, hkv, d, ps, P, S, seed, scale=None, std=1.0, split=None, slack_pages=3, options=None):
     """Original session of T = P + S tokens, crop to tau = P + 1, append the
-    counterfactual suffix, replay; returns (pair, seq, gpu out [L][S][Hq][d], oracle fp64)."""
+    counterfactual suffix, replay; returns (pair, seq, gpu out [L][S][Hq][d], oracle fp64).
+    `options`: further cache options (pe_set_option) set before the replay."""
     T = P + S
     npg = -(-T // ps) + slack_pages
     pair = Pair(L, hkv, d, ps, npg, 2, npg, seed=seed)
     if split is not None:
         pair.gpu.set_option("splitkv", split)
+    for key, value in (options or {}).items():
+        pair.gpu.set_option(key, value)
     g = synth.rng(seed, 11)
     k0 = synth.normal_bf16(g, (L, T, hkv, d), std)
     v0 = synth.normal_bf16(g, (L, T, hkv, d), std)

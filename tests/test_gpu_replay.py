@@ -119,13 +119,17 @@ def _view_device(ptr, n):
     return torch.as_tensor(_Arr(), device="cuda").view(torch.bfloat16)
 
 
+@pytest.mark.parametrize("order", [-1, 1])
 @pytest.mark.parametrize("split", [0, 1])
-def test_splitkv_forced(split):
-    """The split-KV kernel + LSE combine and the single-pass kernel, forced."""
-    for case in [(128, 32, 8, 16, 4000, 16), (64, 8, 2, 64, 1500, 70), (128, 8, 8, 16, 130, 3)]:
+def test_splitkv_forced(split, order):
+    """The split-KV kernel + LSE combine and the single-pass kernel, forced;
+    CTAs numbered in the default order and pairs fastest ("attn_order" = 1)."""
+    for case in [(128, 32, 8, 16, 4000, 16), (64, 8, 2, 64, 1500, 70), (128, 8, 8, 16, 130, 3),
+                 (128, 32, 8, 16, 900, 700)]:
         d, hq, hkv, ps, P, S = case
-        pair, s, outs, refs, _ = replay_case(1, hq, hkv, d, ps, P, S, seed=17, split=split)
-        assert_close(outs[0], refs[0], f"split={split} {case}")
+        pair, s, outs, refs, _ = replay_case(1, hq, hkv, d, ps, P, S, seed=17, split=split,
+                                             options={"attn_order": order, "attn_kernel": 0})
+        assert_close(outs[0], refs[0], f"split={split} order={order} {case}")
 
 
 def test_splitkv_many_splits():

@@ -178,6 +178,11 @@ def test_error_codes():
     with pytest.raises(binding.PEError) as e:
         c.set_option("nonsense", 1)
     assert e.value.kind == "invalid"
+    for key, good, bad in (("attn_order", 1, 2), ("attn_kernel", 2, 3), ("splitkv", -1, 2)):
+        c.set_option(key, good)
+        with pytest.raises(binding.PEError) as e:
+            c.set_option(key, bad)
+        assert e.value.kind == "invalid", key
     with pytest.raises(binding.PEError) as e:
         pe.PagedKVCache(1, 1, 64, 16, 4, 2, 4, init_free_order=[0, 1, 1, 2], host_only=True)
     assert e.value.kind == "invalid"
