@@ -308,8 +308,8 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "tiny": {"bytes": 1.499136e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
-             "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d"}},
+    "tiny": {"bytes": 1.500672e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
+             "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
     "agent_batch": {"bytes": 684.605e6 + 317.062e6, "profile": "profiles/traffic_attention_configs.md",
                     "kernels": ["prefill"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
     "short_suffix": {"bytes": 1.078952192e9 + 5.8368e6, "profile": "profiles/traffic_attention_configs.md",
@@ -318,8 +318,8 @@ NCU_TRAFFIC = {
                     "kernels": ["prefill"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
     # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
     # tail launch runs), per layer: bytes / 160
-    "tau_sweep": {"bytes": (47299.836416e6 + 9032.658944e6) / 160, "profile": "profiles/traffic_attention_configs.md",
-                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "f67f533ae7f9e74bcde88ce37fae2d86c7e5ae753bf72072d22a0edcebde416d", "prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
+    "tau_sweep": {"bytes": (47494.0e6 + 9046.57e6) / 160, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad", "prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
     "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
                      "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},
