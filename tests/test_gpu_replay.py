@@ -323,3 +323,36 @@ def test_gpu_error_paths_leave_state_unchanged():
         c.replay_attn(s, 0, qm)
     assert e.value.kind == "invalid"
     assert c.device_status() == 0
+
+
+@pytest.mark.parametrize("order", [0, 1])
+@pytest.mark.parametrize("split", [0, 1])
+def test_batch_item_orders(order, split):
+    """A launch of six sequences of mixed lengths (one-item kernel), with and
+    without key splits, its CTAs numbered kv-heads fastest or pairs fastest:
+    every sequence's rows against the oracle."""
+    d, hq, hkv, ps = 128, 32, 8, 16
+    g = synth.rng(71, 5)
+    lens = [int(x) for x in g.integers(200, 2500, size=6)]
+    nq = [int(x) for x in g.integers(1, 300, size=6)]
+    npg = sum(-(-n // ps) for n in lens) + 8
+    pair = Pair(1, hkv, d, ps, npg, 6, 200, seed=71)
+    pair.gpu.set_option("attn_kernel", 0)
+    pair.gpu.set_option("attn_order", order)
+    pair.gpu.set_option("splitkv", split)
+    seqs = []
+    for n in lens:
+        s = pair.seq()
+        pair.append(s, synth.normal_bf16(g, (1, n, hkv, d)), synth.normal_bf16(g, (1, n, hkv, d)))
+        seqs.append(s)
+    cu = [0]
+    for k in nq:
+        cu.append(cu[-1] + k)
+    q = synth.normal_bf16(g, (cu[-1], hq, d))
+    scale = 1 / math.sqrt(d)
+    out = pair.gpu.replay_attn_batch(seqs, 0, dev(q), cu, softmax_scale=scale)
+    torch.cuda.synchronize()
+    for i, s in enumerate(seqs):
+        ref = oracle.replay_attention(pair.orc, s, 0, q[cu[i]:cu[i + 1]], scale)
+        assert_close(out[cu[i]:cu[i + 1]], ref, f"order={order} split={split} seq {i}")
+    assert pair.gpu.device_status() == 0
