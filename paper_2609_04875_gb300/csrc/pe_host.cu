@@ -906,8 +906,10 @@ pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, si
         cuts_in.clear();
         n_slots = 0;
         max_parts = 1;
-        for (const SkBound &x : bb) {
-            if (x.t <= 0 || x.u >= U) continue;
+        for (size_t i = 0; i < bb.size(); ++i) {
+            const SkBound &x = bb[i];
+            // an empty stretch repeats its boundary: count each cut once
+            if (x.t <= 0 || x.u >= U || (i > 0 && bb[i - 1] == x)) continue;
             if (slot_of[x.u] < 0) {
                 slot_of[x.u] = n_slots++;
                 cuts_in.push_back(0);
@@ -968,9 +970,11 @@ pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, si
         w.t1 = z.t;
         if (cuts && slot_of[a.u] >= 0) {
             w.slot0 = slot_of[a.u];
-            int32_t part = 0;  // interior boundaries of unit a.u at or before tile a.t
-            for (const SkBound &x : pl.b)
-                if (x.u == a.u && x.t > 0 && x.t <= a.t) ++part;
+            int32_t part = 0;  // interior boundaries of unit a.u at or before tile a.t, each counted once
+            for (size_t i = 0; i < pl.b.size(); ++i) {
+                const SkBound &x = pl.b[i];
+                if (x.u == a.u && x.t > 0 && x.t <= a.t && !(i > 0 && pl.b[i - 1] == x)) ++part;
+            }
             w.part0 = part;
         }
         if (cuts && z.u != a.u && z.t > 0) {

@@ -129,3 +129,38 @@ def test_cut_unit_merge_is_deterministic(ctas):
         assert torch.equal(o, outs[0])
     assert_close(outs[0], oracle.replay_attention(pair.orc, s, 0, q, 1 / math.sqrt(d)), f"ctas={ctas}")
     assert pair.gpu.device_status() == 0
+
+
+def test_plan_with_empty_stretches():
+    """Whole-unit rounds can leave a CTA at or above the mean load, so its tail
+    stretch is empty and its two boundaries coincide inside a cut unit (this
+    batch on 9 CTAs: twice, at key tile 4 of the last unit).  Each cut is
+    counted once, so the unit's part count, and the count its merge waits
+    for, stay right."""
+    d, hq, hkv, ps = 128, 32, 8, 16
+    lens = [3216, 684, 1623, 1045, 743]
+    nq = [337, 85, 233, 411, 475]
+    g = synth.rng(9, 63)
+    npg = sum(-(-n // ps) for n in lens) + 8
+    pair = Pair(1, hkv, d, ps, npg, 5, 256, seed=9)
+    pair.gpu.set_option("attn_kernel", 2)
+    pair.gpu.set_option("attn_ctas", 9)
+    pair.gpu.set_option("splitkv", 1)
+    seqs = []
+    for n in lens:
+        s = pair.seq()
+        pair.append(s, synth.normal_bf16(g, (1, n, hkv, d)), synth.normal_bf16(g, (1, n, hkv, d)))
+        seqs.append(s)
+    cu = [0]
+    for k in nq:
+        cu.append(cu[-1] + k)
+    q = synth.normal_bf16(g, (cu[-1], hq, d))
+    scale = 1 / math.sqrt(d)
+    out = pair.gpu.replay_attn_batch(seqs, 0, dev(q), cu, softmax_scale=scale)
+    torch.cuda.synchronize()
+    split, parts, n_ctas = pair.gpu.last_attn_plan()
+    assert split == 1 and n_ctas == 9, (split, parts, n_ctas)
+    for i, s in enumerate(seqs):
+        ref = oracle.replay_attention(pair.orc, s, 0, q[cu[i]:cu[i + 1]], scale)
+        assert_close(out[cu[i]:cu[i + 1]], ref, f"seq {i}")
+    assert pair.gpu.device_status() == 0
