@@ -56,29 +56,3 @@ def test_tail_launch_matches_oracle(n_q, prefix, d, hq):
     assert pair.gpu.last_attn_plan()[2] == n_pairs * 8
     assert_close(out0[torch.from_numpy(rows).cuda()], ref, f"single pass n_q={n_q}")
 
-
-@pytest.mark.parametrize("n_q,prefix,d,hq", [(1280, 4096, 128, 32), (1344, 3000, 128, 32), (5120, 2048, 64, 8)])
-def test_tail_on_persistent_kernel(n_q, prefix, d, hq):
-    """The default kernel choice: the tail plan's lightest pairs run on the
-    persistent kernel, launched right behind the one-item launch, starting as
-    its CTAs finish and waiting for it only before exiting.  Rows of both
-    launches against the oracle."""
-    pair, s, q = _case(n_q, prefix, seed=n_q + 1, d=d, hq=hq)
-    pair.gpu.set_option("attn_kernel", 1)
-    scale = 1 / math.sqrt(d)
-    g4 = hq // 8
-    bmq = 128 // g4
-    tail_rows = np.arange(0, 4 * bmq)
-    rest = np.unique(np.concatenate([np.arange(4 * bmq, n_q, 29), [n_q - 1]]))
-    rows = np.concatenate([tail_rows, rest])
-    ref = oracle.replay_attention(pair.orc, s, 0, q, scale, rows=rows)
-    out = pair.gpu.replay_attn(s, 0, dev(q))
-    torch.cuda.synchronize()
-    split, n_splits, ctas = pair.gpu.last_attn_plan()
-    assert split == 1 and ctas > 152, (split, n_splits, ctas)
-    assert_close(out[torch.from_numpy(rows).cuda()], ref, f"persistent tail n_q={n_q}")
-    assert pair.gpu.device_status() == 0
-    # a second call on the same cache (its merge counters back at zero) gives the same bits
-    out2 = pair.gpu.replay_attn(s, 0, dev(q))
-    torch.cuda.synchronize()
-    assert torch.equal(out, out2)
