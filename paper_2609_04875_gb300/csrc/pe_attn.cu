@@ -14,7 +14,8 @@
 //                   (TMEM lane r); masks, online softmax in fp32 (exp2),
 //                   writes P (bf16) back into TMEM (d = 128: over its S
 //                   columns; d = 64: into its own P columns), rescales O in
-//                   TMEM when needed, epilogue.
+//                   TMEM when needed, epilogue (a full q-tile's O goes to
+//                   shared memory, then out by one TMA store per 64 columns).
 //   warp 8          producer: reads the page table; its lanes issue one TMA
 //                   box per (page, 64-column half) into K and V stage rings.
 //   warp 9          MMA: allocates TMEM; one thread issues tcgen05.mma for
@@ -66,8 +67,8 @@ struct AttnCfg {
     static constexpr int kOffV = kOffK + kStages * kTileBytes;
     static constexpr int kOffBar = kOffV + kStages * kTileBytes;
     // barriers: q_full, k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_full[2], o_done[2],
-    // s_free[2]
-    static constexpr int kNumBars = 1 + 4 * kStages + 8;
+    // s_free[2], o_staged[2]
+    static constexpr int kNumBars = 1 + 4 * kStages + 10;
     // TMEM columns: S_0, S_1 (128 each), O_0, O_1 (HD each); for d = 64 the 128 left over hold P_0 and
     // P_1 (64 each), so S(j+1) need not wait for the P V GEMM of tile j (P(j) lives apart from S)
     static constexpr bool kSepP = HD == 64;
@@ -90,7 +91,8 @@ struct TileGeo {
 template <int HD, bool SPLIT>
 __global__ void __launch_bounds__(kThreads, 1)
     replay_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                       const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ AttnParams p)
+                       const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o,
+                       const __grid_constant__ AttnParams p)
 {
     using C = AttnCfg<HD>;
     extern __shared__ uint8_t smem_raw[];
@@ -167,6 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t b_p_full = b_s_full + 16;               // [2]
     const uint32_t b_o_done = b_p_full + 16;               // [2]
     const uint32_t b_s_free = b_o_done + 16;               // [2] (d = 64) S_t has been read into registers
+    const uint32_t b_o_staged = b_s_free + 16;             // [2] O_t (bf16) is in Q_t's shared memory
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kOffMisc);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + C::kOffMisc + 4);
     const WaitCtx wctx{abort_flag, p.status};
@@ -220,6 +223,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ptx::mbar_init(b_p_full + 8 * t, 128);
                 ptx::mbar_init(b_o_done + 8 * t, 1);
                 ptx::mbar_init(b_s_free + 8 * t, 128);
+                ptx::mbar_init(b_o_staged + 8 * t, 128);
             }
             *abort_flag = 0;
             ptx::fence_barrier_init();
@@ -227,6 +231,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::prefetch_tensormap(&tm_q);
             ptx::prefetch_tensormap(&tm_k);
             ptx::prefetch_tensormap(&tm_v);
+            if (!SPLIT) ptx::prefetch_tensormap(&tm_o);
         }
         ptx::griddep_wait();
         if (n_all > 0) page_next = page_of(0);
@@ -487,7 +492,43 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ptx::tc_fence_after();
                 const float inv = l > 0.f ? 1.0f / l : 0.f;
                 const int head = kvh * g + (row % g);
-                if (!SPLIT) {
+                if (!SPLIT && (G.q_last - G.q_first + 1) * g == kBM) {
+                    // a full q-tile: O in bf16 into Q_t's shared memory (its S GEMMs are long done), laid
+                    // out as the Q box was loaded (128-byte rows, 16-byte chunks swizzled by row & 7), then
+                    // one TMA store per 64-column region; a ragged tile (other sequences' rows follow its
+                    // last query) takes the plain stores below
+                    const uint32_t qt_smem = q_smem + t * C::kTileBytes;
+#pragma unroll
+                    for (int ch = 0; ch < HD / 32; ++ch) {
+                        float o[32];
+                        ptx::tmem_ld32(tO + ch * 32, o);
+                        ptx::tmem_wait_ld();
+                        const uint32_t rbase = qt_smem + (ch >> 1) * C::kRegionBytes + row * 128;
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const int c = (ch & 1) * 4 + k;  // 16-byte chunk within the 128-byte row
+                            const uint32_t a = rbase + ((c ^ (row & 7)) << 4);
+                            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a),
+                                         "r"(pack_bf16(o[8 * k + 0] * inv, o[8 * k + 1] * inv)),
+                                         "r"(pack_bf16(o[8 * k + 2] * inv, o[8 * k + 3] * inv)),
+                                         "r"(pack_bf16(o[8 * k + 4] * inv, o[8 * k + 5] * inv)),
+                                         "r"(pack_bf16(o[8 * k + 6] * inv, o[8 * k + 7] * inv))
+                                         : "memory");
+                        }
+                    }
+                    ptx::fence_proxy_async_smem();  // the stores above, seen by the TMA store
+                    ptx::mbar_arrive(b_o_staged + 8 * t);
+                    if (row == 0) {
+                        if (wait_bar(b_o_staged + 8 * t, 0, wctx)) {
+#pragma unroll
+                            for (int r = 0; r < C::kRegions; ++r)
+                                ptx::tma_store_3d(&tm_o, r * 64, kvh * g, sq.q_row0 + G.q_first,
+                                                  qt_smem + r * C::kRegionBytes);
+                            ptx::bulk_commit_group();
+                            ptx::bulk_wait_read_all();  // shared memory stays until the copies have read it
+                        }
+                    }
+                } else if (!SPLIT) {
                     __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) +
                                          (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD;
 #pragma unroll
@@ -652,7 +693,7 @@ cudaError_t static_scratch(float **ptr)
 
 template <int HD, bool SPLIT>
 static cudaError_t launch_attn_t(const CUtensorMap &q, const CUtensorMap &k, const CUtensorMap &v,
-                                 const AttnParams &p, cudaStream_t st)
+                                 const CUtensorMap &o, const AttnParams &p, cudaStream_t st)
 {
     using C = AttnCfg<HD>;
     static bool configured = false;
@@ -672,19 +713,19 @@ static cudaError_t launch_attn_t(const CUtensorMap &q, const CUtensorMap &k, con
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, replay_attn_kernel<HD, SPLIT>, q, k, v, p);
+    return cudaLaunchKernelEx(&cfg, replay_attn_kernel<HD, SPLIT>, q, k, v, o, p);
 }
 
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
-                               const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st)
+                               const CUtensorMap &tm_v, const CUtensorMap &tm_o, const AttnParams &p, cudaStream_t st)
 {
     if (p.total_items <= 0) return cudaSuccess;
     if (head_dim == 128)
-        return split ? launch_attn_t<128, true>(tm_q, tm_k, tm_v, p, st)
-                     : launch_attn_t<128, false>(tm_q, tm_k, tm_v, p, st);
+        return split ? launch_attn_t<128, true>(tm_q, tm_k, tm_v, tm_o, p, st)
+                     : launch_attn_t<128, false>(tm_q, tm_k, tm_v, tm_o, p, st);
     if (head_dim == 64)
-        return split ? launch_attn_t<64, true>(tm_q, tm_k, tm_v, p, st)
-                     : launch_attn_t<64, false>(tm_q, tm_k, tm_v, p, st);
+        return split ? launch_attn_t<64, true>(tm_q, tm_k, tm_v, tm_o, p, st)
+                     : launch_attn_t<64, false>(tm_q, tm_k, tm_v, tm_o, p, st);
     return cudaErrorInvalidValue;
 }
 

@@ -1014,9 +1014,10 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     });
     if (order.empty()) return PE_OK;
 
-    CUtensorMap tm_q;
+    CUtensorMap tm_q, tm_o;  // Q, and the output as a map of the same shape (TMA stores of full q-tiles)
     pe_status s = encode_q(&tm_q, Q, q_rows, hq, d, g);
     if (s != PE_OK) return s;
+    if ((s = encode_q(&tm_o, out, q_rows, hq, d, g)) != PE_OK) return s;
 
     // split-KV decision over the whole launch group; plan_est: the cost model's time of the plan
     double plan_est = 0.0;
@@ -1226,7 +1227,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         c->last_splits = tail ? static_cast<int32_t>(tp.splits) : (split ? p.seqs[0].n_splits : 1);
         c->last_ctas = p.total_items + (tail ? static_cast<int32_t>(tp.pairs * hkv * tp.splits) : 0);
         if (injected_failure(c)) return launch_fault("replay attention");
-        cudaError_t e = launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, p, st);
+        cudaError_t e = launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, tm_o, p, st);
         if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
         c->launches++;
         if (split) {
@@ -1250,7 +1251,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             p.part_o = c->d_ws;
             p.part_lse = c->d_ws + tp.qtiles * hkv * tp.splits * kBM * d;
             if (injected_failure(c)) return launch_fault("replay attention tail");
-            e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, p, st);
+            e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, tm_q, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "replay attention tail launch");
             c->launches++;
             if (injected_failure(c)) return launch_fault("split-KV combine");
@@ -1789,7 +1790,7 @@ pe_status pe_replay_attn_static_scratch(pe_cache *c, int32_t seq, int32_t layer,
     p.part_lse = scratch + prow * d;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (injected_failure(c)) return launch_fault("replay attention");
-    e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, p, st);
+    e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, tm_q, p, st);
     if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
     c->launches++;
     if (injected_failure(c)) return launch_fault("split-KV combine");

@@ -193,8 +193,9 @@ cudaError_t launch_table_copy(int32_t *page_table, int32_t src_row, int32_t dst_
 cudaError_t launch_cow_copy(uint4 *k_pool, uint4 *v_pool, int32_t src, int32_t dst, int32_t slots, int32_t L,
                             int32_t hkv, int32_t ps, int32_t dvec, int32_t num_pages, int32_t *table_entry,
                             cudaStream_t st);
+// tm_o: the output as a map of the same shape as tm_q (full q-tiles are stored by TMA); unused when split
 cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q, const CUtensorMap &tm_k,
-                               const CUtensorMap &tm_v, const AttnParams &p, cudaStream_t st);
+                               const CUtensorMap &tm_v, const CUtensorMap &tm_o, const AttnParams &p, cudaStream_t st);
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st);
 // Persistent stream-K attention (p.n_ctas CTAs), cut units merged in the kernel.
 cudaError_t launch_replay_attn_sk(int head_dim, const CUtensorMap &tm_q, const CUtensorMap &tm_k,

@@ -108,6 +108,19 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+// Tiled store shared -> global of one box (cp.async.bulk.tensor, bulk-group
+// completion): commit the group, then wait until the copies have read shared
+// memory before it is reused or the CTA exits.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, int32_t x, int32_t y, int32_t z, uint32_t src)
+{
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(z), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit_group() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+
 // Untiled bulk copy global -> shared (cp.async.bulk): `bytes` (a multiple of
 // 16) from a 16-byte aligned global address to a 16-byte aligned shared
 // address, completing its bytes on the mbarrier.
