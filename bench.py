@@ -308,18 +308,18 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "tiny": {"bytes": 1.500672e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
-             "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
-    "agent_batch": {"bytes": 684.605e6 + 317.062e6, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
+    "tiny": {"bytes": 1.504e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
+             "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5"}},
+    "agent_batch": {"bytes": 684.728576e6 + 320.38016e6, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5"}},
     "short_suffix": {"bytes": 1.078952192e9 + 5.8368e6, "profile": "profiles/traffic_attention_configs.md",
                      "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
-    "long_suffix": {"bytes": 1.41242e9 + 1.03806e9, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad"}},
+    "long_suffix": {"bytes": 1.41010381e9 + 1.04442266e9, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5"}},
     # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
     # tail launch runs), per layer: bytes / 160
-    "tau_sweep": {"bytes": (47494.0e6 + 9046.57e6) / 160, "profile": "profiles/traffic_attention_configs.md",
-                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "8e585eef63b81350f8848a191e416e6f583f776d7af20c327c8d7b1ffa66a5ad", "prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
+    "tau_sweep": {"bytes": (48747.7e6 + 9344.64e6) / 160, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5", "prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
     "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
                      "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},
