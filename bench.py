@@ -615,6 +615,9 @@ def measure(name, args, rank, world, local_rank, dev, peaks, peak_src, headline)
     stream = torch.cuda.current_stream(dev)
     dist = world > 1
     units, comp, shared = build_units(name, rank, dev)
+    for u in units + ([comp] if comp else []):
+        for key, val in args.set:
+            u.drv.cache.set_option(key, val)
     for _ in range(args.warmup):
         for u in units:
             u.drv.step()
@@ -782,7 +785,7 @@ def run_pe(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": f"synthetic (seeded N(0,{w.std:.4g}^2) bf16 Q/K/V; no dataset)",
-        "config": cfg,
+        "config": dict(cfg, **({"options": dict(args.set)} if args.set else {})),
         "roofline": rep["roofline"],
         "cpu_baseline": rep.get("cpu_baseline"),
         "clocks": rep["clocks"],
@@ -1048,6 +1051,13 @@ def run_reference(args, rank, world):
     print(json.dumps(result), flush=True)
 
 
+def _option(text):
+    key, sep, val = text.partition("=")
+    if not sep or not key:
+        raise argparse.ArgumentTypeError(f"expected KEY=VALUE, got {text!r}")
+    return key, int(val)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -1068,6 +1078,9 @@ def main():
     ap.add_argument("--cpu-budget-other", type=float, default=3.0,
                     help="seconds of oracle work for each non-headline configuration's cpu_baseline")
     ap.add_argument("--ref-step-budget", type=float, default=2.0, help="seconds of oracle work per reference step")
+    ap.add_argument("--set", action="append", default=[], type=_option, metavar="KEY=VALUE",
+                    help="a cache option (pe_cache_set_option) applied to every workload cache, e.g. attn_kernel=2; "
+                         "named in config.options")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))

@@ -61,3 +61,14 @@ def test_reference_arm_prints_one_contract_line():
     assert "N(0,1^2)" in d["data"]  # the tiny workload draws unscaled N(0, 1) values
     # ms_per_step is the measured wall time of a step's bounded sample, not an extrapolation
     assert d["ms_per_step"] < 5000 and d["full_step_ms_extrapolated"] > 0
+
+
+def test_option_flag_parses_key_value_pairs():
+    import argparse
+
+    import pytest
+    assert bench._option("attn_kernel=2") == ("attn_kernel", 2)
+    assert bench._option("splitkv=-1") == ("splitkv", -1)
+    for bad in ("attn_kernel", "=2", "attn_kernel=x"):
+        with pytest.raises((argparse.ArgumentTypeError, ValueError)):
+            bench._option(bad)
