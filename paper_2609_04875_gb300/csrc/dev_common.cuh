@@ -119,6 +119,15 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
         : "memory");
 }
 
+// Split partials (O / l, fp32, HD columns a row) are stored in blocks of 32 rows, 16-byte chunk major:
+// chunk k of row r at [r & ~31][k][r & 31].  Row blocks start at multiples of 32 rows, so a warp whose
+// lane i holds row 32 w + i writes or reads one chunk of its 32 rows as 512 contiguous bytes.
+template <int HD>
+__device__ __forceinline__ float4 *part_chunk(float *part_o, int64_t row, int k)
+{
+    return reinterpret_cast<float4 *>(part_o + (row & ~static_cast<int64_t>(31)) * HD) + k * 32 + (row & 31);
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);

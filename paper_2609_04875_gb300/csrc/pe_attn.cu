@@ -549,18 +549,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 } else {
                     const int64_t prow = sq.part_row0 +
                                          (static_cast<int64_t>(G.qt * p.hkv + kvh) * sq.n_splits + split) * kBM + row;
-                    float *dst = p.part_o + prow * HD;
 #pragma unroll
                     for (int ch = 0; ch < HD / 32; ++ch) {
                         float o[32];
                         ptx::tmem_ld32(tO + ch * 32, o);
                         ptx::tmem_wait_ld();
                         if (valid && l > 0.f) {
-                            float4 *d4 = reinterpret_cast<float4 *>(dst + ch * 32);
 #pragma unroll
                             for (int k = 0; k < 8; ++k)
-                                d4[k] = make_float4(o[4 * k] * inv, o[4 * k + 1] * inv, o[4 * k + 2] * inv,
-                                                    o[4 * k + 3] * inv);
+                                *part_chunk<HD>(p.part_o, prow, ch * 8 + k) =
+                                    make_float4(o[4 * k] * inv, o[4 * k + 1] * inv, o[4 * k + 2] * inv,
+                                                o[4 * k + 3] * inv);
                         }
                     }
                     if (valid) p.part_lse[prow] = l > 0.f ? m_ref + __log2f(l) : -INFINITY;
@@ -605,7 +604,9 @@ cudaError_t launch_bounded_wait_selftest(int32_t *status, uint64_t limit_ns, cud
     return cudaGetLastError();
 }
 
-// One warp per output row: LSE-weighted merge of the split partials.
+// LSE-weighted merge of the split partials: one warp per 32 rows (a row block of the partials) and 32
+// columns, lane i on row 32 w + i, so every load of a split's chunk is 512 contiguous bytes.  For each
+// row, in split order: w_s = 2^(lse_s - max lse), den += w_s, acc += w_s O_s.
 template <int HD>
 __global__ void __launch_bounds__(256) splitkv_combine_kernel(const __grid_constant__ AttnParams p)
 {
@@ -613,56 +614,59 @@ __global__ void __launch_bounds__(256) splitkv_combine_kernel(const __grid_const
     // for its partials; the next kernel may start its own set-up meanwhile
     ptx::griddep_launch_dependents();
     ptx::griddep_wait();
+    constexpr int kGroups = HD / 32;  // column groups of 32 (8 chunks of 16 bytes)
     const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
-    if (gw >= p.total_comb) return;
+    const int blk = gw / kGroups, cg = gw % kGroups;
+    const int rbase = blk * 32;  // first combine row of this warp's block
+    if (rbase >= p.total_comb) return;
     int si = 0;
-    while (si + 1 < p.n_seqs && gw >= p.seqs[si + 1].comb0) ++si;
+    while (si + 1 < p.n_seqs && rbase >= p.seqs[si + 1].comb0) ++si;
     const AttnSeq &sq = p.seqs[si];
-    const int local = gw - sq.comb0;
+    const int local = rbase + lane - sq.comb0;
     const int row = local % kBM;
-    const int unit = local / kBM;  // qt * hkv + kvh
+    const int unit = local / kBM;  // qt * hkv + kvh (the same for the whole block)
     const int kvh = unit % p.hkv;
     const int qt = unit / p.hkv;
     const int g = p.group;
     const int qi = qt * (kBM / g) + row / g;
-    if (qi >= sq.n_q) return;
     const int64_t base = sq.part_row0 + static_cast<int64_t>(unit) * sq.n_splits * kBM + row;
     const int ns = sq.n_splits;
-    // the splits' LSEs in one round of loads (lane s holds split s's, s < 32), then their max
-    float my = lane < ns ? p.part_lse[base + static_cast<int64_t>(lane) * kBM] : -INFINITY;
-    float mx = my;
-    for (int s = 32 + lane; s < ns; s += 32) mx = fmaxf(mx, p.part_lse[base + static_cast<int64_t>(s) * kBM]);
+    float mx = -INFINITY;
+    for (int s = 0; s < ns; ++s) mx = fmaxf(mx, p.part_lse[base + static_cast<int64_t>(s) * kBM]);
+    float acc[32];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    constexpr int kPer = HD / 32;
-    float acc[kPer];
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
+    for (int i = 0; i < 32; ++i) acc[i] = 0.f;
     float den = 0.f;
     if (mx != -INFINITY) {
-#pragma unroll 4
+#pragma unroll 2
         for (int s = 0; s < ns; ++s) {
             const int64_t r = base + static_cast<int64_t>(s) * kBM;
-            const float lse = s < 32 ? __shfl_sync(0xffffffffu, my, s) : p.part_lse[r];
+            const float lse = p.part_lse[r];
             if (lse == -INFINITY) continue;
             const float w = ex2(lse - mx);
             den += w;
-            const float *src = p.part_o + r * HD + lane * kPer;
 #pragma unroll
-            for (int k = 0; k < kPer; ++k) acc[k] += w * src[k];
+            for (int k = 0; k < 8; ++k) {
+                const float4 v = *part_chunk<HD>(p.part_o, r, cg * 8 + k);
+                acc[4 * k + 0] += w * v.x;
+                acc[4 * k + 1] += w * v.y;
+                acc[4 * k + 2] += w * v.z;
+                acc[4 * k + 3] += w * v.w;
+            }
         }
     }
+    if (qi >= sq.n_q) return;
     const float inv = den > 0.f ? 1.0f / den : 0.f;
     const int head = kvh * g + (row % g);
-    __nv_bfloat16 *dst = reinterpret_cast<__nv_bfloat16 *>(p.out) +
-                         (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD + lane * kPer;
-    if constexpr (kPer == 4) {
-        *reinterpret_cast<uint2 *>(dst) =
-            make_uint2(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv));
-    } else {
-        *reinterpret_cast<uint32_t *>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
-    }
+    uint4 *dst = reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(p.out) +
+                                           (static_cast<int64_t>(sq.q_row0 + qi) * p.hq + head) * HD + cg * 32);
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        dst[k] = make_uint4(pack_bf16(acc[8 * k + 0] * inv, acc[8 * k + 1] * inv),
+                            pack_bf16(acc[8 * k + 2] * inv, acc[8 * k + 3] * inv),
+                            pack_bf16(acc[8 * k + 4] * inv, acc[8 * k + 5] * inv),
+                            pack_bf16(acc[8 * k + 6] * inv, acc[8 * k + 7] * inv));
 }
 
 // Split-KV partials of pe_replay_attn_static_scratch: a fixed 16 MiB array that
@@ -732,8 +736,10 @@ cudaError_t launch_replay_attn(int head_dim, bool split, const CUtensorMap &tm_q
 cudaError_t launch_splitkv_combine(int head_dim, const AttnParams &p, cudaStream_t st)
 {
     if (p.total_comb <= 0) return cudaSuccess;
+    if (head_dim != 64 && head_dim != 128) return cudaErrorInvalidValue;
     const int warps_per_block = 8;
-    const int blocks = (p.total_comb + warps_per_block - 1) / warps_per_block;
+    const int64_t warps = static_cast<int64_t>(p.total_comb + 31) / 32 * (head_dim / 32);  // row blocks x column groups
+    const int blocks = static_cast<int>((warps + warps_per_block - 1) / warps_per_block);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(blocks));
     cfg.blockDim = dim3(256);

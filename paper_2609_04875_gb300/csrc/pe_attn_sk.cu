@@ -189,10 +189,9 @@ __device__ __forceinline__ void merge_parts_row(const SkParams &P, int slot, int
             const float lse = __ldcg(p.part_lse + r0 + q * kStride);
             if (lse == -INFINITY) continue;
             const float w = ex2(lse - mx);
-            const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (r0 + q * kStride) * HD + c0);
 #pragma unroll
             for (int i = 0; i < kCh / 4; ++i) {
-                const float4 v = __ldcg(src + i);
+                const float4 v = __ldcg(part_chunk<HD>(p.part_o, r0 + q * kStride, c0 / 4 + i));
                 acc[4 * i + 0] += w * v.x;
                 acc[4 * i + 1] += w * v.y;
                 acc[4 * i + 2] += w * v.z;
@@ -266,10 +265,9 @@ __device__ __forceinline__ void merge_own_row(const SkParams &P, int slot, int t
                 }
             } else if (valid && lse[q] != -INFINITY) {
                 const float w = ex2(lse[q] - mx);
-                const float4 *src = reinterpret_cast<const float4 *>(p.part_o + (r0 + q * kStride) * HD + c0);
 #pragma unroll
                 for (int i = 0; i < kCh / 4; ++i) {
-                    const float4 v = __ldcg(src + i);
+                    const float4 v = __ldcg(part_chunk<HD>(p.part_o, r0 + q * kStride, c0 / 4 + i));
                     acc[4 * i + 0] += w * v.x;
                     acc[4 * i + 1] += w * v.y;
                     acc[4 * i + 2] += w * v.z;
@@ -675,18 +673,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                     merge_own_row<HD, true>(P, pc.slot, t, row, n_parts, pc.part, true, tO, l, m_ref, valid,
                                             out_row);
                 } else if (pc.slot >= 0) {
-                    float *dst = p.part_o + prow * HD;
 #pragma unroll
                     for (int ch = 0; ch < HD / 32; ++ch) {
                         float o[32];
                         ptx::tmem_ld32(tO + ch * 32, o);
                         ptx::tmem_wait_ld();
                         if (valid && l > 0.f) {
-                            float4 *d4 = reinterpret_cast<float4 *>(dst + ch * 32);
 #pragma unroll
                             for (int q = 0; q < 8; ++q)
-                                d4[q] = make_float4(o[4 * q] * inv, o[4 * q + 1] * inv, o[4 * q + 2] * inv,
-                                                    o[4 * q + 3] * inv);
+                                *part_chunk<HD>(p.part_o, prow, ch * 8 + q) =
+                                    make_float4(o[4 * q] * inv, o[4 * q + 1] * inv, o[4 * q + 2] * inv,
+                                                o[4 * q + 3] * inv);
                         }
                     }
                     if (valid) p.part_lse[prow] = l > 0.f ? m_ref + __log2f(l) : -INFINITY;

@@ -88,7 +88,7 @@ struct AttnSeq {
 struct AttnParams {
     const int32_t *page_table;
     void *out;             // bf16 [rows][Hq][d]
-    float *part_o;         // split-KV partial outputs [rows][d]
+    float *part_o;         // split-KV partial outputs, rows of d fp32 in blocks of 32 rows (part_chunk)
     float *part_lse;       // split-KV partial log2-sum-exp [rows]
     int32_t *status;
     int32_t n_seqs, hq, hkv, group, layer, num_pages, ps, oob_row;
