@@ -309,17 +309,17 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
     "tiny": {"bytes": 1.504e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
-             "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5"}},
-    "agent_batch": {"bytes": 684.728576e6 + 320.38016e6, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5"}},
-    "short_suffix": {"bytes": 1.078952192e9 + 5.8368e6, "profile": "profiles/traffic_attention_configs.md",
-                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
-    "long_suffix": {"bytes": 1.41010381e9 + 1.04442266e9, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5"}},
+             "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359"}},
+    "agent_batch": {"bytes": 685.711e6 + 320.274e6, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359"}},
+    "short_suffix": {"bytes": 1.07887e9 + 6.36774e6, "profile": "profiles/traffic_attention_configs.md",
+                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "ffe591d6de5c87ba8464bc1189084cb0396d057c64577477cb0569b032625c0a"}},
+    "long_suffix": {"bytes": 1.41209e9 + 1.04485e9, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359"}},
     # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
     # tail launch runs), per layer: bytes / 160
-    "tau_sweep": {"bytes": (48747.7e6 + 9344.64e6) / 160, "profile": "profiles/traffic_attention_configs.md",
-                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "f3496bfaadc0e34a1b0f24742df1e0855e50011858a4b191ec55bb7b708b97f5", "prefill_sk": "f0aa50c0085f4b67fbd8105b7719f9584c8e9948d3114c502c14d98a6fb22544"}},
+    "tau_sweep": {"bytes": (49582.1e6 + 9415.19e6) / 160, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359", "prefill_sk": "ffe591d6de5c87ba8464bc1189084cb0396d057c64577477cb0569b032625c0a"}},
     "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
                      "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},
