@@ -646,6 +646,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool last = pc.slot >= 0 && n_parts <= kMaxOwnMergeParts &&
                               __shfl_sync(0xffffffffu, seen, 0) == n_parts - 1;
             if (last) __threadfence();  // the other parts' rows, written before their tickets
+            if (last && lane == 0) {
+                // the other parts were written long before (often back in DRAM by now): start bringing
+                // this warp's 32-row blocks of them into L2 while the last P V GEMM completes
+                for (int q = 0; q < n_parts; ++q) {
+                    if (q == pc.part) continue;
+                    const int64_t rq = (static_cast<int64_t>(pc.slot) * P.max_parts + q) * (2 * kBM) + t * kBM +
+                                       (warp & 3) * 32;
+                    ptx::prefetch_l2_bulk(p.part_o + rq * HD, 32 * HD * 4);
+                    ptx::prefetch_l2_bulk(p.part_lse + rq, 32 * 4);
+                }
+            }
             if (G.ntiles > 0) {
                 // ---- epilogue: O / l, bf16 output or fp32 partial
                 if (!wait_bar_warp(b_o, (cnt + G.ntiles - 1) & 1, wctx)) { ok = false; break; }
