@@ -107,29 +107,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     // sequence the kv-heads run fastest (every head's heaviest pairs first), or, when p.pairs_fastest
     // is set (launches of many waves), the pairs: then the CTAs resident at once work on one or two
     // kv-heads' keys, which stay in L2 while Q and O stream through.
-    const int item = blockIdx.x;
-    int si = 0, si_hi = p.n_seqs;  // the last sequence whose first item is at most `item` (binary search)
-    while (si_hi - si > 1) {
-        const int mid = (si + si_hi) >> 1;
-        if (p.seqs[mid].item0 <= item) si = mid;
-        else si_hi = mid;
-    }
+    auto decode_item = [&](int item, int &si, int &kvh, int &split, int &pair) {
+        si = 0;
+        int si_hi = p.n_seqs;  // the last sequence whose first item is at most `item` (binary search)
+        while (si_hi - si > 1) {
+            const int mid = (si + si_hi) >> 1;
+            if (p.seqs[mid].item0 <= item) si = mid;
+            else si_hi = mid;
+        }
+        const AttnSeq &q = p.seqs[si];
+        int local = item - q.item0;
+        if (p.pairs_fastest) {
+            const int seq_items = (si + 1 < p.n_seqs ? p.seqs[si + 1].item0 : p.total_items) - q.item0;
+            const int n_pairs = seq_items / (p.hkv * q.n_splits);  // pairs of this sequence in the launch
+            pair = q.pair_top - 1 - local % n_pairs;
+            local /= n_pairs;
+            split = local % q.n_splits;
+            kvh = local / q.n_splits;
+        } else {
+            kvh = local % p.hkv;
+            local /= p.hkv;
+            split = local % q.n_splits;
+            pair = q.pair_top - 1 - local / q.n_splits;
+        }
+    };
+    int si, kvh, split, pair;
+    decode_item(blockIdx.x, si, kvh, split, pair);
     const AttnSeq &sq = p.seqs[si];
-    int local = item - sq.item0;
-    int kvh, split, pair;
-    if (p.pairs_fastest) {
-        const int seq_items = (si + 1 < p.n_seqs ? p.seqs[si + 1].item0 : p.total_items) - sq.item0;
-        const int n_pairs = seq_items / (p.hkv * sq.n_splits);  // pairs of this sequence in the launch
-        pair = sq.pair_top - 1 - local % n_pairs;
-        local /= n_pairs;
-        split = local % sq.n_splits;
-        kvh = local / sq.n_splits;
-    } else {
-        kvh = local % p.hkv;
-        local /= p.hkv;
-        split = local % sq.n_splits;
-        pair = sq.pair_top - 1 - local / sq.n_splits;
-    }
     const int g = p.group;
     const int bmq = kBM / g;
     const int kt0 = SPLIT ? split * p.split_tiles : 0;
@@ -267,6 +271,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int page = page_next;
             if (i + 1 < n_all) page_next = page_of(i + 1);  // prefetch the next tile's page ids
             if (!issue_kv(i, page)) break;
+        }
+        // With one CTA per SM, the CTA that starts on this SM next is about blockIdx.x + next_stride:
+        // bring its Q tiles (read once, from DRAM) into L2 now, so that its first S GEMMs wait less.
+        const int nxt = blockIdx.x + p.next_stride;
+        if (p.next_stride > 0 && nxt < p.total_items && lane == 0 && !*abort_flag) {
+            int nsi, nkvh, nsplit, npair;
+            decode_item(nxt, nsi, nkvh, nsplit, npair);
+            const AttnSeq &nq = p.seqs[nsi];
+            for (int t = 0; t < 2; ++t) {
+                const int qt = 2 * npair + t;
+                if (qt >= nq.n_qtiles) break;
+                for (int r = 0; r < C::kRegions; ++r)
+                    ptx::tma_prefetch_3d(&tm_q, r * 64, nkvh * g, nq.q_row0 + qt * (kBM / g));
+            }
         }
         __syncwarp();
         if (*abort_flag && lane == 0) {

@@ -1085,6 +1085,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         p.ps = cf.page_size;
         p.oob_row = static_cast<int32_t>(c->pool_rows);
         p.scale_log2 = scale * 1.4426950408889634f;
+        p.next_stride = c->num_sms;  // one CTA per SM: CTA b's successor on its SM is about b + SMs
         for (;;) {
             int32_t item = 0, comb = 0;
             int64_t prow = 0;

@@ -96,6 +96,7 @@ struct AttnParams {
     int32_t total_items;
     int32_t total_comb;
     int32_t pairs_fastest;  // one-item kernel: number a sequence's items pairs fastest (else kv-heads fastest)
+    int32_t next_stride;   // one-item kernel: CTA b prefetches item b + next_stride's Q tiles into L2 (0: off)
     float scale_log2;      // softmax_scale * log2(e)
     AttnSeq seqs[kMaxSegs];
 };
