@@ -308,18 +308,18 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "tiny": {"bytes": 1.504e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
-             "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359"}},
-    "agent_batch": {"bytes": 685.711e6 + 320.274e6, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359"}},
-    "short_suffix": {"bytes": 1.07887e9 + 6.36774e6, "profile": "profiles/traffic_attention_configs.md",
-                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "ffe591d6de5c87ba8464bc1189084cb0396d057c64577477cb0569b032625c0a"}},
-    "long_suffix": {"bytes": 1.41209e9 + 1.04485e9, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359"}},
+    "tiny": {"bytes": 1.50733e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
+             "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
+    "agent_batch": {"bytes": 684.808e6 + 320.792e6, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
+    "short_suffix": {"bytes": 1.08893e9 + 6.25408e6, "profile": "profiles/traffic_attention_configs.md",
+                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f1abba8aade34190b2bd21509868db3ddaad1a6d9cba5e702417187444220de5"}},
+    "long_suffix": {"bytes": 1.41177e9 + 1.04557e9, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
     # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
     # tail launch runs), per layer: bytes / 160
-    "tau_sweep": {"bytes": (49582.1e6 + 9415.19e6) / 160, "profile": "profiles/traffic_attention_configs.md",
-                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "7fc6efc4fa8bb7768ce33e51f5c2b8df061835c1d1cd1425964073bf13054359", "prefill_sk": "ffe591d6de5c87ba8464bc1189084cb0396d057c64577477cb0569b032625c0a"}},
+    "tau_sweep": {"bytes": (49219.7e6 + 9467.3e6) / 160, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653", "prefill_sk": "f1abba8aade34190b2bd21509868db3ddaad1a6d9cba5e702417187444220de5"}},
     "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
                      "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},
