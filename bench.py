@@ -312,14 +312,14 @@ NCU_TRAFFIC = {
              "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
     "agent_batch": {"bytes": 684.808e6 + 320.792e6, "profile": "profiles/traffic_attention_configs.md",
                     "kernels": ["prefill"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
-    "short_suffix": {"bytes": 1.08893e9 + 6.25408e6, "profile": "profiles/traffic_attention_configs.md",
-                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "f1abba8aade34190b2bd21509868db3ddaad1a6d9cba5e702417187444220de5"}},
+    "short_suffix": {"bytes": 1.0883e9 + 5.88058e6, "profile": "profiles/traffic_attention_configs.md",
+                     "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "b25d958540e6002039fda210f04a46af7fb34514ee9402af13b2c16be2709172"}},
     "long_suffix": {"bytes": 1.41177e9 + 1.04557e9, "profile": "profiles/traffic_attention_configs.md",
                     "kernels": ["prefill"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
     # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
     # tail launch runs), per layer: bytes / 160
-    "tau_sweep": {"bytes": (49219.7e6 + 9467.3e6) / 160, "profile": "profiles/traffic_attention_configs.md",
-                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653", "prefill_sk": "f1abba8aade34190b2bd21509868db3ddaad1a6d9cba5e702417187444220de5"}},
+    "tau_sweep": {"bytes": (50092.5e6 + 9465.17e6) / 160, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653", "prefill_sk": "b25d958540e6002039fda210f04a46af7fb34514ee9402af13b2c16be2709172"}},
     "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
                      "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},

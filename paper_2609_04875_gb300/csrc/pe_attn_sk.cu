@@ -163,9 +163,11 @@ __device__ __forceinline__ bool piece_of(const SkParams &P, const SkCta &cw, int
 // Merge of one row of a cut unit's q-tile t from its n parts (slot `slot`):
 // O = sum_p 2^(lse_p - m) O_p / sum_p 2^(lse_p - m), m = max_p lse_p, where
 // O_p is part p's O / l and lse_p its log2-sum-exp (-inf: no visible key).
-// The parts were written by other CTAs of this grid: read through L2.
+// The parts were written by other CTAs of this grid: read through L2.  Out of
+// line (as merge_own_row), so that their accumulators do not add to the
+// register pressure of the kernel's tile loop (halves the kernel's spills).
 template <int HD>
-__device__ __forceinline__ void merge_parts_row(const SkParams &P, int slot, int t, int row, int n, uint4 *dst)
+__device__ __noinline__ void merge_parts_row(const SkParams &P, int slot, int t, int row, int n, uint4 *dst)
 {
     const AttnParams &p = P.a;
     constexpr int64_t kStride = 2 * kBM;  // rows from one part to the next
@@ -217,7 +219,7 @@ __device__ __forceinline__ void merge_parts_row(const SkParams &P, int slot, int
 // (own, tO, l and m_ref unused).  Whole warp.
 constexpr int kMaxOwnMergeParts = 4;
 template <int HD, bool kOwn>
-__device__ __forceinline__ void merge_own_row(const SkParams &P, int slot, int t, int row, int n, int own,
+__device__ __noinline__ void merge_own_row(const SkParams &P, int slot, int t, int row, int n, int own,
                                               bool has_tmem, uint32_t tO, float l, float m_ref, bool valid,
                                               uint4 *dst)
 {
