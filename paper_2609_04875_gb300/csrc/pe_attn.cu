@@ -246,7 +246,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int t = 0; t < nq; ++t)
                     for (int r = 0; r < C::kRegions; ++r)
                         ptx::tma_load_3d(q_smem + t * C::kTileBytes + r * C::kRegionBytes, &tm_q, r * 64, kvh * g,
-                                         sq.q_row0 + geo[t].q_first, b_q_full);
+                                         sq.q_row0 + (2 * pair + t) * bmq, b_q_full);
             }
         }
         __syncwarp();
@@ -386,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // =================================================== softmax / epilogue
         ptx::griddep_wait();                     // before this role's first global write
         const int t = warp >> 2;                 // q-tile of this warpgroup
-        const TileGeo &G = geo[t];
+        const TileGeo G = t ? geo[1] : geo[0];   // by value: no run-time index into geo (local memory)
         const int row = threadIdx.x & 127;       // TMEM lane
         const int qi = G.q_first + row / g;
         const bool valid = G.qt >= 0 && qi <= G.q_last;
