@@ -308,18 +308,18 @@ def oracle_tokens_per_s(units, budget_s, seed=7):
 # DRAM traffic per attention launch from one ncu capture (profiles/), valid only
 # while the kernel source is the one that was captured.
 NCU_TRAFFIC = {
-    "tiny": {"bytes": 1.50733e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
-             "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
-    "agent_batch": {"bytes": 684.808e6 + 320.792e6, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
+    "tiny": {"bytes": 1.5081e6, "profile": "profiles/traffic_attention_configs.md", "kernels": ["prefill"],
+             "src_sha256": {"prefill": "91bcdf4963eaa5385a46b5fc32b465f5b50af0d236a020b33013751418d6a9b6"}},
+    "agent_batch": {"bytes": 684.646e6 + 315.236e6, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "91bcdf4963eaa5385a46b5fc32b465f5b50af0d236a020b33013751418d6a9b6"}},
     "short_suffix": {"bytes": 1.0883e9 + 5.88058e6, "profile": "profiles/traffic_attention_configs.md",
                      "kernels": ["prefill_sk"], "src_sha256": {"prefill_sk": "b25d958540e6002039fda210f04a46af7fb34514ee9402af13b2c16be2709172"}},
-    "long_suffix": {"bytes": 1.41177e9 + 1.04557e9, "profile": "profiles/traffic_attention_configs.md",
-                    "kernels": ["prefill"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653"}},
+    "long_suffix": {"bytes": 1.41056e9 + 1.0372e9, "profile": "profiles/traffic_attention_configs.md",
+                    "kernels": ["prefill"], "src_sha256": {"prefill": "91bcdf4963eaa5385a46b5fc32b465f5b50af0d236a020b33013751418d6a9b6"}},
     # one sweep step's 224 attention launches (5 forget requests x 32 layers, two launches per layer where a
     # tail launch runs), per layer: bytes / 160
-    "tau_sweep": {"bytes": (50092.5e6 + 9465.17e6) / 160, "profile": "profiles/traffic_attention_configs.md",
-                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "da0c4ddcee0175832edcf4c33204d8e881b3a00006576425b3d221d450a78653", "prefill_sk": "b25d958540e6002039fda210f04a46af7fb34514ee9402af13b2c16be2709172"}},
+    "tau_sweep": {"bytes": (48092.5e6 + 8159.95e6) / 160, "profile": "profiles/traffic_attention_configs.md",
+                  "kernels": ["prefill", "prefill_sk"], "src_sha256": {"prefill": "91bcdf4963eaa5385a46b5fc32b465f5b50af0d236a020b33013751418d6a9b6", "prefill_sk": "b25d958540e6002039fda210f04a46af7fb34514ee9402af13b2c16be2709172"}},
     "decode_batch": {"bytes": 341.569792e6 + 3.933952e6, "profile": "profiles/decode_tc_decode_batch.md",
                      "kernels": ["decode"],
                      "src_sha256": {"decode": "a29203afa92b6d3d8108227a2ee31a613331b3c42dd2904b8ef84b5de69006ab"}},
