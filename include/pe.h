@@ -84,7 +84,11 @@ typedef struct {
 } pe_cache_config;
 
 /* Creates a cache.  Sizes are checked (d, ps, positive counts, int32-addressable
- * pool rows).  Device buffers are allocated on the current CUDA device.
+ * pool rows).  Device buffers are allocated on the current CUDA device, which
+ * must be of compute capability 10.3 (the kernels are sm_103a code).  Every
+ * later call that does device work must be made with that device current
+ * (INVALID otherwise, before any state changes); pe_cache_destroy waits for
+ * and frees the cache on its own device, whichever device is current.
  * Errors: INVALID, UNSUPPORTED, OOM (host), CUDA. */
 pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out);
 pe_status pe_cache_destroy(pe_cache *cache);

@@ -176,15 +176,24 @@ def _stream(stream):
     return ctypes.c_void_p(int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream))
 
 
-def _dev_ptr(t, name):
+def _dev_ptr(t, name, device=None):
+    """Device pointer of a contiguous bf16 CUDA tensor; with ``device`` given,
+    the tensor must live on that CUDA device (the cache's)."""
     import torch
     if t.dtype != torch.bfloat16:
         raise TypeError(f"{name} must be bfloat16")
     if not t.is_cuda:
         raise TypeError(f"{name} must be a CUDA tensor")
+    if device is not None and t.device.index != device:
+        raise ValueError(f"{name} is on cuda:{t.device.index}, the cache on cuda:{device}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     return ctypes.c_void_p(t.data_ptr())
+
+
+def _same_shape(out, Q):
+    if out is not None and tuple(out.shape) != tuple(Q.shape):
+        raise ValueError(f"out has shape {tuple(out.shape)}, Q {tuple(Q.shape)}: they must match")
 
 
 class PagedKVCache:
@@ -194,6 +203,8 @@ class PagedKVCache:
     ``k_pool`` / ``v_pool``: optional caller-owned CUDA tensors of shape
     [L][num_pages][Hkv][page_size][d] (bf16); otherwise the library allocates.
     ``host_only=True`` keeps only the host bookkeeping (no device memory).
+    A device cache lives on the CUDA device current at construction; its calls
+    must be made with that device current, on tensors that live there.
     """
 
     def __init__(self, num_layers, num_kv_heads, head_dim, page_size, num_pages, max_seqs, max_pages_per_seq,
@@ -208,10 +219,14 @@ class PagedKVCache:
             if len(init_free_order) != num_pages:
                 raise ValueError("init_free_order must list every page")
             cfg.init_free_order = ctypes.cast(self._order, _I32P)
+        self._device = None
+        if not host_only:
+            import torch
+            self._device = torch.cuda.current_device()
         self._pools = (k_pool, v_pool)  # keep caller tensors alive
         if k_pool is not None:
-            cfg.k_pool = _dev_ptr(k_pool, "k_pool").value
-            cfg.v_pool = _dev_ptr(v_pool, "v_pool").value
+            cfg.k_pool = self._ptr(k_pool, "k_pool").value
+            cfg.v_pool = self._ptr(v_pool, "v_pool").value
         cfg.workspace_bytes = int(workspace_bytes)
         self.num_layers, self.num_kv_heads, self.head_dim = num_layers, num_kv_heads, head_dim
         self.page_size, self.num_pages, self.max_seqs = page_size, num_pages, max_seqs
@@ -245,6 +260,9 @@ class PagedKVCache:
 
     def _s(self, stream):
         return ctypes.c_void_p(None) if self.host_only else _stream(stream)
+
+    def _ptr(self, t, name):
+        return _dev_ptr(t, name, self._device)
 
     # -- sequences -----------------------------------------------------------
     def seq_create(self) -> int:
@@ -312,7 +330,7 @@ class PagedKVCache:
             _check(_lib.pe_append_kv(self._h, seq, None, None, int(n_tokens), self._s(stream)))
             return
         self._check_kv(K, V)
-        _check(_lib.pe_append_kv(self._h, seq, _dev_ptr(K, "K"), _dev_ptr(V, "V"), K.shape[1], self._s(stream)))
+        _check(_lib.pe_append_kv(self._h, seq, self._ptr(K, "K"), self._ptr(V, "V"), K.shape[1], self._s(stream)))
 
     def append_kv_batch(self, seqs, K=None, V=None, cu_tokens=None, stream=None):
         """K, V: CUDA bf16 [L][cu_tokens[-1]][Hkv][d]; sequence i gets tokens cu_tokens[i]:cu_tokens[i+1]."""
@@ -325,7 +343,7 @@ class PagedKVCache:
         self._check_kv(K, V)
         if K.shape[1] != cu_tokens[-1]:
             raise ValueError("K token count does not match cu_tokens")
-        _check(_lib.pe_append_kv_batch(self._h, len(seqs), _i32_array(seqs), _dev_ptr(K, "K"), _dev_ptr(V, "V"),
+        _check(_lib.pe_append_kv_batch(self._h, len(seqs), _i32_array(seqs), self._ptr(K, "K"), self._ptr(V, "V"),
                                        cu, self._s(stream)))
 
     def _check_kv(self, K, V):
@@ -340,10 +358,11 @@ class PagedKVCache:
         import torch
         if Q.dim() != 3 or Q.shape[2] != self.head_dim:
             raise ValueError("Q must be [n_q][Hq][d]")
+        _same_shape(out, Q)
         if out is None:
             out = torch.empty_like(Q)
         scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
-        _check(_lib.pe_replay_attn(self._h, seq, layer, _dev_ptr(Q, "Q"), _dev_ptr(out, "out"), Q.shape[0],
+        _check(_lib.pe_replay_attn(self._h, seq, layer, self._ptr(Q, "Q"), self._ptr(out, "out"), Q.shape[0],
                                    Q.shape[1], scale, self._s(stream)))
         return out
 
@@ -352,11 +371,12 @@ class PagedKVCache:
         import torch
         if Q.dim() != 3 or Q.shape[2] != self.head_dim or Q.shape[0] != cu_q[-1]:
             raise ValueError("Q must be [cu_q[-1]][Hq][d]")
+        _same_shape(out, Q)
         if out is None:
             out = torch.empty_like(Q)
         scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
-        _check(_lib.pe_replay_attn_batch(self._h, len(seqs), _i32_array(seqs), layer, _dev_ptr(Q, "Q"),
-                                         _i32_array(cu_q), _dev_ptr(out, "out"), Q.shape[1], scale,
+        _check(_lib.pe_replay_attn_batch(self._h, len(seqs), _i32_array(seqs), layer, self._ptr(Q, "Q"),
+                                         _i32_array(cu_q), self._ptr(out, "out"), Q.shape[1], scale,
                                          self._s(stream)))
         return out
 
@@ -384,10 +404,11 @@ class PagedKVCache:
             raise ValueError("Q must be [L][N][Hq][d] with the rows of K")
         if K.shape[1] != cu_tok[-1]:
             raise ValueError("K row count does not match cu_tok")
+        _same_shape(out, Q)
         if out is None:
             out = torch.empty_like(Q)
         _check(_lib.pe_replay_rounds(self._h, len(seqs), _i32_array(seqs), n_rounds, take_p, _i32_array(cu_tok),
-                                     _dev_ptr(K, "K"), _dev_ptr(V, "V"), _dev_ptr(Q, "Q"), _dev_ptr(out, "out"),
+                                     self._ptr(K, "K"), self._ptr(V, "V"), self._ptr(Q, "Q"), self._ptr(out, "out"),
                                      Q.shape[2], scale, self._s(stream)))
         return out
 
@@ -413,7 +434,7 @@ class PagedKVCache:
         if K.shape[1] != cu_tokens[-1]:
             raise ValueError("K token count does not match cu_tokens")
         keep = (K, V)
-        args = (self._h, len(seqs), _i32_array(seqs), _dev_ptr(K, "K"), _dev_ptr(V, "V"), _i32_array(cu_tokens),
+        args = (self._h, len(seqs), _i32_array(seqs), self._ptr(K, "K"), self._ptr(V, "V"), _i32_array(cu_tokens),
                 self._s(stream))
         fn = _lib.pe_append_kv_batch
 
@@ -429,8 +450,8 @@ class PagedKVCache:
             raise ValueError("Q and out must be [cu_q[-1]][Hq][d]")
         scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
         keep = (Q, out)
-        args = (self._h, len(seqs), _i32_array(seqs), int(layer), _dev_ptr(Q, "Q"), _i32_array(cu_q),
-                _dev_ptr(out, "out"), Q.shape[1], ctypes.c_float(scale), self._s(stream))
+        args = (self._h, len(seqs), _i32_array(seqs), int(layer), self._ptr(Q, "Q"), _i32_array(cu_q),
+                self._ptr(out, "out"), Q.shape[1], ctypes.c_float(scale), self._s(stream))
         fn = _lib.pe_replay_attn_batch
 
         def call():
@@ -446,10 +467,11 @@ class PagedKVCache:
         import torch
         if Q.dim() != 3 or Q.shape[2] != self.head_dim:
             raise ValueError("Q must be [n_q][Hq][d]")
+        _same_shape(out, Q)
         if out is None:
             out = torch.empty_like(Q)
         scale = 1.0 / math.sqrt(self.head_dim) if softmax_scale is None else float(softmax_scale)
-        _check(_lib.pe_replay_attn_static_scratch(self._h, seq, layer, _dev_ptr(Q, "Q"), _dev_ptr(out, "out"),
+        _check(_lib.pe_replay_attn_static_scratch(self._h, seq, layer, self._ptr(Q, "Q"), self._ptr(out, "out"),
                                                   Q.shape[0], Q.shape[1], scale, self._s(stream)))
         return out
 

@@ -718,13 +718,9 @@ static cudaError_t launch_attn_t(const CUtensorMap &q, const CUtensorMap &k, con
                                  const CUtensorMap &o, const AttnParams &p, cudaStream_t st)
 {
     using C = AttnCfg<HD>;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(replay_attn_kernel<HD, SPLIT>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::kDynSmem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    static std::atomic<uint64_t> configured{0};
+    cudaError_t e = set_dyn_smem_once(replay_attn_kernel<HD, SPLIT>, C::kDynSmem, configured);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.total_items));
     cfg.blockDim = dim3(kThreads);

@@ -745,13 +745,9 @@ cudaError_t launch_sk_t(const CUtensorMap &q, const CUtensorMap &k, const CUtens
                         cudaStream_t st)
 {
     using C = SkCfg<HD>;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(replay_attn_sk_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             C::kDynSmem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    static std::atomic<uint64_t> configured{0};
+    cudaError_t e = set_dyn_smem_once(replay_attn_sk_kernel<HD>, C::kDynSmem, configured);
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.n_ctas));
     cfg.blockDim = dim3(kThreads);

@@ -1249,13 +1249,9 @@ template <int HD, int RB>
 cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st)
 {
     using C = TcCfg<HD, RB>;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e =
-            cudaFuncSetAttribute(decode_tc_kernel<HD, RB>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kDynSmem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    static std::atomic<uint64_t> configured{0};
+    cudaError_t e = set_dyn_smem_once(decode_tc_kernel<HD, RB>, C::kDynSmem, configured);
+    if (e != cudaSuccess) return e;
     // programmatic serialization: the CTAs' set-up may overlap the tail of the previous kernel
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(p.total_ctas));
@@ -1267,7 +1263,7 @@ cudaError_t launch_tc(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const De
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<HD, RB>, tm_k, tm_v, p);
+    e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<HD, RB>, tm_k, tm_v, p);
     if (e != cudaSuccess) return e;
     // the merges, also with programmatic serialization (its launch overlaps the decode grid's end)
     cudaLaunchConfig_t ccfg = {};
@@ -1284,13 +1280,9 @@ template <int HD, int RB>
 cudaError_t launch_t(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st)
 {
     using C = DecCfg<HD, RB>;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_attn_kernel<HD, RB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             C::kDynSmem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    static std::atomic<uint64_t> configured{0};
+    cudaError_t e = set_dyn_smem_once(decode_attn_kernel<HD, RB>, C::kDynSmem, configured);
+    if (e != cudaSuccess) return e;
     decode_attn_kernel<HD, RB><<<p.total_ctas, kDecThreads, C::kDynSmem, st>>>(tm_k, tm_v, p);
     return cudaGetLastError();
 }

@@ -145,6 +145,22 @@ pe_status check_seq(const pe_cache *c, int32_t seq)
     return PE_OK;
 }
 
+// A device cache's memory and tensor maps belong to the device that was current
+// when it was created; a call made with another device current would launch
+// there with pointers that device cannot use, so it is refused before any
+// state changes.
+pe_status check_device(const pe_cache *c)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (c->host_only) return PE_OK;
+    int dev = -1;
+    const cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev != c->device)
+        return fail(PE_ERR_INVALID, "the cache lives on device %d, but device %d is current", c->device, dev);
+    return PE_OK;
+}
+
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // ---- journal: every bookkeeping change of a call, undone if the call fails
@@ -1269,6 +1285,7 @@ pe_status check_attn_args(const pe_cache *c, int32_t layer, const void *Q, const
                           bool has_rows = true)
 {
     if (c->host_only) return fail(PE_ERR_UNSUPPORTED, "attention on a host-only cache");
+    if (pe_status s = check_device(c)) return s;
     if (layer < 0 || layer >= c->cfg.num_layers) return fail(PE_ERR_RANGE, "layer %d out of range", layer);
     if (has_rows && (!Q || !out)) return fail(PE_ERR_INVALID, "null Q or out");
     if (has_rows && (!aligned16(Q) || !aligned16(out))) return fail(PE_ERR_INVALID, "Q and out must be 16-byte aligned");
@@ -1347,7 +1364,7 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
     int major = 0, minor = 0;
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, cc->device);
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, cc->device);
-    if (major != 10) {
+    if (major != 10 || minor != 3) {  // sm_103a code runs on compute capability 10.3 only
         delete cc;
         return fail(PE_ERR_UNSUPPORTED, "kernels are built for sm_103a; device is sm_%d%d", major, minor);
     }
@@ -1399,8 +1416,13 @@ pe_status pe_cache_destroy(pe_cache *cache)
 {
     if (!cache) return fail(PE_ERR_INVALID, "null cache");
     if (!cache->host_only) {
+        // wait for and free on the cache's own device, whichever device is current
+        int prev = -1;
+        const bool switched = cudaGetDevice(&prev) == cudaSuccess && prev != cache->device &&
+                              cudaSetDevice(cache->device) == cudaSuccess;
         cudaDeviceSynchronize();
         free_device(cache);
+        if (switched) cudaSetDevice(prev);
     }
     delete cache;
     return PE_OK;
@@ -1426,7 +1448,9 @@ pe_status pe_seq_create(pe_cache *c, int32_t *seq_out)
 pe_status pe_seq_release(pe_cache *c, int32_t seq, void *stream)
 {
     std::vector<CropPlan> pl(1);
-    pe_status s = plan_crop(c, seq, 1, &pl[0]);
+    pe_status s = check_device(c);
+    if (s != PE_OK) return s;
+    s = plan_crop(c, seq, 1, &pl[0]);
     if (s != PE_OK) return s;
     CallTxn tx(c, static_cast<cudaStream_t>(stream));
     apply_crop(c, pl[0], nullptr);
@@ -1439,6 +1463,7 @@ pe_status pe_seq_fork(pe_cache *c, int32_t seq, int32_t *new_seq, void *stream)
 {
     pe_status s = check_seq(c, seq);
     if (s != PE_OK) return s;
+    if ((s = check_device(c)) != PE_OK) return s;
     if (!new_seq) return fail(PE_ERR_INVALID, "null new_seq");
     int32_t ns = -1;
     for (int32_t q = 0; q < c->cfg.max_seqs; ++q)
@@ -1528,7 +1553,9 @@ pe_status pe_crop(pe_cache *c, int32_t seq, int64_t tau, int32_t *freed_out, int
                   void *stream)
 {
     std::vector<CropPlan> pl(1);
-    pe_status s = plan_crop(c, seq, tau, &pl[0]);
+    pe_status s = check_device(c);
+    if (s != PE_OK) return s;
+    s = plan_crop(c, seq, tau, &pl[0]);
     if (s != PE_OK) return s;
     const int32_t nf = pl[0].n_freed;
     if (freed_out && freed_cap < nf) return fail(PE_ERR_RANGE, "freed_cap %d < %d freed pages", freed_cap, nf);
@@ -1541,7 +1568,7 @@ pe_status pe_crop(pe_cache *c, int32_t seq, int64_t tau, int32_t *freed_out, int
 
 pe_status pe_crop_batch(pe_cache *c, int32_t n, const int32_t *seqs, const int64_t *taus, void *stream)
 {
-    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (pe_status s = check_device(c)) return s;
     if (n < 0 || (n > 0 && (!seqs || !taus))) return fail(PE_ERR_INVALID, "bad batch arguments");
     std::vector<CropPlan> plans(n);
     std::vector<uint8_t> seen(c->cfg.max_seqs, 0);
@@ -1559,8 +1586,9 @@ pe_status pe_crop_batch(pe_cache *c, int32_t n, const int32_t *seqs, const int64
 pe_status pe_append_kv(pe_cache *c, int32_t seq, const void *K, const void *V, int32_t n_tokens, void *stream)
 {
     AppendPlan pl{};
-    pe_status s = plan_append(c, seq, n_tokens, &pl);
+    pe_status s = check_device(c);
     if (s != PE_OK) return s;
+    if ((s = plan_append(c, seq, n_tokens, &pl)) != PE_OK) return s;
     if (!c->host_only && n_tokens > 0) {
         if (!K || !V) return fail(PE_ERR_INVALID, "null K or V");
         if (!aligned16(K) || !aligned16(V)) return fail(PE_ERR_INVALID, "K and V must be 16-byte aligned");
@@ -1575,7 +1603,7 @@ pe_status pe_append_kv(pe_cache *c, int32_t seq, const void *K, const void *V, i
 pe_status pe_append_kv_batch(pe_cache *c, int32_t n, const int32_t *seqs, const void *K, const void *V,
                              const int32_t *cu_tokens, void *stream)
 {
-    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (pe_status s = check_device(c)) return s;
     if (n < 0 || (n > 0 && (!seqs || !cu_tokens))) return fail(PE_ERR_INVALID, "bad batch arguments");
     if (n > 0 && cu_tokens[0] != 0) return fail(PE_ERR_INVALID, "cu_tokens[0] must be 0");
     std::vector<AppendPlan> plans(n);
@@ -1645,7 +1673,7 @@ pe_status pe_replay_rounds(pe_cache *c, int32_t n, const int32_t *seqs, int32_t 
                            const int32_t *cu_tok, const void *K, const void *V, const void *Q, void *out,
                            int32_t num_q_heads, float softmax_scale, void *stream)
 {
-    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (pe_status s = check_device(c)) return s;
     if (n < 0 || n_rounds < 0 || (n > 0 && (!seqs || !cu_tok)) || (n > 0 && n_rounds > 0 && !take))
         return fail(PE_ERR_INVALID, "bad rounds arguments");
     if (n == 0) return PE_OK;
@@ -1840,6 +1868,7 @@ pe_status pe_seq_device_page_table(pe_cache *c, int32_t seq, int32_t *out, int32
     pe_status s = check_seq(c, seq);
     if (s != PE_OK) return s;
     if (c->host_only) return fail(PE_ERR_UNSUPPORTED, "host-only cache has no device table");
+    if ((s = check_device(c)) != PE_OK) return s;
     if (!out || cap < 0 || cap > c->cfg.max_pages_per_seq) return fail(PE_ERR_INVALID, "bad output buffer");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaStreamSynchronize(st);
@@ -1897,6 +1926,7 @@ pe_status pe_selftest_bounded_wait(pe_cache *c, int64_t limit_ns, void *stream)
 {
     if (!c) return fail(PE_ERR_INVALID, "null cache");
     if (c->host_only) return fail(PE_ERR_UNSUPPORTED, "host-only cache has no device");
+    if (pe_status s = check_device(c)) return s;
     if (limit_ns < 1000 || limit_ns > 2000000000ll) return fail(PE_ERR_RANGE, "limit_ns must be in [1 us, 2 s]");
     cudaError_t e = launch_bounded_wait_selftest(c->d_status, static_cast<uint64_t>(limit_ns),
                                                  static_cast<cudaStream_t>(stream));
@@ -1926,6 +1956,7 @@ pe_status pe_device_status(pe_cache *c, int32_t *code, int32_t clear, void *stre
     if (!c || !code) return fail(PE_ERR_INVALID, "null argument");
     *code = 0;
     if (c->host_only) return PE_OK;
+    if (pe_status s = check_device(c)) return s;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaStreamSynchronize(st);
     if (e == cudaSuccess) e = cudaMemcpy(code, c->d_status, sizeof(int32_t), cudaMemcpyDeviceToHost);

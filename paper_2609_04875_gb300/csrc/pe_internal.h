@@ -2,6 +2,7 @@
 // (pe_host.cu) and the kernels (pe_kv.cu, pe_attn.cu).
 #pragma once
 
+#include <atomic>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -208,6 +209,23 @@ cudaError_t launch_replay_attn_sk(int head_dim, const CUtensorMap &tm_q, const C
 cudaError_t launch_decode_attn(int head_dim, int rows_cap, bool tensor_core, const CUtensorMap &tm_k,
                                const CUtensorMap &tm_v, const DecodeParams &p, cudaStream_t st);
 cudaError_t launch_bounded_wait_selftest(int32_t *status, uint64_t limit_ns, cudaStream_t st);
+
+// Raises `kernel`'s dynamic shared-memory limit to `bytes` on the current
+// device, once per device: the attribute is set on the device that is current
+// at the call, so a process that runs caches on several GPUs sets it on each.
+// `done` holds one bit per device (devices past 63 set it on every call).
+template <typename Kernel>
+inline cudaError_t set_dyn_smem_once(Kernel kernel, int bytes, std::atomic<uint64_t> &done)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = (dev >= 0 && dev < 64) ? (1ull << dev) : 0;
+    if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_acq_rel);
+    return e;
+}
 
 // Fixed split-KV scratch compiled into the library (pe_attn.cu), used only by
 // pe_replay_attn_static_scratch.  static_scratch() returns its device address

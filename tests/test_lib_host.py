@@ -286,3 +286,42 @@ def test_random_fork_ops_match_oracle(ps):
             assert lib.page_table(q) == orc.page_table(q), f"step {step}"
             assert lib.seq_info(q) == orc.seq_info(q), f"step {step}"
             assert lib.checkpoints(q) == orc.checkpoints[q], f"step {step}"
+
+
+def test_binding_rejects_mismatched_out_before_any_device_call():
+    """An `out` of another shape than Q would let the kernels write past its
+    end; the binding refuses it before reaching the library (checked here on a
+    host-only cache with CPU tensors, so nothing is launched)."""
+    import torch
+    c = pe.PagedKVCache(1, 2, 64, 8, 16, 2, 16, host_only=True)
+    s = c.seq_create()
+    c.append_kv(s, n_tokens=20)
+    q = torch.zeros(4, 4, 64, dtype=torch.bfloat16)
+    short = torch.zeros(3, 4, 64, dtype=torch.bfloat16)
+    for call in (lambda: c.replay_attn(s, 0, q, out=short),
+                 lambda: c.replay_attn_static_scratch(s, 0, q, out=short),
+                 lambda: c.replay_attn_batch([s], 0, q, [0, 4], out=short)):
+        with pytest.raises(ValueError, match="must match"):
+            call()
+    c.close()
+
+
+def test_binding_rejects_tensors_off_the_cache_device():
+    """Tensors must live on the cache's device; the check runs before the
+    pointer is handed to the library."""
+    class FakeCuda:
+        dtype = __import__("torch").bfloat16
+        is_cuda = True
+
+        class device:
+            index = 1
+
+        def is_contiguous(self):
+            return True
+
+        def data_ptr(self):
+            return 0
+
+    with pytest.raises(ValueError, match="cuda:1, the cache on cuda:0"):
+        binding._dev_ptr(FakeCuda(), "Q", 0)
+    assert binding._dev_ptr(FakeCuda(), "Q", 1).value is None  # same device: accepted
