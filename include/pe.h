@@ -306,6 +306,40 @@ pe_status pe_selftest_bounded_wait(pe_cache *cache, int64_t limit_ns, void *stre
  * in a second, split-KV launch), ctas = attention CTAs launched in all. */
 pe_status pe_last_attn_plan(const pe_cache *cache, int32_t *split, int32_t *n_splits, int32_t *ctas);
 
+/* The persistent prefill kernel's work plan for one launch group, made by the
+ * same host planner an attention call runs when it takes that kernel
+ * ("attn_kernel" = 2), without any device work; host-only caches too.  It
+ * lets a caller (or a test) check on the host that the plan covers every key
+ * tile once.  The group is sequences seqs[0..n) (1 <= n <= 64, live, distinct)
+ * whose queries are their last cu_q[i+1] - cu_q[i] positions (cu_q host [n+1],
+ * from 0; each count in [1, len]), with num_q_heads as in pe_replay_attn; the
+ * planner orders them longest first (ties in the given order).  num_sms: the
+ * SM count to plan for, 1..160 (0 = the cache's device; required for a
+ * host-only cache).  The split partials are sized against the cache's
+ * workspace_bytes.  A unit is (sequence, kv-head, pair of 128-row q-tiles):
+ * sequences in planning order, then pairs heaviest (latest queries) first,
+ * kv-heads fastest; its key tiles are the 128-key tiles its later q-tile sees.
+ * The kernel's CTA k first takes whole units in `rounds` lockstep rounds (in
+ * round r the unit r*n_ctas + k, or r*n_ctas + n_ctas-1-k when r is odd), then
+ * its tail stretch: from key tile t0 of unit u0 up to key tile t1 of unit u1
+ * (t1 = 0: up to the start of u1), or nothing when u0 > u1.  A cut unit's
+ * pieces are its parts, written as fp32 partials and merged in the kernel.
+ * Outputs (host):
+ *   info[5] (required): n_ctas, rounds, n_slots (cut units), max_parts, n_units;
+ *   order_out[n] (nullable): the sequences in planning order;
+ *   unit_tiles[units_cap] (nullable): each unit's key tiles;
+ *   ctas[ctas_cap][8] (nullable): per CTA u0, t0, u1, t1, slot0, part0, slot1,
+ *     part1 -- the partial slot and part of the stretch's first and last
+ *     piece (slot -1: that piece is a whole unit, written directly);
+ *   slots[slots_cap][2] (nullable): per cut unit its unit and part count.
+ * Errors: INVALID, UNSUPPORTED (group size), RANGE (a cap below the plan's
+ * size; info is written first).  The paper has no counterpart: this plans the
+ * build's own kernel. */
+pe_status pe_attn_plan_persistent(pe_cache *cache, int32_t n, const int32_t *seqs, const int32_t *cu_q,
+                                  int32_t num_q_heads, int32_t num_sms, int32_t *info, int32_t *order_out,
+                                  int32_t *unit_tiles, int32_t units_cap, int32_t *ctas, int32_t ctas_cap,
+                                  int32_t *slots, int32_t slots_cap);
+
 /* Number of kernel launches this cache has made so far (crop, append,
  * attention, combine); lets a caller count its device work. */
 pe_status pe_kernel_launches(const pe_cache *cache, int64_t *count);

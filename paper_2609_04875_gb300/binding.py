@@ -31,7 +31,7 @@ EXPORTED = [
     "pe_last_attn_plan", "pe_seq_fork", "pe_checkpoint_add", "pe_checkpoint_select", "pe_restore",
     "pe_seq_checkpoints", "pe_page_refs", "pe_prov_create", "pe_prov_destroy", "pe_prov_add",
     "pe_prov_locate_source", "pe_prov_taint_closure", "pe_prov_first_entry", "pe_replay_schedule",
-    "pe_replay_rounds", "pe_last_error", "pe_version",
+    "pe_replay_rounds", "pe_attn_plan_persistent", "pe_last_error", "pe_version",
 ]
 
 # Turn kinds and replay policies of pe_replay_schedule (pe.h).
@@ -98,6 +98,8 @@ _sigs = {
     "pe_replay_attn_static_scratch": [_P, _I32, _I32, _P, _P, _I32, _I32, ctypes.c_float, _P],
     "pe_replay_schedule": [_I32, _I32P, _I32P, _I32P, _I32, _I32P, _I64, _I32P, _I64P],
     "pe_replay_rounds": [_P, _I32, _I32P, _I32, _I32P, _I32P, _P, _P, _P, _P, _I32, ctypes.c_float, _P],
+    "pe_attn_plan_persistent": [_P, _I32, _I32P, _I32P, _I32, _I32, _I32P, _I32P, _I32P, _I32, _I32P, _I32,
+                                _I32P, _I32],
 }
 for _name, _args in _sigs.items():
     _fn = getattr(_lib, _name)
@@ -514,6 +516,29 @@ class PagedKVCache:
         a, b, c = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
         _check(_lib.pe_last_attn_plan(self._h, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
         return bool(a.value), b.value, c.value
+
+    def plan_persistent(self, seqs, n_q, num_q_heads, num_sms=0):
+        """pe_attn_plan_persistent: the persistent kernel's plan for the group
+        (sequence i attends its last n_q[i] positions), made on the host.
+        Returns a dict: n_ctas, rounds, n_slots, max_parts, order (sequences in
+        planning order), unit_tiles, ctas (rows u0, t0, u1, t1, slot0, part0,
+        slot1, part1) and slots (rows unit, n_parts)."""
+        cu = [0]
+        for q in n_q:
+            cu.append(cu[-1] + int(q))
+        info = (ctypes.c_int32 * 5)()
+        order = (ctypes.c_int32 * max(1, len(seqs)))()
+        args = (self._h, len(seqs), _i32_array(seqs), _i32_array(cu), int(num_q_heads), int(num_sms), info, order)
+        _check(_lib.pe_attn_plan_persistent(*args, None, 0, None, 0, None, 0))
+        n_ctas, rounds, n_slots, max_parts, n_units = list(info)
+        tiles = (ctypes.c_int32 * max(1, n_units))()
+        ctas = (ctypes.c_int32 * max(1, 8 * n_ctas))()
+        slots = (ctypes.c_int32 * max(1, 2 * n_slots))()
+        _check(_lib.pe_attn_plan_persistent(*args, tiles, n_units, ctas, n_ctas, slots, n_slots))
+        return {"n_ctas": n_ctas, "rounds": rounds, "n_slots": n_slots, "max_parts": max_parts,
+                "order": list(order[: len(seqs)]), "unit_tiles": list(tiles[:n_units]),
+                "ctas": [list(ctas[8 * k: 8 * k + 8]) for k in range(n_ctas)],
+                "slots": [list(slots[2 * k: 2 * k + 2]) for k in range(n_slots)]}
 
     def kernel_launches(self) -> int:
         n = ctypes.c_int64()

@@ -813,7 +813,7 @@ struct SkBound {
 };
 
 pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, size_t hi, int32_t layer, void *out,
-                  int32_t hq, float scale, SkParams &P)
+                  int32_t hq, float scale, SkParams &P, std::vector<int32_t> *unit_tiles = nullptr)
 {
     const pe_cache_config &cf = c->cfg;
     const int hkv = cf.num_kv_heads, d = cf.head_dim, g = hq / hkv, bmq = kBM / g;
@@ -965,10 +965,10 @@ pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, si
     if (cuts) {
         for (int32_t u = 0; u < U; ++u)
             if (slot_of[u] >= 0) P.slots[slot_of[u]] = SkSlot{u, cuts_in[slot_of[u]] + 1};
-        p.part_o = c->d_ws;
-        p.part_lse = c->d_ws + static_cast<int64_t>(n_slots) * max_parts * 2 * kBM * d;
+        p.part_o = c->d_ws;  // (null on a host-only cache, which only plans)
+        p.part_lse = c->d_ws ? c->d_ws + static_cast<int64_t>(n_slots) * max_parts * 2 * kBM * d : nullptr;
     }
-    P.tickets = c->d_tickets + kMaxSegs * hkv + 2;
+    P.tickets = c->d_tickets ? c->d_tickets + kMaxSegs * hkv + 2 : nullptr;
     for (int32_t k = 0; k < pl.nc; ++k) {
         const SkBound &a = pl.b[k], &z = pl.b[k + 1];
         SkCta &w = P.cta[k];
@@ -998,6 +998,7 @@ pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, si
             w.part1 = 0;
         }
     }
+    if (unit_tiles) *unit_tiles = n_all;
     return PE_OK;
 }
 
@@ -1350,6 +1351,7 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
     cc->refs.assign(c.num_pages, 0);
     cc->ckpt.resize(c.max_seqs);
     cc->pool_rows = pool_rows;
+    cc->ws_bytes = c.workspace_bytes > 0 ? c.workspace_bytes : (256ll << 20);  // (also sizes host-only plans)
     if (cc->host_only) {
         *out = cc;
         return PE_OK;
@@ -1370,7 +1372,6 @@ pe_status pe_cache_create(const pe_cache_config *cfg, pe_cache **out)
     }
     const size_t pool_bytes = static_cast<size_t>(pool_rows) * c.head_dim * 2;
     const size_t table_bytes = static_cast<size_t>(c.max_seqs) * c.max_pages_per_seq * sizeof(int32_t);
-    cc->ws_bytes = c.workspace_bytes > 0 ? c.workspace_bytes : (256ll << 20);
     pe_status st = PE_OK;
     do {
         if (c.k_pool) {
@@ -1941,6 +1942,70 @@ pe_status pe_last_attn_plan(const pe_cache *c, int32_t *split, int32_t *n_splits
     if (split) *split = c->last_split;
     if (n_splits) *n_splits = c->last_splits;
     if (ctas) *ctas = c->last_ctas;
+    return PE_OK;
+}
+
+pe_status pe_attn_plan_persistent(pe_cache *c, int32_t n, const int32_t *seqs, const int32_t *cu_q,
+                                  int32_t num_q_heads, int32_t num_sms, int32_t *info, int32_t *order_out,
+                                  int32_t *unit_tiles, int32_t units_cap, int32_t *ctas, int32_t ctas_cap,
+                                  int32_t *slots, int32_t slots_cap)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (n < 1 || n > kMaxSegs || !seqs || !cu_q || !info) return fail(PE_ERR_INVALID, "bad plan arguments");
+    if (cu_q[0] != 0) return fail(PE_ERR_INVALID, "cu_q[0] must be 0");
+    const int32_t hkv = c->cfg.num_kv_heads;
+    if (num_q_heads <= 0 || num_q_heads % hkv != 0)
+        return fail(PE_ERR_INVALID, "num_q_heads %d is not a multiple of num_kv_heads %d", num_q_heads, hkv);
+    const int32_t g = num_q_heads / hkv;
+    if (g > kBM || (g & (g - 1)) != 0) return fail(PE_ERR_UNSUPPORTED, "group size %d must be a power of two <= %d", g, kBM);
+    if (num_sms < 0 || num_sms > kMaxSkCtas) return fail(PE_ERR_RANGE, "num_sms must be 0..%d", kMaxSkCtas);
+    if (num_sms == 0 && c->host_only) return fail(PE_ERR_INVALID, "a host-only cache has no SM count: give num_sms");
+    std::vector<AttnItem> order;
+    std::vector<uint8_t> seen(c->cfg.max_seqs, 0);
+    for (int32_t i = 0; i < n; ++i) {
+        pe_status s = check_seq(c, seqs[i]);
+        if (s != PE_OK) return s;
+        if (seen[seqs[i]]) return fail(PE_ERR_INVALID, "sequence %d appears twice", seqs[i]);
+        seen[seqs[i]] = 1;
+        const int32_t nq = cu_q[i + 1] - cu_q[i];
+        if (nq < 1 || nq > c->len[seqs[i]])
+            return fail(PE_ERR_RANGE, "sequence %d: n_q = %d outside [1, %lld]", seqs[i], nq,
+                        static_cast<long long>(c->len[seqs[i]]));
+        order.push_back(AttnItem{seqs[i], cu_q[i], nq});
+    }
+    // the attention call's order: longest sequence first, ties in call order
+    std::stable_sort(order.begin(), order.end(),
+                     [&](const AttnItem &a, const AttnItem &b) { return c->len[a.seq] > c->len[b.seq]; });
+    std::vector<char> buf(sizeof(SkParams));
+    SkParams &P = *reinterpret_cast<SkParams *>(buf.data());
+    std::vector<int32_t> tiles;
+    const int saved_sms = c->num_sms;
+    if (num_sms > 0) c->num_sms = num_sms;
+    const pe_status s = plan_sk(c, order, 0, order.size(), 0, nullptr, num_q_heads, 1.0f, P, &tiles);
+    c->num_sms = saved_sms;
+    if (s != PE_OK) return s;
+    const int32_t n_units = static_cast<int32_t>(tiles.size());
+    info[0] = P.n_ctas;
+    info[1] = P.rounds;
+    info[2] = P.n_slots;
+    info[3] = P.max_parts;
+    info[4] = n_units;
+    if (order_out)
+        for (size_t i = 0; i < order.size(); ++i) order_out[i] = order[i].seq;
+    if ((unit_tiles && units_cap < n_units) || (ctas && ctas_cap < P.n_ctas) || (slots && slots_cap < P.n_slots))
+        return fail(PE_ERR_RANGE, "plan needs %d units, %d CTAs, %d slots", n_units, P.n_ctas, P.n_slots);
+    if (unit_tiles) std::copy(tiles.begin(), tiles.end(), unit_tiles);
+    if (ctas)
+        for (int32_t k = 0; k < P.n_ctas; ++k) {
+            const SkCta &w = P.cta[k];
+            const int32_t row[8] = {w.u0, w.t0, w.u1, w.t1, w.slot0, w.part0, w.slot1, w.part1};
+            std::copy(row, row + 8, ctas + 8 * k);
+        }
+    if (slots)
+        for (int32_t k = 0; k < P.n_slots; ++k) {
+            slots[2 * k] = P.slots[k].unit;
+            slots[2 * k + 1] = P.slots[k].n_parts;
+        }
     return PE_OK;
 }
 
