@@ -340,6 +340,38 @@ pe_status pe_attn_plan_persistent(pe_cache *cache, int32_t n, const int32_t *seq
                                   int32_t *unit_tiles, int32_t units_cap, int32_t *ctas, int32_t ctas_cap,
                                   int32_t *slots, int32_t slots_cap);
 
+/* Every launch an attention call would make for this batch (the arguments of
+ * pe_replay_attn_batch without tensors), planned by the same host code with
+ * no device work and no change to the cache; host-only caches too.  It lets a
+ * caller (or a test) check the plans on the host.  A sequence with no queries
+ * takes no launch.  num_sms as in pe_attn_plan_persistent.  The launches are written to words[cap] (host,
+ * nullable: call with NULL to learn *n_words, required) one after another,
+ * each as 7 + 10 * n_seqs int64 words:
+ *   kind (0: the one-item prefill kernel; 1: its split-KV tail launch, over
+ *     pairs [0, pair_top) of its one sequence; 2: the persistent kernel, see
+ *     pe_attn_plan_persistent; 3: sequences the decode kernel takes, not
+ *     planned further), split (partials merged by a combine launch, or cut
+ *     units for kind 2), CTAs, combine rows, split_tiles (128-key tiles per
+ *     split), pairs_fastest (the one-item kernel's CTA order), n_seqs;
+ *   then per sequence: seq, item0 (its first CTA), n_q, n_keys, n_qtiles,
+ *     n_splits, pair_top, part_row0 (its first partial row), comb0 (its first
+ *     combine row), q_row0 (its first row of Q and out).
+ * A one-item launch's CTA b works on sequence i with item0_i <= b < item0_{i+1}
+ * (the last: CTAs), local = b - item0_i; with pairs_fastest, pair = pair_top -
+ * 1 - local % P (P = that sequence's CTAs / (Hkv x n_splits)), split = (local
+ * / P) % n_splits, kv-head = local / P / n_splits; else kv-head = local % Hkv,
+ * split = (local / Hkv) % n_splits, pair = pair_top - 1 - local / Hkv /
+ * n_splits.  It computes q-tiles 2 pair and 2 pair + 1 (those below n_qtiles)
+ * over key tiles [split x split_tiles, +split_tiles); a split launch writes
+ * partial row part_row0 + ((q-tile x Hkv + kv-head) x n_splits + split) x 128
+ * + r for row r, and its combine merges, for each of its combine rows
+ * comb0 + (q-tile x Hkv + kv-head) x 128 + r, the n_splits rows from there.
+ * Errors: INVALID, RANGE (cap below *n_words, n_q > len), UNSUPPORTED.  The
+ * paper has no counterpart: this plans the build's own kernels. */
+pe_status pe_attn_plan_launches(pe_cache *cache, int32_t n, const int32_t *seqs, const int32_t *cu_q,
+                                int32_t num_q_heads, int32_t num_sms, int64_t *words, int64_t cap,
+                                int64_t *n_words);
+
 /* Number of kernel launches this cache has made so far (crop, append,
  * attention, combine); lets a caller count its device work. */
 pe_status pe_kernel_launches(const pe_cache *cache, int64_t *count);

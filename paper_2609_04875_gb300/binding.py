@@ -31,7 +31,7 @@ EXPORTED = [
     "pe_last_attn_plan", "pe_seq_fork", "pe_checkpoint_add", "pe_checkpoint_select", "pe_restore",
     "pe_seq_checkpoints", "pe_page_refs", "pe_prov_create", "pe_prov_destroy", "pe_prov_add",
     "pe_prov_locate_source", "pe_prov_taint_closure", "pe_prov_first_entry", "pe_replay_schedule",
-    "pe_replay_rounds", "pe_attn_plan_persistent", "pe_last_error", "pe_version",
+    "pe_replay_rounds", "pe_attn_plan_persistent", "pe_attn_plan_launches", "pe_last_error", "pe_version",
 ]
 
 # Turn kinds and replay policies of pe_replay_schedule (pe.h).
@@ -100,6 +100,7 @@ _sigs = {
     "pe_replay_rounds": [_P, _I32, _I32P, _I32, _I32P, _I32P, _P, _P, _P, _P, _I32, ctypes.c_float, _P],
     "pe_attn_plan_persistent": [_P, _I32, _I32P, _I32P, _I32, _I32, _I32P, _I32P, _I32P, _I32, _I32P, _I32,
                                 _I32P, _I32],
+    "pe_attn_plan_launches": [_P, _I32, _I32P, _I32P, _I32, _I32, _I64P, _I64, _I64P],
 }
 for _name, _args in _sigs.items():
     _fn = getattr(_lib, _name)
@@ -539,6 +540,34 @@ class PagedKVCache:
                 "order": list(order[: len(seqs)]), "unit_tiles": list(tiles[:n_units]),
                 "ctas": [list(ctas[8 * k: 8 * k + 8]) for k in range(n_ctas)],
                 "slots": [list(slots[2 * k: 2 * k + 2]) for k in range(n_slots)]}
+
+    LAUNCH_KINDS = {0: "one_item", 1: "one_item_tail", 2: "persistent", 3: "decode"}
+    _SEQ_FIELDS = ("seq", "item0", "n_q", "n_keys", "n_qtiles", "n_splits", "pair_top", "part_row0", "comb0",
+                   "q_row0")
+
+    def plan_launches(self, seqs, n_q, num_q_heads, num_sms=0):
+        """pe_attn_plan_launches: the launches an attention call over these
+        sequences (each attending its last n_q[i] positions) would make, planned
+        on the host.  A list of dicts: kind, split, ctas, combine_rows,
+        split_tiles, pairs_fastest and seqs (one dict per sequence)."""
+        cu = [0]
+        for q in n_q:
+            cu.append(cu[-1] + int(q))
+        n_words = ctypes.c_int64()
+        args = (self._h, len(seqs), _i32_array(seqs), _i32_array(cu), int(num_q_heads), int(num_sms))
+        _check(_lib.pe_attn_plan_launches(*args, None, 0, ctypes.byref(n_words)))
+        buf = (ctypes.c_int64 * max(1, n_words.value))()
+        _check(_lib.pe_attn_plan_launches(*args, buf, n_words.value, ctypes.byref(n_words)))
+        words, out, i = list(buf[: n_words.value]), [], 0
+        while i < len(words):
+            kind, split, ctas, comb, split_tiles, pairs_fastest, n = words[i: i + 7]
+            i += 7
+            rows = [dict(zip(self._SEQ_FIELDS, words[i + 10 * k: i + 10 * k + 10])) for k in range(n)]
+            i += 10 * n
+            out.append({"kind": self.LAUNCH_KINDS[kind], "split": bool(split), "ctas": ctas,
+                        "combine_rows": comb, "split_tiles": split_tiles, "pairs_fastest": bool(pairs_fastest),
+                        "seqs": rows})
+        return out
 
     def kernel_launches(self) -> int:
         n = ctypes.c_int64()

@@ -133,6 +133,7 @@ struct pe_cache {
     int64_t launches = 0;
     int32_t last_split = 0, last_splits = 0, last_ctas = 0;  // plan of the last attention launch
     Journal jr;                   // changes of the call in progress
+    std::vector<int64_t> *plan_rec = nullptr;  // set only inside pe_attn_plan_launches: record, do not launch
     int64_t fail_after = -1;      // test hook "fail_launch_after": device steps left before an injected failure
 };
 
@@ -1002,6 +1003,23 @@ pe_status plan_sk(pe_cache *c, const std::vector<AttnItem> &order, size_t lo, si
     return PE_OK;
 }
 
+// Plan query (pe_attn_plan_launches): one launch as words -- kind, split,
+// CTAs, combine rows, split_tiles, pairs_fastest, n_seqs, then per sequence
+// seq, item0, n_q, n_keys, n_qtiles, n_splits, pair_top, part_row0, comb0,
+// q_row0.
+void record_launch(const pe_cache *c, int32_t kind, bool split, const AttnParams &p, int32_t ctas)
+{
+    std::vector<int64_t> &r = *c->plan_rec;
+    const int64_t head[7] = {kind, split ? 1 : 0, ctas, p.total_comb, p.split_tiles, p.pairs_fastest, p.n_seqs};
+    r.insert(r.end(), head, head + 7);
+    for (int32_t i = 0; i < p.n_seqs; ++i) {
+        const AttnSeq &q = p.seqs[i];
+        const int64_t w[10] = {q.table_row / c->cfg.max_pages_per_seq, q.item0, q.n_q, q.n_keys, q.n_qtiles,
+                               q.n_splits, q.pair_top, q.part_row0, q.comb0, q.q_row0};
+        r.insert(r.end(), w, w + 10);
+    }
+}
+
 pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t layer, const void *Q,
                         int64_t q_rows, void *out, int32_t hq, float scale, cudaStream_t st)
 {
@@ -1022,7 +1040,21 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         else
             order.push_back(it);
     }
-    if (!dec.empty()) {
+    if (!dec.empty() && c->plan_rec) {  // plan query: the decode kernel's sequences, not planned here
+        std::vector<char> dbuf(sizeof(AttnParams));
+        AttnParams &dp = *reinterpret_cast<AttnParams *>(dbuf.data());
+        for (size_t lo = 0; lo < dec.size(); lo += kMaxSegs) {
+            std::memset(&dp, 0, sizeof dp);
+            for (size_t i = lo; i < std::min(dec.size(), lo + kMaxSegs); ++i) {
+                AttnSeq &q = dp.seqs[dp.n_seqs++];
+                q.table_row = dec[i].seq * cf.max_pages_per_seq;
+                q.n_q = dec[i].n_q;
+                q.n_keys = static_cast<int32_t>(c->len[dec[i].seq]);
+                q.q_row0 = dec[i].q_row0;
+            }
+            record_launch(c, 3, false, dp, 0);
+        }
+    } else if (!dec.empty()) {
         pe_status s = run_decode(c, dec, layer, Q, out, hq, scale, st);
         if (s != PE_OK) return s;
     }
@@ -1032,9 +1064,10 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
     if (order.empty()) return PE_OK;
 
     CUtensorMap tm_q, tm_o;  // Q, and the output as a map of the same shape (TMA stores of full q-tiles)
-    pe_status s = encode_q(&tm_q, Q, q_rows, hq, d, g);
-    if (s != PE_OK) return s;
-    if ((s = encode_q(&tm_o, out, q_rows, hq, d, g)) != PE_OK) return s;
+    const bool rec = c->plan_rec != nullptr;  // a plan query: no tensors, no launches
+    pe_status s = PE_OK;
+    if (!rec && (s = encode_q(&tm_q, Q, q_rows, hq, d, g)) != PE_OK) return s;
+    if (!rec && (s = encode_q(&tm_o, out, q_rows, hq, d, g)) != PE_OK) return s;
 
     // split-KV decision over the whole launch group; plan_est: the cost model's time of the plan
     double plan_est = 0.0;
@@ -1139,7 +1172,7 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             const int64_t need = prow * (static_cast<int64_t>(d) * 4 + 4);
             if (need <= c->ws_bytes) {
                 p.part_o = c->d_ws;
-                p.part_lse = c->d_ws + prow * d;
+                p.part_lse = c->d_ws ? c->d_ws + prow * d : nullptr;  // (null on a host-only cache)
                 break;
             }
             if (split_tiles >= max_tiles) {
@@ -1226,6 +1259,10 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             c->last_split = P.n_slots > 0 ? 1 : 0;
             c->last_splits = P.max_parts;
             c->last_ctas = P.n_ctas;
+            if (rec) {
+                record_launch(c, 2, P.n_slots > 0, P.a, P.n_ctas);
+                continue;
+            }
             if (injected_failure(c)) return launch_fault("replay attention");
             cudaError_t e = launch_replay_attn_sk(d, tm_q, c->tm_k, c->tm_v, P, st);
             if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
@@ -1244,11 +1281,12 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
         c->last_split = split || tail ? 1 : 0;
         c->last_splits = tail ? static_cast<int32_t>(tp.splits) : (split ? p.seqs[0].n_splits : 1);
         c->last_ctas = p.total_items + (tail ? static_cast<int32_t>(tp.pairs * hkv * tp.splits) : 0);
+        if (rec) record_launch(c, 0, split, p, p.total_items);
         if (injected_failure(c)) return launch_fault("replay attention");
-        cudaError_t e = launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, tm_o, p, st);
+        cudaError_t e = rec ? cudaSuccess : launch_replay_attn(d, split, tm_q, c->tm_k, c->tm_v, tm_o, p, st);
         if (e != cudaSuccess) return cuda_fail(e, "replay attention launch");
-        c->launches++;
-        if (split) {
+        if (!rec) c->launches++;
+        if (split && !rec) {
             if (injected_failure(c)) return launch_fault("split-KV combine");
             e = launch_splitkv_combine(d, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "split-KV combine launch");
@@ -1267,7 +1305,11 @@ pe_status run_attention(pe_cache *c, const std::vector<AttnItem> &items, int32_t
             p.total_comb = static_cast<int32_t>(tp.qtiles * hkv * kBM);  // q-tiles [0, 2 cut)
             p.pairs_fastest = c->attn_order > 0 ? 1 : 0;
             p.part_o = c->d_ws;
-            p.part_lse = c->d_ws + tp.qtiles * hkv * tp.splits * kBM * d;
+            p.part_lse = c->d_ws ? c->d_ws + tp.qtiles * hkv * tp.splits * kBM * d : nullptr;
+            if (rec) {
+                record_launch(c, 1, true, p, p.total_items);
+                continue;
+            }
             if (injected_failure(c)) return launch_fault("replay attention tail");
             e = launch_replay_attn(d, true, tm_q, c->tm_k, c->tm_v, tm_q, p, st);
             if (e != cudaSuccess) return cuda_fail(e, "replay attention tail launch");
@@ -2006,6 +2048,55 @@ pe_status pe_attn_plan_persistent(pe_cache *c, int32_t n, const int32_t *seqs, c
             slots[2 * k] = P.slots[k].unit;
             slots[2 * k + 1] = P.slots[k].n_parts;
         }
+    return PE_OK;
+}
+
+pe_status pe_attn_plan_launches(pe_cache *c, int32_t n, const int32_t *seqs, const int32_t *cu_q, int32_t num_q_heads,
+                                int32_t num_sms, int64_t *words, int64_t cap, int64_t *n_words)
+{
+    if (!c) return fail(PE_ERR_INVALID, "null cache");
+    if (n < 1 || !seqs || !cu_q || !n_words) return fail(PE_ERR_INVALID, "bad plan arguments");
+    if (cu_q[0] != 0) return fail(PE_ERR_INVALID, "cu_q[0] must be 0");
+    const int32_t hkv = c->cfg.num_kv_heads;
+    if (num_q_heads <= 0 || num_q_heads % hkv != 0)
+        return fail(PE_ERR_INVALID, "num_q_heads %d is not a multiple of num_kv_heads %d", num_q_heads, hkv);
+    const int32_t g = num_q_heads / hkv;
+    if (g > kBM || (g & (g - 1)) != 0) return fail(PE_ERR_UNSUPPORTED, "group size %d must be a power of two <= %d", g, kBM);
+    if (num_sms < 0 || num_sms > kMaxSkCtas) return fail(PE_ERR_RANGE, "num_sms must be 0..%d", kMaxSkCtas);
+    if (num_sms == 0 && c->host_only) return fail(PE_ERR_INVALID, "a host-only cache has no SM count: give num_sms");
+    std::vector<AttnItem> items(n);
+    for (int32_t i = 0; i < n; ++i) {
+        pe_status s = check_seq(c, seqs[i]);
+        if (s != PE_OK) return s;
+        const int32_t nq = cu_q[i + 1] - cu_q[i];
+        if (nq < 0) return fail(PE_ERR_INVALID, "cu_q must be non-decreasing");
+        if (nq > c->len[seqs[i]])
+            return fail(PE_ERR_RANGE, "sequence %d: n_q = %d exceeds its length %lld", seqs[i], nq,
+                        static_cast<long long>(c->len[seqs[i]]));
+        items[i] = AttnItem{seqs[i], cu_q[i], nq};
+    }
+    // plan as an attention call would, recording instead of launching; nothing of the cache changes
+    std::vector<int64_t> rec;
+    const int saved_sms = c->num_sms;
+    const int64_t saved_fail = c->fail_after;
+    const int32_t saved_plan[3] = {c->last_split, c->last_splits, c->last_ctas};
+    if (num_sms > 0) c->num_sms = num_sms;
+    c->fail_after = -1;
+    c->plan_rec = &rec;
+    const pe_status s = run_attention(c, items, 0, nullptr, cu_q[n], nullptr, num_q_heads, 1.0f, nullptr);
+    c->plan_rec = nullptr;
+    c->num_sms = saved_sms;
+    c->fail_after = saved_fail;
+    c->last_split = saved_plan[0];
+    c->last_splits = saved_plan[1];
+    c->last_ctas = saved_plan[2];
+    if (s != PE_OK) return s;
+    *n_words = static_cast<int64_t>(rec.size());
+    if (words) {
+        if (cap < *n_words) return fail(PE_ERR_RANGE, "the plan takes %lld words, cap is %lld",
+                                        static_cast<long long>(*n_words), static_cast<long long>(cap));
+        std::copy(rec.begin(), rec.end(), words);
+    }
     return PE_OK;
 }
 

@@ -239,3 +239,197 @@ def test_checker_rejects_broken_plans():
     broken(lambda p: p["ctas"][k].__setitem__(5, (p["ctas"][k][5] + 1) % p["slots"][p["ctas"][k][4]][1]))
     broken(lambda p: p["ctas"][k].__setitem__(4, -1))
     broken(lambda p: p["unit_tiles"].__setitem__(0, p["unit_tiles"][0] + 1))
+
+
+# ---------------------------------------------------------------- every launch of an attention call
+def q_tile_key_tiles(n, nq, g, qt):
+    """128-key tiles q-tile qt of a sequence of n keys whose last nq positions
+    are the queries sees: its last row sits at position n - nq + q_last."""
+    q_last = min((qt + 1) * (BM // g), nq) - 1
+    return -(-(n - nq + q_last + 1) // BN)
+
+
+def one_item_ctas(launch, hkv):
+    """(sequence index, kv-head, split, pair) of every CTA of a one-item launch,
+    decoded by the kernel's rules (stated with pe_attn_plan_launches)."""
+    seqs, ctas = launch["seqs"], launch["ctas"]
+    out = []
+    for b in range(ctas):
+        i = max(k for k, q in enumerate(seqs) if q["item0"] <= b)
+        q = seqs[i]
+        end = seqs[i + 1]["item0"] if i + 1 < len(seqs) else ctas
+        local, ns = b - q["item0"], q["n_splits"]
+        assert (end - q["item0"]) % (hkv * ns) == 0
+        if launch["pairs_fastest"]:
+            pairs = (end - q["item0"]) // (hkv * ns)
+            pair, split, kvh = q["pair_top"] - 1 - local % pairs, (local // pairs) % ns, local // pairs // ns
+        else:
+            kvh, split, pair = local % hkv, (local // hkv) % ns, q["pair_top"] - 1 - local // hkv // ns
+        out.append((i, kvh, split, pair))
+    return out
+
+
+def check_launches(plan, lens, nqs, seqs, g, hkv, d, ws_bytes, decode_rows_max):
+    by_seq = dict(zip(seqs, zip(lens, nqs)))
+    done = {}          # (seq, kv-head, q-tile) -> how it was computed
+    seen = {s: [] for s in seqs if by_seq[s][1] > 0}
+    for li, launch in enumerate(plan):
+        assert 1 <= len(launch["seqs"]) <= 64
+        for q in launch["seqs"]:
+            seen[q["seq"]].append(launch["kind"])
+            assert (q["n_keys"], q["n_q"]) == by_seq[q["seq"]]
+        if launch["kind"] == "decode":
+            for q in launch["seqs"]:
+                assert q["n_q"] * g <= decode_rows_max
+            continue
+        for q in launch["seqs"]:
+            assert q["n_q"] * g > decode_rows_max
+            assert q["n_qtiles"] == -(-q["n_q"] * g // BM)
+        if launch["kind"] == "persistent":
+            continue
+        split, st = launch["split"], launch["split_tiles"]
+        cover = {}
+        for i, kvh, sp, pair in one_item_ctas(launch, hkv):
+            q = launch["seqs"][i]
+            assert 0 <= kvh < hkv and 0 <= sp < q["n_splits"] and 0 <= pair < q["pair_top"]
+            assert 2 * pair < q["n_qtiles"]
+            for qt in (2 * pair, 2 * pair + 1):
+                if qt >= q["n_qtiles"]:
+                    continue
+                key = (q["seq"], kvh, qt)
+                cover.setdefault(key, []).append(sp)
+                if split:
+                    # every key tile the q-tile sees lies in one of the splits
+                    assert q["n_splits"] * st >= q_tile_key_tiles(q["n_keys"], q["n_q"], g, qt)
+        for key, sps in cover.items():
+            ns = launch["seqs"][[q["seq"] for q in launch["seqs"]].index(key[0])]["n_splits"]
+            assert sorted(sps) == list(range(ns)), (key, sps)     # each split once
+            assert key not in done, f"{key} computed twice"
+            done[key] = (li, split)
+        if not split:
+            assert launch["combine_rows"] == 0 and all(q["n_splits"] == 1 for q in launch["seqs"])
+            continue
+        # partial rows: each sequence's block in the workspace, disjoint; the combine reads what was written
+        blocks, comb = [], 0
+        for i, q in enumerate(launch["seqs"]):
+            n_qt = q["n_qtiles"] if launch["kind"] == "one_item" else min(q["n_qtiles"], 2 * q["pair_top"])
+            blocks.append((q["part_row0"], q["part_row0"] + n_qt * hkv * q["n_splits"] * BM))
+            assert q["comb0"] == comb
+            comb += n_qt * hkv * BM
+            for qt in range(n_qt):
+                for kvh in range(hkv):
+                    assert sorted(cover[(q["seq"], kvh, qt)]) == list(range(q["n_splits"]))
+        assert launch["combine_rows"] == comb
+        blocks.sort()
+        for a, b in zip(blocks, blocks[1:]):
+            assert a[1] <= b[0], blocks
+        assert blocks[-1][1] * (4 * d + 4) <= ws_bytes
+    for s, kinds in seen.items():
+        assert kinds in (["decode"], ["persistent"], ["one_item"], ["one_item", "one_item_tail"]), (s, kinds)
+        if kinds[0] in ("one_item",):
+            n, nq = by_seq[s]
+            for kvh in range(hkv):
+                for qt in range(-(-nq * g // BM)):
+                    assert (s, kvh, qt) in done, f"sequence {s} q-tile {qt} kv-head {kvh} never computed"
+
+
+def test_random_launch_plans():
+    rng = random.Random(4875)
+    kinds = {}
+    for _ in range(1200):
+        d = rng.choice([64, 128])
+        hkv = rng.choice([1, 2, 4, 8])
+        g = rng.choice([1, 2, 4, 8, 16])
+        n = rng.choice([1, 1, 1, 2, 3, 5, 16, 70])
+        lens, nqs = [], []
+        for _ in range(n):
+            length = rng.choice([rng.randint(1, 300), rng.randint(300, 4000), rng.randint(4000, 16384)])
+            if n > 16:
+                length = min(length, 3000)
+            lens.append(length)
+            nqs.append(rng.choice([0, 1, rng.randint(1, min(length, 64)), rng.randint(1, length)]))
+        sms = rng.choice([7, 37, 148, 152, 160])
+        ws = rng.choice([0, 1 << 20, 8 << 20])
+        c = pe.PagedKVCache(1, hkv, d, 16, 40000, max(n, 1), 1100, host_only=True, workspace_bytes=ws)
+        opts = {"splitkv": rng.choice([-1, -1, 0, 1]), "num_splits": rng.choice([0, 0, 0, rng.randint(1, 9)]),
+                "attn_kernel": rng.choice([1, 1, 0, 2]), "attn_order": rng.choice([-1, -1, 0, 1]),
+                "decode_kernel": rng.choice([1, 1, 0, 2])}
+        for k, v in opts.items():
+            c.set_option(k, v)
+        seqs = []
+        for length in lens:
+            s = c.seq_create()
+            c.append_kv(s, n_tokens=length)
+            seqs.append(s)
+        plan = c.plan_launches(seqs, nqs, g * hkv, num_sms=sms)
+        decodes = opts["decode_kernel"] and not (opts["decode_kernel"] == 1 and opts["splitkv"] == 0)
+        check_launches(plan, lens, nqs, seqs, g, hkv, d, ws or (256 << 20), 16 if decodes else 0)
+        for launch in plan:
+            k = (launch["kind"], launch["split"], launch["pairs_fastest"])
+            kinds[k] = kinds.get(k, 0) + 1
+        c.close()
+    # the plans span every launch kind, split and unsplit, in both CTA orders
+    for k in [("decode", False, False), ("persistent", False, False), ("persistent", True, False),
+              ("one_item", False, False), ("one_item", False, True), ("one_item", True, False),
+              ("one_item", True, True), ("one_item_tail", True, False)]:
+        assert kinds.get(k, 0) > 0, (k, kinds)
+
+
+def test_launch_plans_of_the_workloads():
+    """The configurations' own launch groups plan as measured: tau/T 0.7 with a
+    tail launch of 19 splits over 8 units, tau/T 0.9 and the short suffix on the
+    persistent kernel, the tiny launch in one pass of 8 CTAs, tau/T 0.5 in four
+    waves, the long suffix's 16384 CTAs pairs fastest."""
+    def plan_of(hkv, d, lens, nqs, hq, ps=16):
+        c = pe.PagedKVCache(1, hkv, d, ps, 40000, len(lens), 4100, host_only=True)
+        seqs = []
+        for n in lens:
+            s = c.seq_create()
+            c.append_kv(s, n_tokens=n)
+            seqs.append(s)
+        p = c.plan_launches(seqs, nqs, hq, num_sms=152)
+        check_launches(p, lens, nqs, seqs, hq // hkv, hkv, d, 256 << 20, 16)
+        return [(x["kind"], x["split"], x["ctas"], x["pairs_fastest"]) for x in p]
+
+    assert plan_of(8, 128, [16384], [4915], 32) == [("one_item", False, 608, False), ("one_item_tail", True, 152, False)]
+    assert plan_of(8, 128, [16384], [1638], 32)[0][0] == "persistent"
+    assert plan_of(8, 128, [32784] * 8, [16] * 8, 32)[0][0] == "persistent"
+    assert plan_of(8, 64, [640], [128], 8) == [("one_item", False, 8, False)]
+    assert plan_of(8, 128, [16384], [8192], 32) == [("one_item", False, 1024, False)]
+    lens = [20480] * 4
+    assert plan_of(8, 128, lens, [16384] * 4, 64, ps=64) == [("one_item", False, 16384, True)]
+
+
+def test_launch_checker_rejects_broken_plans():
+    """check_launches catches a lost split, a sequence boundary between CTAs
+    moved by one (kv-head x split) group, overlapping partial blocks, a combine
+    that misses rows, a sequence left out of every launch and splits too short
+    for the keys.  (The two CTA orders are both valid numberings of the same
+    work, so swapping them is not a mistake.)"""
+    import copy
+    c = pe.PagedKVCache(1, 8, 128, 16, 40000, 4, 4100, host_only=True)
+    c.set_option("splitkv", 1)
+    c.set_option("attn_kernel", 0)   # the one-item kernel with key splits
+    lens, nqs = [9000, 5000, 3000], [700, 300, 129]
+    seqs = []
+    for n in lens:
+        s = c.seq_create()
+        c.append_kv(s, n_tokens=n)
+        seqs.append(s)
+    plan = c.plan_launches(seqs, nqs, 32, num_sms=152)
+    args = (lens, nqs, seqs, 4, 8, 128, 256 << 20, 16)
+    check_launches(plan, *args)
+    assert [x["kind"] for x in plan] == ["one_item"] and plan[0]["split"] and len(plan[0]["seqs"]) == 3
+
+    def broken(edit):
+        p = copy.deepcopy(plan)
+        edit(p[0])
+        with pytest.raises(AssertionError):
+            check_launches(p, *args)
+
+    broken(lambda x: x["seqs"][0].__setitem__("n_splits", x["seqs"][0]["n_splits"] - 1))
+    broken(lambda x: x["seqs"][1].__setitem__("item0", x["seqs"][1]["item0"] + 16))
+    broken(lambda x: x["seqs"][1].__setitem__("part_row0", x["seqs"][1]["part_row0"] - BM))
+    broken(lambda x: x.__setitem__("combine_rows", x["combine_rows"] - BM))
+    broken(lambda x: x["seqs"].pop())
+    broken(lambda x: x.__setitem__("split_tiles", x["split_tiles"] - 1))
