@@ -433,3 +433,31 @@ def test_launch_checker_rejects_broken_plans():
     broken(lambda x: x.__setitem__("combine_rows", x["combine_rows"] - BM))
     broken(lambda x: x["seqs"].pop())
     broken(lambda x: x.__setitem__("split_tiles", x["split_tiles"] - 1))
+
+
+def test_persistent_launches_agree_with_the_persistent_plan():
+    """Where an attention call takes the persistent kernel, its launch record
+    and pe_attn_plan_persistent describe the same plan: the same sequences in
+    the same order and the same CTA count and cut units."""
+    rng = random.Random(99)
+    for _ in range(300):
+        hkv, g = rng.choice([1, 2, 8]), rng.choice([2, 4, 8])
+        n = rng.choice([1, 2, 4, 9])
+        lens = [rng.randint(200, 12000) for _ in range(n)]
+        nqs = [rng.randint(max(1, 17 // g + 1), min(x, 3000)) for x in lens]
+        c = pe.PagedKVCache(1, hkv, 128, 16, 40000, n, 1100, host_only=True)
+        c.set_option("attn_kernel", 2)
+        c.set_option("splitkv", rng.choice([-1, 1]))
+        seqs = []
+        for length in lens:
+            s = c.seq_create()
+            c.append_kv(s, n_tokens=length)
+            seqs.append(s)
+        sms = rng.choice([9, 152])
+        launches = c.plan_launches(seqs, nqs, g * hkv, num_sms=sms)
+        plan = c.plan_persistent(seqs, nqs, g * hkv, num_sms=sms)
+        assert [x["kind"] for x in launches] == ["persistent"]
+        rec = launches[0]
+        assert [q["seq"] for q in rec["seqs"]] == plan["order"]
+        assert rec["ctas"] == plan["n_ctas"] and rec["split"] == (plan["n_slots"] > 0)
+        c.close()
