@@ -325,3 +325,21 @@ def test_binding_rejects_tensors_off_the_cache_device():
     with pytest.raises(ValueError, match="cuda:1, the cache on cuda:0"):
         binding._dev_ptr(FakeCuda(), "Q", 0)
     assert binding._dev_ptr(FakeCuda(), "Q", 1).value is None  # same device: accepted
+
+
+def test_header_is_plain_c():
+    """include/pe.h is a C ABI: it compiles as strict C99 with no warnings,
+    so a C caller (no C++ compiler, no CUDA headers) can use it."""
+    import shutil
+    import subprocess
+    import tempfile
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    with tempfile.TemporaryDirectory() as tmp:
+        src = os.path.join(tmp, "use_pe.c")
+        with open(src, "w") as f:
+            f.write('#include "pe.h"\nint main(void) { pe_cache *c = 0; (void)c; return PE_OK; }\n')
+        r = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-fsyntax-only",
+                            "-I", os.path.join(ROOT, "include"), src], capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
